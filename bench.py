@@ -1,0 +1,409 @@
+#!/usr/bin/env python3
+"""Benchmark: the VGG-16 3x3 conv stack, batch 32, fp32, through libpatconv on one GB300 per rank.
+
+One step = the 13 pattern-pruned 3x3 convolutions (bias + ReLU fused) and the 5 2x2 max-pools
+between blocks, over one batch of 32 synthetic 3x224x224 images resident in HBM.  Keep ratio
+1.0 on the first layer and 0.3 on the others, 8-pattern library, seeded He-normal weights and
+N(0,1) images (the paper's trained networks and ImageNet images are not available).
+
+Prints one JSON line (rank 0).  `value` is images/s over all ranks (each rank runs its own
+batch: weak scaling, no collective in the data path).  Extra keys:
+  roofline      the dominant kernel (pconv_main) against the FP32 CUDA-core peak
+                (SMs x 128 lanes x 2 FLOP x max SM clock), from CUDA events around each of its
+                launches inside the timed region;
+  e2e           the same metric with the input batch copied from pinned host memory and the
+                final feature map copied back inside the timed region;
+  cpu_baseline  the float64 oracle timed on this host's cores on a bounded sample (rank 0, N=1).
+`--impl reference` times the oracle alone as the reference arm.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "pattern-sparse 3x3 conv useful GFLOP/s & % roofline; VGG-16 img/s at 1 GB300"
+BATCH = 32
+WORKLOAD = "vgg16_3x3_stack_b32"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=60)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0, help="oracle sample budget")
+    return ap.parse_args()
+
+
+def conv_cost(beta, cin, cout, h, w, ho, wo, n, G, es=4):
+    flops = 8.0 * beta * n * ho * wo
+    image = 4 * G * 8 + 8 * G * cin + 4 * (G * cin + 1) + 16 * beta
+    bytes_ = es * (n * cin * h * w + n * cout * ho * wo) + image + 4 * cout
+    return flops, float(bytes_)
+
+
+def config_dict():
+    return {"workload": WORKLOAD, "model": "VGG-16 (13 3x3 convs, 5 max-pools)", "batch": BATCH,
+            "global_batch": BATCH, "image": "3x224x224", "keep": "1.0 first layer, 0.3 others",
+            "patterns": "8 four-tap patterns", "io": "fp32",
+            "l2": "no flush: activations per layer up to 411 MB, larger than the 129 MB L2",
+            "pool": "pp_maxpool2x2 between blocks", "parallelism": "batch replicas"}
+
+
+# ------------------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *a):
+        self.lines = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+                out = ""
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        sm, mx, reasons = [], [], set()
+        for l in getattr(self, "lines", []):
+            parts = [p.strip() for p in l.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for name, v in zip(names, parts[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------------ oracle (CPU)
+
+def blas_threads():
+    """Threads of the BLAS numpy runs on (OpenBLAS queried directly), else the usable cores."""
+    try:
+        with open("/proc/self/maps") as f:
+            libs = {l.split()[-1] for l in f if "openblas" in l.lower() and l.split()[-1].startswith("/")}
+        for path in libs:
+            lib = ctypes.CDLL(path)
+            for fn in ("openblas_get_num_threads", "openblas_get_num_threads64_",
+                       "scipy_openblas_get_num_threads", "scipy_openblas_get_num_threads64_"):
+                if hasattr(lib, fn):
+                    return int(getattr(lib, fn)())
+    except Exception:
+        pass
+    return len(os.sched_getaffinity(0))
+
+
+def oracle_setup(max_images=8):
+    """Projected weights of the 13 layers (outside any timed region) and the sample images."""
+    from oracle import patterns as OP
+    from oracle import project as OPR
+    from paper_2003_06513_gb300 import workloads as WL
+    layers = WL.vgg16()
+    proj = [(OPR.project(WL.weights(L), OP.default8(), L.keep)["W_hat"], WL.bias(L)) for L in layers]
+    return layers, proj, WL.vgg16_image(max_images)
+
+
+def oracle_forward(layers, proj, x):
+    """One image batch through the stack: float64 conv over the projected weights + max-pool."""
+    import numpy as np
+    from oracle import conv as OC
+    x = x.astype(np.float64)
+    for L, (Wh, b) in zip(layers, proj):
+        x = OC.conv_ref(x, Wh, b, 1, True)
+        if L.pool_after:
+            x = OC.maxpool2x2(x)
+    return x
+
+
+def oracle_forward_images(budget_s, max_images=8):
+    """Images pushed through the oracle one at a time until ``budget_s`` elapses;
+    returns (images, seconds, threads)."""
+    layers, proj, imgs = oracle_setup(max_images)
+    t0 = time.perf_counter()
+    done = 0
+    while done < max_images:
+        oracle_forward(layers, proj, imgs[done:done + 1])
+        done += 1
+        if time.perf_counter() - t0 >= budget_s:
+            break
+    return done, time.perf_counter() - t0, blas_threads()
+
+
+def reference_arm(args, rank, world):
+    if rank != 0:
+        return
+    steps, warm = args.steps, args.warmup
+    per_step = []
+    n_img_total, t_total = 0, 0.0
+    threads = blas_threads()
+    # each step: one image through the whole stack (bounded sample of the batch-32 workload)
+    layers, proj, imgs = oracle_setup(1)
+    budget = 240.0
+    t_start = time.perf_counter()
+    k_done = 0
+    for k in range(warm + steps):
+        if time.perf_counter() - t_start > budget and k >= warm + 1:
+            break
+        t0 = time.perf_counter()
+        oracle_forward(layers, proj, imgs[:1])
+        dt = time.perf_counter() - t0
+        if k >= warm:
+            per_step.append(dt)
+            n_img_total += 1
+            t_total += dt
+            k_done += 1
+    value = n_img_total / t_total if t_total > 0 else 0.0
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "img/s",
+            "n_gpus": world, "steps": k_done, "warmup": warm,
+            "ms_per_step": 1e3 * t_total / max(k_done, 1), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": config_dict(),
+            "cpu_baseline": {"value": value, "unit": "img/s", "cores": threads, "kind": "oracle",
+                             "sample": "1 image through the 13-layer stack per step (numpy float64)"},
+            "e2e": {"value": value, "unit": "img/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------------------ our arm
+
+def fp32_peak(props, clocks):
+    """FP32 CUDA-core peak: SMs x 128 FMA lanes x 2 FLOP x max SM clock."""
+    mhz = None
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            mhz = float(json.load(f).get("sm_max_mhz"))
+    except Exception:
+        pass
+    if not mhz:
+        mhz = clocks.get("sm_max_mhz") or 2070.0
+    return props.multi_processor_count * 128 * 2 * mhz * 1e6, mhz
+
+
+def hbm_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"]) * 1e9, "measured"
+    except Exception:
+        return 6.8e12, "fallback"
+
+
+def traffic_record():
+    """Per-launch DRAM bytes of pconv_main from the committed ncu summary, or None when the
+    kernel source changed since the counters were taken."""
+    path = os.path.join(ROOT, "profiles", "pconv_main_vgg16_traffic.json")
+    src = os.path.join(ROOT, "paper_2003_06513_gb300", "csrc", "conv.cu")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+        with open(src, "rb") as f:
+            sha = hashlib.sha256(f.read()).hexdigest()
+        if rec.get("conv_cu_sha256") == sha:
+            return rec
+    except Exception:
+        pass
+    return None
+
+
+def our_arm(args, rank, world, local_rank):
+    import numpy as np
+    import torch
+    from paper_2003_06513_gb300 import api
+    from paper_2003_06513_gb300 import workloads as WL
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+
+    layers = WL.vgg16()
+    packed, biases, costs = [], [], []
+    shapes = []
+    h = 224
+    for L in layers:
+        lay = api.pp_pack(WL.weights(L), None, L.keep).bind(dev)
+        packed.append(lay)
+        biases.append(torch.from_numpy(WL.bias(L)).to(dev))
+        G = (L.cout + 7) // 8
+        costs.append(conv_cost(lay.beta, L.cin, L.cout, h, h, h, h, BATCH, G))
+        shapes.append((BATCH, L.cout, h, h))
+        if L.pool_after:
+            h //= 2
+    x0 = torch.from_numpy(WL.vgg16_image(BATCH)).to(dev)
+    big = max(int(np.prod(s)) for s in shapes)
+    bufA = torch.empty(big, dtype=torch.float32, device=dev)
+    bufB = torch.empty(big, dtype=torch.float32, device=dev)
+    out_final = torch.empty((BATCH, 512, 7, 7), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(x, ev=None):
+        cur = x
+        bufs = (bufA, bufB)
+        j = 0
+        for i, (L, lay, b) in enumerate(zip(layers, packed, biases)):
+            y = bufs[j].narrow(0, 0, int(np.prod(shapes[i]))).view(shapes[i])
+            j ^= 1
+            if ev is not None:
+                ev[i][0].record(stream)
+            lay.conv(cur, b, True, y, stream)
+            if ev is not None:
+                ev[i][1].record(stream)
+            cur = y
+            if L.pool_after:
+                ps = (BATCH, L.cout, shapes[i][2] // 2, shapes[i][3] // 2)
+                p = out_final if i == len(layers) - 1 else bufs[j].narrow(0, 0, int(np.prod(ps))).view(ps)
+                j ^= 1
+                api.pp_maxpool2x2(cur, p, stream)
+                cur = p
+        return cur
+
+    def barrier():
+        torch.cuda.synchronize(dev)
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    for _ in range(max(args.warmup, 3)):
+        step(x0)
+    barrier()
+
+    K = args.steps
+    launches_per_step = len(layers) + sum(1 for L in layers if L.pool_after)
+    evs = [[[torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)]
+            for _ in layers] for _ in range(K)]
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(dev.index) as clk:
+        barrier()
+        t0.record(stream)
+        for k in range(K):
+            step(x0, evs[k])
+        t1.record(stream)
+        barrier()
+    elapsed_ms = t0.elapsed_time(t1)
+    conv_ms = [[evs[k][i][0].elapsed_time(evs[k][i][1]) for i in range(len(layers))] for k in range(K)]
+
+    # e2e: input from pinned host memory and the final feature map back, inside the timed region
+    host_in = torch.from_numpy(WL.vgg16_image(BATCH)).pin_memory()
+    host_out = torch.empty((BATCH, 512, 7, 7), dtype=torch.float32).pin_memory()
+    x_dev = torch.empty_like(x0)
+    for _ in range(2):
+        x_dev.copy_(host_in, non_blocking=True)
+        host_out.copy_(step(x_dev), non_blocking=True)
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    Ke = max(1, K // 2)
+    e0.record(stream)
+    for _ in range(Ke):
+        x_dev.copy_(host_in, non_blocking=True)
+        host_out.copy_(step(x_dev), non_blocking=True)
+    e1.record(stream)
+    barrier()
+    e2e_ms = e0.elapsed_time(e1) / Ke
+
+    t = torch.tensor([elapsed_ms, e2e_ms], device=dev, dtype=torch.float64)
+    if dist is not None:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    elapsed_ms, e2e_ms = float(t[0]), float(t[1])
+
+    if rank == 0:
+        props = torch.cuda.get_device_properties(dev)
+        clocks = clk.summary()
+        peak, mhz = fp32_peak(props, clocks)
+        hbm, hbm_kind = hbm_peak()
+        flops = [c[0] for c in costs]
+        bytes_ = [c[1] for c in costs]
+        per_layer_ms = [statistics.median(conv_ms[k][i] for k in range(K)) for i in range(len(layers))]
+        tot_conv_ms = sum(statistics.mean(conv_ms[k][i] for k in range(K)) for i in range(len(layers)))
+        achieved = sum(flops) / (tot_conv_ms * 1e-3)
+        roof_ms = sum(max(f / peak, b / hbm) for f, b in zip(flops, bytes_)) * 1e3
+        ms_step = elapsed_ms / K
+        img_s = world * BATCH / (ms_step * 1e-3)
+        trec = traffic_record()
+        line = {
+            "metric": METRIC, "value": img_s, "unit": "img/s", "n_gpus": world, "steps": K,
+            "warmup": max(args.warmup, 3), "ms_per_step": ms_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic (seeded He-normal weights, N(0,1) images)",
+            "config": config_dict(),
+            "useful_gflops": world * sum(flops) / (ms_step * 1e-3) / 1e9,
+            "network_roofline_frac": roof_ms / tot_conv_ms,
+            "roofline": {"bound": "alu", "kernel": "pconv_main<S=1,4x4,f32>",
+                         "achieved": achieved / 1e12, "peak": peak / 1e12, "unit": "TFLOP/s",
+                         "frac": achieved / peak,
+                         "peak_basis": f"{props.multi_processor_count} SMs x 128 FP32 lanes x 2 x {mhz:.0f} MHz",
+                         "traffic": (trec or {}).get("dram_bytes_per_launch"),
+                         "algorithmic_bytes_per_launch": sum(bytes_) / len(bytes_),
+                         "hbm_peak_gbs": hbm / 1e9, "hbm_peak_kind": hbm_kind},
+            "per_layer_ms": [round(v, 4) for v in per_layer_ms],
+            "e2e": {"value": world * BATCH / (e2e_ms * 1e-3), "unit": "img/s",
+                    "h2d_bytes_per_step": int(host_in.numel() * 4),
+                    "d2h_bytes_per_step": int(host_out.numel() * 4)},
+            "gpu_launches": K * launches_per_step,
+            "clocks": clocks,
+        }
+        if world == 1 and not args.no_cpu_baseline:
+            n, dt, thr = oracle_forward_images(args.cpu_seconds, max_images=BATCH)
+            line["cpu_baseline"] = {"value": n / dt, "unit": "img/s", "cores": thr, "kind": "oracle",
+                                    "sample": f"{n} image(s) through the 13-layer stack, numpy float64"}
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        reference_arm(args, rank, world)
+        return
+    our_arm(args, rank, world, local_rank)
+
+
+if __name__ == "__main__":
+    main()

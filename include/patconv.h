@@ -1,0 +1,146 @@
+/*
+ * patconv.h -- C ABI of libpatconv: pattern-pruned 3x3 convolution inference on one GB300.
+ *
+ * Method (arXiv 2003.06513):
+ *   - kernel pattern pruning (§3.2): every kept 3x3 kernel keeps exactly 4 weights whose
+ *     positions form one pattern of a small library P = {M_1..M_m} (§4.2, m = 6..8);
+ *   - the projection onto that constraint set keeps, per kernel, the pattern whose pruned kernel
+ *     has the largest Frobenius norm (§4.3, Eq. 5-6);
+ *   - connectivity pruning (§4.4) keeps at most beta kernels per layer;
+ *   - the compiler-level passes (§3.4) group filters of similar pattern sequence ("filter kernel
+ *     reorder") and store the kept weights compactly ("compressed weight storage");
+ *   - the layer computes X_n = sigma(W_n X_{n-1} + b_n) (§4.1, Eq. 1) with sigma = ReLU or
+ *     identity, as a 3x3 convolution with zero padding 1.
+ *
+ * Conventions shared by every entry point:
+ *   - every function returns a pp_status (0 = PP_OK, negative = error); no exception, abort or
+ *     device synchronisation crosses the ABI; out-parameters are written only on PP_OK;
+ *   - the library owns host memory only (the handle).  Device memory and streams belong to the
+ *     caller; streams are passed as `void*` holding a cudaStream_t (NULL = legacy default);
+ *   - taps are numbered in raster order t = 3*(dy+1) + (dx+1), dy, dx in {-1,0,1}; a pattern is
+ *     a 9-bit mask with bit t set for each kept tap;
+ *   - tensors are contiguous NCHW; weights are host fp32 [Cout][Cin/groups][3][3].
+ *
+ * Thread safety: a handle is immutable after pp_pack/pp_bind_device, so pp_conv on one handle
+ * may be called from several host threads and streams at once.
+ */
+#ifndef PATCONV_H
+#define PATCONV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct pp_layer* pp_handle;
+
+typedef enum {
+    PP_OK = 0,
+    PP_ERR_NULL = -1,         /* a required pointer is NULL                                  */
+    PP_ERR_SHAPE = -2,        /* a size is out of range or inconsistent                      */
+    PP_ERR_PATTERN = -3,      /* pattern library invalid (count, popcount, duplicates)       */
+    PP_ERR_KEEP = -4,         /* keep ratio outside (0, 1] or NaN                            */
+    PP_ERR_NONFINITE = -5,    /* a weight is NaN or infinite                                 */
+    PP_ERR_ALIGN = -6,        /* a device pointer is not aligned as documented               */
+    PP_ERR_DTYPE = -7,        /* unknown pp_dtype                                            */
+    PP_ERR_NOT_BOUND = -8,    /* pp_conv before pp_bind_device                               */
+    PP_ERR_BUFFER = -9,       /* caller buffer too small / wrong size, or x and y overlap     */
+    PP_ERR_CUDA = -10,        /* a CUDA runtime call failed (launch or copy)                 */
+    PP_ERR_ARG = -11,         /* any other invalid argument (section, query key, flag)       */
+    PP_ERR_ALLOC = -12        /* host allocation failed                                      */
+} pp_status;
+
+typedef enum { PP_F32 = 0, PP_F16 = 1 } pp_dtype;
+
+/* Sections of a packed layer (pp_export).  Byte layouts:
+ *   HEADER u32[16]: 'PPK1' (0x314B5050), version 1, Cout, Cin_g, groups, stride, n_patterns,
+ *                   beta, F (= 8), G = ceil(Cout/8), masks two per word (low half first), 0, 0
+ *   PID    i8 [Cout][Cin_g]   pattern index of each kernel, -1 = pruned (original order)
+ *   PERM   u32[G*8]           original filter of each slot, 0xFFFFFFFF = padding slot
+ *   DESC   u64[G][Cin_g]      bits 0-3: kept kernels c of group g at input channel ci; entry
+ *                             j < c at bits 4+6j..9+6j = (slot << 3) | pattern, slots ascending
+ *   KOFS   u32[G*Cin_g + 1]   kept kernels before (g, ci) in (g, ci, slot) order; last = beta
+ *   VALS   f32[beta][4]       kept weights in (g, ci, slot) order, taps ascending (bit copies)
+ *   DENSE  f32[Cout][Cin_g][9] projected weights with zeros in place
+ *   IMAGE  the device image: PERM | DESC | KOFS | VALS, each starting at a multiple of 256 B.
+ * Filter slot order (filter kernel reorder, §3.4): filters sorted by kept count descending, then
+ * by their pattern-index sequence over ci (pruned = 15) ascending, then by original index. */
+typedef enum {
+    PP_SEC_HEADER = 0, PP_SEC_PID = 1, PP_SEC_PERM = 2, PP_SEC_DESC = 3,
+    PP_SEC_KOFS = 4, PP_SEC_VALS = 5, PP_SEC_DENSE = 6, PP_SEC_IMAGE = 7
+} pp_section;
+
+typedef enum {
+    PP_Q_BETA = 0, PP_Q_COUT = 1, PP_Q_CIN_G = 2, PP_Q_GROUPS = 3, PP_Q_STRIDE = 4,
+    PP_Q_N_GROUPS = 5, PP_Q_N_PATTERNS = 6, PP_Q_IMAGE_BYTES = 7,
+    PP_Q_FAST_PATH = 8,       /* 1 if the library equals pp_default_patterns (compiled bodies)  */
+    PP_Q_SECTION_BYTES = 16   /* + section id: byte size of that section                      */
+} pp_query_key;
+
+/* The 8-pattern library the fast kernels are compiled for (§3.2, §4.2): indices 0-3 keep the
+ * centre and three of the four edge neighbours (dropping up, left, right, down in turn);
+ * indices 4-7 keep the centre, one edge neighbour (up, left, right, down) and the two corners
+ * flanking it.  Writes min(capacity, 8) masks to `masks` and returns 8 (or a negative status
+ * if masks is NULL with capacity > 0). */
+int pp_default_patterns(uint16_t* masks, int capacity);
+
+/* Pattern projection (§4.3 Eq. 6), connectivity pruning (§4.4) and packing (§3.4) of one layer.
+ *   W        host fp32 [Cout][Cin/groups][3][3], read only, caller-owned;
+ *   groups   1 (dense) or Cout == Cin (depthwise);
+ *   stride   1 or 2 (padding is always 1);
+ *   masks    n_patterns 9-bit masks, 1 <= n_patterns <= 8, each with exactly 4 bits, distinct;
+ *   keep     connectivity keep ratio in (0, 1]: beta = floor(keep * Cout * Cin_g + 0.5) in
+ *            float64, clamped to [1, Cout*Cin_g]; the beta kernels with the largest retained
+ *            energy survive, ties to the lower flat index co*Cin_g + ci;
+ * Projection scores are float64 sums ((a^2 + b^2) + c^2) + d^2 over the pattern's taps in
+ * ascending order; ties go to the lowest pattern index.  Host-only: touches no GPU.
+ * Errors: PP_ERR_NULL, PP_ERR_SHAPE, PP_ERR_PATTERN, PP_ERR_KEEP, PP_ERR_NONFINITE,
+ * PP_ERR_ALLOC.  On success *out owns host memory released by pp_destroy. */
+int pp_pack(const float* W, int Cout, int Cin, int groups, int stride,
+            const uint16_t* masks, int n_patterns, double keep, pp_handle* out);
+
+/* Read one scalar property (pp_query_key) of a packed layer. */
+int pp_query(pp_handle h, int key, int64_t* value);
+
+/* Copy one section (pp_section) into host memory; `bytes` must equal its size exactly
+ * (PP_Q_SECTION_BYTES + section), else PP_ERR_BUFFER. */
+int pp_export(pp_handle h, int section, void* host_dst, size_t bytes);
+
+/* Upload the device image into caller-owned DEVICE memory `dev_image` (>= PP_Q_IMAGE_BYTES
+ * bytes, 256-byte aligned) with an asynchronous host-to-device copy on `stream`, and remember
+ * the pointer for pp_conv.  The caller keeps the memory alive (and unmodified) while the handle
+ * is used, and must order the copy before the first pp_conv (same stream, or an event).
+ * Errors: PP_ERR_NULL, PP_ERR_BUFFER (too small), PP_ERR_ALIGN, PP_ERR_CUDA. */
+int pp_bind_device(pp_handle h, void* dev_image, size_t bytes, void* stream);
+
+/* y = sigma(conv3x3(x, W_hat, stride, pad 1) + bias) on the GPU, enqueued on `stream`.
+ *   x     DEVICE [N][Cin][H][W] of `dtype` (PP_F32 or PP_F16);
+ *   y     DEVICE [N][Cout][Ho][Wo] of the same dtype, Ho = (H-1)/stride + 1 (likewise Wo);
+ *         must not overlap x;
+ *   bias  DEVICE fp32 [Cout] or NULL (no bias);  relu 0 or 1.
+ * Accumulation is fp32 (FFMA on the CUDA cores) in input-channel order; fp16 inputs are
+ * widened exactly and the fp16 output is rounded to nearest even.  Pointers need only element
+ * alignment; 16-byte aligned x/y with W % 4 == 0 take the vector paths.  N == 0 is a no-op.
+ * Validation errors return before any launch; a failed launch returns PP_ERR_CUDA.  Never
+ * synchronises. */
+int pp_conv(pp_handle h, const void* x, int dtype, int N, int H, int W,
+            const float* bias, int relu, void* y, void* stream);
+
+/* 2x2 max-pool, stride 2, floor mode: y[n,c,i,j] = max x[n,c,2i+a,2j+b] (a,b in {0,1}).
+ * The pooling between VGG blocks; x DEVICE [N][C][H][W], y DEVICE [N][C][H/2][W/2], same dtype,
+ * no overlap.  Enqueue only. */
+int pp_maxpool2x2(const void* x, int dtype, int N, int C, int H, int W, void* y, void* stream);
+
+/* Release the handle's host memory (the bound device image stays the caller's).  NULL is OK. */
+int pp_destroy(pp_handle h);
+
+/* Static English text for a status code. */
+const char* pp_status_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PATCONV_H */

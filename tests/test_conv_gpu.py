@@ -1,0 +1,206 @@
+"""GPU parity of pp_conv / pp_maxpool2x2 with the float64 oracle (§4.1 Eq. 1 over the projected
+weights of §4.3 Eq. 6 and §4.4).
+
+Error metric: |y_gpu - y_ref| / (sum |W_hat| |x| + |b| + 2^-1000) per output, max over outputs;
+bar 1e-4 for fp32 I/O and 2e-3 for fp16 I/O.  The oracle projects the weights itself: nothing
+it uses comes from the CUDA path.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import conv as OC
+from oracle import patterns as OP
+from oracle import project as OPR
+from paper_2003_06513_gb300 import api
+from paper_2003_06513_gb300 import workloads as WL
+
+pytestmark = pytest.mark.gpu
+
+TOL = {torch.float32: 1e-4, torch.float16: 2e-3}
+
+
+def _np_dt(dt):
+    return np.float32 if dt == torch.float32 else np.float16
+
+
+def run_gpu(W, x, b, keep, stride=1, relu=True, depthwise=False, dtype=torch.float32, masks=None,
+            guard=0, to_host=True):
+    """Pack + bind + pp_conv; x host array; returns the output (host float64 unless
+    ``to_host=False``) and the layer."""
+    layer = api.pp_pack(W, masks, keep, W.shape[0] if depthwise else 1, stride)
+    dev = torch.device("cuda")
+    layer.bind(dev)
+    xt = torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+    bt = None if b is None else torch.from_numpy(b).to(dev)
+    shape = layer.out_shape(x.shape)
+    n = int(np.prod(shape))
+    if guard:
+        buf = torch.full((n + 2 * guard,), float("nan"), dtype=dtype, device=dev)
+        y = buf[guard:guard + n].view(shape)
+    else:
+        y = torch.empty(shape, dtype=dtype, device=dev)
+    layer.conv(xt, bt, relu, y)
+    torch.cuda.synchronize()
+    if guard:
+        g = torch.cat([buf[:guard], buf[guard + n:]])
+        assert torch.isnan(g).all(), "pp_conv wrote outside its output tensor"
+    return (y.double().cpu().numpy() if to_host else y), layer
+
+
+def oracle(W, x, b, keep, stride=1, relu=True, depthwise=False, masks=None):
+    masks = OP.default8() if masks is None else masks
+    Wh = OPR.project(W, masks, keep)["W_hat"]
+    ref = OC.conv_ref(x.astype(np.float64), Wh, b, stride, relu, depthwise)
+    den = OC.denominator(x.astype(np.float64), Wh, b, stride, depthwise)
+    return ref, den
+
+
+def check(W, x, b, keep, stride=1, relu=True, depthwise=False, dtype=torch.float32, masks=None,
+          guard=64):
+    y, layer = run_gpu(W, x, b, keep, stride, relu, depthwise, dtype, masks, guard)
+    ref, den = oracle(W, x, b, keep, stride, relu, depthwise, masks)
+    err = OC.max_norm_err(y, ref, den)
+    assert err <= TOL[dtype], f"normalised error {err:.3e} > {TOL[dtype]}"
+    return y, err
+
+
+def rnd(shape, seed, relu=False, dtype=np.float32):
+    return WL.activations(shape, seed, relu=relu, dtype=dtype)
+
+
+# --------------------------------------------------------------------------- single layer
+
+def test_single_layer_workload():
+    L = WL.single_layer()
+    x = WL.layer_input(L, 1)
+    check(WL.weights(L), x, WL.bias(L), L.keep)
+
+
+@pytest.mark.parametrize("N,Cin,Cout,H,W,keep,stride", [
+    (1, 3, 5, 7, 7, 1.0, 1), (2, 16, 13, 13, 11, 0.5, 1), (1, 1, 1, 1, 1, 1.0, 1),
+    (3, 5, 9, 1, 9, 0.7, 1), (1, 64, 24, 9, 13, 0.3, 1), (2, 8, 8, 15, 15, 0.5, 2),
+    (1, 20, 17, 14, 14, 0.4, 2), (1, 3, 64, 2, 2, 1.0, 2), (4, 33, 40, 6, 5, 0.25, 1),
+    (1, 130, 16, 8, 8, 0.6, 1), (2, 48, 72, 28, 28, 0.3, 1), (1, 16, 16, 17, 31, 0.5, 2)])
+def test_shapes_fp32(N, Cin, Cout, H, W, keep, stride):
+    rng = np.random.default_rng(N * 1000 + Cin * 10 + H)
+    Wt = (rng.standard_normal((Cout, Cin, 3, 3)) * np.sqrt(2 / (9 * Cin))).astype(np.float32)
+    x = rnd((N, Cin, H, W), Cin + H)
+    b = (rng.standard_normal(Cout) * 0.1).astype(np.float32)
+    check(Wt, x, b, keep, stride)
+
+
+@pytest.mark.parametrize("stride", [1, 2])
+def test_fp16_io(stride):
+    rng = np.random.default_rng(5)
+    Wt = (rng.standard_normal((24, 40, 3, 3)) * np.sqrt(2 / 360)).astype(np.float32)
+    x = rnd((2, 40, 18, 20), 6, dtype=np.float16)
+    b = (rng.standard_normal(24) * 0.1).astype(np.float32)
+    check(Wt, x, b, 0.5, stride, dtype=torch.float16)
+
+
+def test_no_bias_no_relu_and_degenerate_keep():
+    rng = np.random.default_rng(8)
+    Wt = rng.standard_normal((12, 10, 3, 3)).astype(np.float32)
+    x = rnd((2, 10, 9, 9), 9)
+    check(Wt, x, None, 0.5, relu=False)
+    # beta = 1: a single kernel survives; every other filter outputs ReLU(bias)
+    b = (rng.standard_normal(12) * 0.1).astype(np.float32)
+    y, _ = check(Wt, x, b, 1e-9)
+    r = OPR.project(Wt, OP.default8(), 1e-9)
+    for co in range(12):
+        if (r["pid"][co] < 0).all():
+            assert np.all(y[:, co] == max(float(b[co]), 0.0))
+
+
+def test_other_pattern_library_generic_path():
+    masks = [OP.mask_of(t) for t in ([0, 4, 5, 8], [1, 4, 6, 7], [2, 3, 4, 8], [0, 1, 4, 7],
+                                     [3, 4, 7, 8], [1, 2, 4, 6])]
+    rng = np.random.default_rng(10)
+    Wt = rng.standard_normal((11, 7, 3, 3)).astype(np.float32)
+    x = rnd((2, 7, 10, 9), 11)
+    b = rng.standard_normal(11).astype(np.float32)
+    for stride in (1, 2):
+        check(Wt, x, b, 0.6, stride, masks=masks)
+    Wd = rng.standard_normal((9, 1, 3, 3)).astype(np.float32)
+    check(Wd, rnd((2, 9, 8, 8), 12), b[:9], 1.0, 1, depthwise=True, masks=masks)
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.float16])
+@pytest.mark.parametrize("stride", [1, 2])
+def test_depthwise(dtype, stride):
+    rng = np.random.default_rng(13)
+    C = 21
+    Wd = (rng.standard_normal((C, 1, 3, 3)) * np.sqrt(2 / 9)).astype(np.float32)
+    x = rnd((3, C, 13, 12), 14, dtype=_np_dt(dtype))
+    b = (rng.standard_normal(C) * 0.1).astype(np.float32)
+    check(Wd, x, b, 1.0, stride, depthwise=True, dtype=dtype)
+    check(Wd, x, b, 0.5, stride, depthwise=True, dtype=dtype)     # pruned channels -> sigma(b)
+
+
+def test_deterministic_and_zero_batch():
+    L = WL.single_layer()
+    x = WL.layer_input(L, 2)
+    y1, layer = run_gpu(WL.weights(L), x, WL.bias(L), L.keep)
+    y2, _ = run_gpu(WL.weights(L), x, WL.bias(L), L.keep)
+    assert np.array_equal(y1, y2)
+    xt = torch.empty((0, 64, 32, 32), device="cuda")
+    out = layer.conv(xt, None, True)
+    assert out.shape == (0, 64, 32, 32)
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.float16])
+def test_maxpool_exact(dtype):
+    x = rnd((3, 5, 14, 15), 15, dtype=_np_dt(dtype))
+    y = api.pp_maxpool2x2(torch.from_numpy(x).cuda())
+    assert np.array_equal(y.cpu().numpy(), OC.maxpool2x2(x))
+
+
+# --------------------------------------------------------------------------- workloads
+
+def _sampled_check(L, n, dtype=torch.float32, samples=(0, -1)):
+    """Full-batch launch (the benchmark's launch configuration), oracle on sampled images."""
+    x = WL.layer_input(L, n, relu=not L.depthwise, dtype=_np_dt(dtype))
+    W, b = WL.weights(L), WL.bias(L)
+    y, _ = run_gpu(W, x, b, L.keep, L.stride, True, L.depthwise, dtype, guard=256, to_host=False)
+    assert bool(torch.isfinite(y).all())
+    idx = [s % n for s in samples]
+    ref, den = oracle(W, x[idx], b, L.keep, L.stride, True, L.depthwise)
+    err = OC.max_norm_err(y[idx].double().cpu().numpy(), ref, den)
+    assert err <= TOL[dtype], f"{L.name}: normalised error {err:.3e}"
+
+
+@pytest.mark.parametrize("idx", range(13))
+def test_vgg16_layer_batch32(idx):
+    _sampled_check(WL.vgg16()[idx], 32)
+
+
+@pytest.mark.parametrize("idx", range(16))
+def test_resnet50_layer_batch64(idx):
+    _sampled_check(WL.resnet50_3x3()[idx], 64)
+
+
+@pytest.mark.parametrize("idx", range(17))
+def test_mobilenet_dw_layer_batch128_fp16(idx):
+    _sampled_check(WL.mobilenet_v2_dw()[idx], 128, torch.float16)
+
+
+def test_vgg16_chained_network():
+    """The whole 13-layer stack with the library's max-pool between blocks, batch 2; every
+    layer is checked on the exact input the GPU layer received."""
+    layers = WL.vgg16()
+    x = torch.from_numpy(WL.vgg16_image(2)).cuda()
+    for L in layers:
+        W, b = WL.weights(L), WL.bias(L)
+        layer = api.pp_pack(W, None, L.keep).bind("cuda")
+        y = layer.conv(x, torch.from_numpy(b).cuda(), True)
+        torch.cuda.synchronize()
+        xin = x.cpu().numpy()
+        ref, den = oracle(W, xin, b, L.keep)
+        err = OC.max_norm_err(y.double().cpu().numpy(), ref, den)
+        assert err <= 1e-4, f"{L.name}: {err:.3e}"
+        if L.pool_after:
+            p = api.pp_maxpool2x2(y)
+            assert np.array_equal(p.cpu().numpy(), OC.maxpool2x2(y.cpu().numpy()))
+            y = p
+        x = y
