@@ -133,6 +133,14 @@ int pp_conv(pp_handle h, const void* x, int dtype, int N, int H, int W,
  * no overlap.  Enqueue only. */
 int pp_maxpool2x2(const void* x, int dtype, int N, int C, int H, int W, void* y, void* stream);
 
+/* Device status word of the conv kernels on the current device.  A kernel whose pipeline wait
+ * runs out of time (about one second; it never happens in a correct run) records a bit here and
+ * returns early instead of hanging: 1 = data stage never arrived, 2 = stage never released,
+ * 4 = copies still in flight at exit.  *status gets the word; clear != 0 resets it.  Synchronous
+ * (a device-to-host copy); call it between launches, e.g. at the end of a test.
+ * Errors: PP_ERR_NULL, PP_ERR_CUDA. */
+int pp_device_status(int clear, unsigned int* status);
+
 /* Release the handle's host memory (the bound device image stays the caller's).  NULL is OK. */
 int pp_destroy(pp_handle h);
 

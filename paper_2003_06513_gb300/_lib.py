@@ -26,6 +26,7 @@ SIGNATURES = {
                          _c_void_p, _c_void_p]),
     "pp_maxpool2x2": (_c_int, [_c_void_p, _c_int, _c_int, _c_int, _c_int, _c_int, _c_void_p,
                                _c_void_p]),
+    "pp_device_status": (_c_int, [_c_int, ctypes.POINTER(ctypes.c_uint)]),
     "pp_destroy": (_c_int, [_c_void_p]),
     "pp_status_string": (ctypes.c_char_p, [_c_int]),
 }

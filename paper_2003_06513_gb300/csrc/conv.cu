@@ -17,12 +17,15 @@
 //     original channel of each slot.
 // The path is a gathered sparse contraction, so it runs on the CUDA-core FFMA pipe.
 #include <cuda_fp16.h>
+#include <cuda.h>
 #include <cuda_runtime.h>
+#include <cudaTypedefs.h>
 
 #include <algorithm>
 #include <atomic>
 #include <climits>
 #include <cstdint>
+#include <cstring>
 
 #include "../../include/patconv.h"
 #include "layer.h"
@@ -47,45 +50,21 @@ __host__ __device__ constexpr int ktap(int p, int k) {
     return -1;
 }
 
-constexpr int kThreads = 256;   // 8 warps = 8 filter groups per CTA
-constexpr int kWarps = kThreads / 32;
-constexpr int kMaxBoundaries = 80;  // chunk boundaries cached per warp (C <= 79*CK)
-
-struct MainParams {
-    const void* x;
-    void* y;
-    const float* bias;
-    const uint32_t* perm;
-    const uint64_t* desc;
-    const uint32_t* kofs;
-    const float4* vals;
-    int N, C, H, W, Cout, Ho, Wo, G, relu;
-    int BY, BX, NB;                   // spatial tile: BY x BX blocks of NB images
-    int tiles_x, tiles_y, tiles_n, n_fchunks;
-    int CK, n_chunks;                 // input channels per pipeline stage, number of stages run
-    int IH, IW, pitch;                // staged rows / cols per (channel, image), row pitch
-    int vec_store;                    // y rows allow RX-wide vector stores
-    int stage_floats;                 // input floats per stage
-};
-
 // ------------------------------------------------------------------------------ helpers
 
 __device__ __forceinline__ void cp_async4(void* smem, const void* gmem, bool valid) {
     const unsigned s = (unsigned)__cvta_generic_to_shared(smem);
     const int n = valid ? 4 : 0;
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(s), "l"(gmem), "r"(n));
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(s), "l"(gmem), "r"(n) : "memory");
 }
 __device__ __forceinline__ void cp_async8(void* smem, const void* gmem) {
     const unsigned s = (unsigned)__cvta_generic_to_shared(smem);
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(s), "l"(gmem));
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(s), "l"(gmem) : "memory");
 }
 __device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
     const unsigned s = (unsigned)__cvta_generic_to_shared(smem);
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(s), "l"(gmem));
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(s), "l"(gmem) : "memory");
 }
-__device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;\n" ::); }
-template <int N>
-__device__ __forceinline__ void cp_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N)); }
 
 template <typename T>
 __device__ __forceinline__ float to_f32(T v);
@@ -103,94 +82,233 @@ __device__ __forceinline__ __half from_f32<__half>(float v) { return __float2hal
 
 // ------------------------------------------------------------------------------ main kernel
 
-template <int S, int RY, int RX>
-struct Win {
-    static constexpr int WY = (RY - 1) * S + 3;
-    static constexpr int WX = (RX - 1) * S + 3;
+constexpr int kCompute = 16;                       // warps per CTA (filter groups x spatial)
+constexpr int kThreadsTM = kCompute * 32;
+constexpr int kStages = 3;                         // input-channel pipeline depth
+constexpr int kMaxChunks = 256;                    // input-channel stages per CTA
+constexpr long long kTimeoutCycles = 2000000000LL; // about one second of SM clock
+constexpr uint32_t kTmemCols = 512;                // 16 warps x 8 slots x 16 accumulators
+
+// Device status word: a wait that ran out of time records its code here and the kernel returns
+// early instead of hanging (read back by pp_device_status).
+__device__ unsigned int g_pp_status;
+enum : unsigned { kStatusFullTimeout = 1u, kStatusDrainTimeout = 4u };
+
+struct TmParams {
+    const void* x;
+    void* y;
+    const float* bias;
+    const uint32_t* perm;
+    const uint64_t* desc;
+    const uint32_t* kofs;
+    const float4* vals;
+    unsigned* status;
+    int N, C, H, W, Cout, Ho, Wo, G, relu;
+    int WG, WS;                        // filter groups x spatial warps per CTA (WG * WS = 16)
+    int BY, BX, NB;                    // spatial tile: BY x BX blocks (4x4 outputs) of NB images
+    int tiles_x, tiles_y, tiles_n, n_fchunks;
+    int CK, n_chunks, maxk;            // channels per stage, stages, max kept kernels per group-stage
+    int IH, BWb;                       // staged rows / row width (floats) per (image, channel)
+    int use_tma, vec_store;
+    unsigned tma_bytes;                // bytes one TMA box delivers
+    unsigned kb_off, stage_off, stage_bytes, desc_off, vals_off;   // shared-memory layout
 };
 
-// acc[F_][*] += the pattern-P_ kernel (weights w) applied to the lane's input window.
-template <int F_, int P_, int S, int RY, int RX, int WY, int WX>
-__device__ __forceinline__ void fma_pattern(float (&acc)[kF][RY * RX], const float (&win)[WY][WX],
-                                            const float4& w) {
-    constexpr int t0 = ktap(P_, 0), t1 = ktap(P_, 1), t2 = ktap(P_, 2), t3 = ktap(P_, 3);
-#pragma unroll
-    for (int r = 0; r < RY; ++r) {
-#pragma unroll
-        for (int c = 0; c < RX; ++c) {
-            float a = acc[F_][r * RX + c];
-            a = fmaf(w.x, win[r * S + t0 / 3][c * S + t0 % 3], a);
-            a = fmaf(w.y, win[r * S + t1 / 3][c * S + t1 % 3], a);
-            a = fmaf(w.z, win[r * S + t2 / 3][c * S + t2 % 3], a);
-            a = fmaf(w.w, win[r * S + t3 / 3][c * S + t3 % 3], a);
-            acc[F_][r * RX + c] = a;
+__device__ __forceinline__ uint32_t smem_u32(const void* ptr) {
+    return (uint32_t)__cvta_generic_to_shared(ptr);
+}
+__device__ __forceinline__ void mbar_init(uint32_t a, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(a), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t a, uint32_t tx) {
+    asm volatile("mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(a), "r"(tx) : "memory");
+}
+// arrives on the barrier once every cp.async this thread issued so far has landed
+__device__ __forceinline__ void cp_async_arrive(uint32_t a) {
+    asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(a) : "memory");
+}
+// Bounded wait for the completion of the phase with the given parity.
+__device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity, unsigned* status, unsigned code) {
+    const long long t0 = clock64();
+    while (true) {
+        uint32_t done;
+        asm volatile(
+            "{\n\t.reg .pred P;\n\t"
+            "mbarrier.try_wait.parity.shared::cta.b64 P, [%1], %2;\n\t"
+            "selp.u32 %0, 1, 0, P;\n\t}"
+            : "=r"(done) : "r"(a), "r"(parity) : "memory");
+        if (done) return true;
+        if (clock64() - t0 > kTimeoutCycles) {
+            atomicOr(status, code);
+            return false;
         }
     }
 }
-
-#define PP_CASE(F_, P_)                                                        \
-    case ((F_) << 3) | (P_):                                                   \
-        fma_pattern<F_, P_, S, RY, RX, WY, WX>(acc, win, w);                   \
-        break;
-#define PP_CASES(F_) \
-    PP_CASE(F_, 0) PP_CASE(F_, 1) PP_CASE(F_, 2) PP_CASE(F_, 3) PP_CASE(F_, 4) PP_CASE(F_, 5) PP_CASE(F_, 6) PP_CASE(F_, 7)
-
-template <int S, int RY, int RX, int WY, int WX>
-__device__ __forceinline__ void dispatch(int code, const float4& w, float (&acc)[kF][RY * RX],
-                                         const float (&win)[WY][WX]) {
-    switch (code) {
-        PP_CASES(0) PP_CASES(1) PP_CASES(2) PP_CASES(3)
-        PP_CASES(4) PP_CASES(5) PP_CASES(6) PP_CASES(7)
-        default: break;
-    }
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map, int x, int y, int c, int n,
+                                            uint32_t mbar) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], [%6];"
+        ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(c), "r"(n), "r"(mbar)
+        : "memory");
+}
+__device__ __forceinline__ void tmem_ld16(uint32_t ta, float (&a)[16]) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n\t"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(ta) : "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) a[i] = __uint_as_float(r[i]);
+}
+__device__ __forceinline__ void tmem_zero16(uint32_t ta) {
+    const uint32_t z = 0;
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1};\n\t"
+        "tcgen05.wait::st.sync.aligned;" ::"r"(ta), "r"(z) : "memory");
 }
 
-// Stage chunk `k` (channels [k*CK, k*CK+CK) ∩ [0, C)) into stage buffer `buf`.
+// One kept kernel applied to a lane's 4x4 accumulator block: the four taps of pattern P_ are
+// compile-time offsets into the input window (the 4 kept weights of §3.2); tap-outer order keeps
+// 16 independent FMAs between two dependent ones while every output still sums its taps in
+// ascending raster order.
+template <int P_, int S, int WY, int WX>
+__device__ __forceinline__ void fma_pattern(float (&a)[16], const float (&win)[WY][WX], const float4& w) {
+    constexpr int t[4] = {ktap(P_, 0), ktap(P_, 1), ktap(P_, 2), ktap(P_, 3)};
+    const float wk[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+#pragma unroll
+            for (int c = 0; c < 4; ++c) a[r * 4 + c] = fmaf(wk[k], win[r * S + t[k] / 3][c * S + t[k] % 3], a[r * 4 + c]);
+}
+
+// Accumulators of filter slot `ta` (16 tensor-memory columns) += pattern `pat` x window.
+template <int S, int WY, int WX>
+__device__ __forceinline__ void apply_kernel(uint32_t ta, uint32_t pat, const float4& w, const float (&win)[WY][WX]) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n\t"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(ta) : "memory");
+    float a[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) a[i] = __uint_as_float(r[i]);
+    switch (pat) {
+        case 0: fma_pattern<0, S, WY, WX>(a, win, w); break;
+        case 1: fma_pattern<1, S, WY, WX>(a, win, w); break;
+        case 2: fma_pattern<2, S, WY, WX>(a, win, w); break;
+        case 3: fma_pattern<3, S, WY, WX>(a, win, w); break;
+        case 4: fma_pattern<4, S, WY, WX>(a, win, w); break;
+        case 5: fma_pattern<5, S, WY, WX>(a, win, w); break;
+        case 6: fma_pattern<6, S, WY, WX>(a, win, w); break;
+        default: fma_pattern<7, S, WY, WX>(a, win, w); break;
+    }
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};"
+        ::"r"(ta), "f"(a[0]), "f"(a[1]), "f"(a[2]), "f"(a[3]), "f"(a[4]), "f"(a[5]), "f"(a[6]), "f"(a[7]),
+          "f"(a[8]), "f"(a[9]), "f"(a[10]), "f"(a[11]), "f"(a[12]), "f"(a[13]), "f"(a[14]), "f"(a[15])
+        : "memory");
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// Fallback input staging when no TMA descriptor applies (row pitch not a multiple of 16 bytes,
+// or fp16 input widened to fp32 on the way): copy the in-image part of the tile; everything else
+// in the stage keeps the zero written at kernel start.
 template <typename TIn>
-__device__ __forceinline__ void stage_chunk(const MainParams& p, int k, float* s_in, uint64_t* s_desc,
-                                            float4* s_vals, const uint32_t* s_kb, int g, int n0,
-                                            int iy0, int ix0) {
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int c0 = k * p.CK;
-    const int ckv = min(p.CK, p.C - c0);
-    // input tile: rows of (cl, img, row) distributed over warps, columns over lanes
-    const int rows = ckv * p.NB * p.IH;
+__device__ __forceinline__ void stage_input_fallback(const TmParams& p, float* s_in, int c0, int ckv, int n0,
+                                                     int iy0, int ix0, int lane) {
     const TIn* x = static_cast<const TIn*>(p.x);
-    for (int r = warp; r < rows; r += kWarps) {
-        const int row = r % p.IH;
-        const int t = r / p.IH;
-        const int img = t % p.NB;
-        const int cl = t / p.NB;
-        const int n = n0 + img, ci = c0 + cl, iy = iy0 + row;
-        const bool row_ok = n < p.N && iy >= 0 && iy < p.H;
-        const size_t gbase = (((size_t)n * p.C + ci) * p.H + (row_ok ? iy : 0)) * p.W;
-        float* srow = s_in + ((size_t)(cl * p.NB + img) * p.IH + row) * p.pitch;
-        for (int c = lane; c < p.IW; c += 32) {
-            const int ix = ix0 + c;
-            const bool ok = row_ok && ix >= 0 && ix < p.W;
-            if constexpr (sizeof(TIn) == 4) {
-                cp_async4(srow + c, ok ? (const void*)(x + gbase + ix) : p.x, ok);
-            } else {
-                srow[c] = ok ? to_f32<TIn>(x[gbase + ix]) : 0.0f;
+    const int ry0 = max(0, iy0), ry1 = min(p.H, iy0 + p.IH);
+    const int rx0 = max(0, ix0), rx1 = min(p.W, ix0 + p.BWb);
+    const int nr = ry1 - ry0, nc = rx1 - rx0;
+    if (nr <= 0 || nc <= 0) return;
+    int nimg = min(p.NB, p.N - n0);
+    const int planes = nimg * ckv;
+    // fp32 rows whose global start and length are even go as 8-byte pairs; the staged column of
+    // image column ix is ix - ix0 with ix0 a multiple of 4, so the shared side is 8-byte aligned too
+    const bool pairs = sizeof(TIn) == 4 && (p.W % 2 == 0) && (rx0 % 2 == 0) && (nc % 2 == 0);
+    const int units = pairs ? nc / 2 : nc;                  // copy units per row
+    const int per_plane = nr * units;
+    const int total = planes * per_plane;
+    // unit e -> (plane, row, unit-in-row), advanced incrementally by 32 per step
+    int pl = lane / per_plane, rem = lane - pl * per_plane;
+    int r = rem / units, u = rem - r * units;
+    const int step_pl = 32 / per_plane, step_rem = 32 - step_pl * per_plane;
+    for (int e = lane; e < total; e += 32) {
+        const int img = pl / ckv, cl = pl - (pl / ckv) * ckv;
+        const int iy = ry0 + r, ix = rx0 + (pairs ? 2 * u : u);
+        const TIn* src = x + (((size_t)(n0 + img) * p.C + c0 + cl) * p.H + iy) * p.W + ix;
+        float* dst = s_in + (((size_t)img * p.CK + cl) * p.IH + (iy - iy0)) * p.BWb + (ix - ix0);
+        if constexpr (sizeof(TIn) == 4) {
+            if (pairs) cp_async8(dst, src);
+            else cp_async4(dst, src, true);
+        } else {
+            *dst = to_f32<TIn>(*src);
+        }
+        pl += step_pl;
+        u += step_rem;
+        while (u >= units) {
+            u -= units;
+            if (++r == nr) {
+                r = 0;
+                ++pl;
             }
         }
     }
-    // this warp's group: descriptors and kept weights of the chunk
-    if (g < p.G) {
-        if (lane < ckv) cp_async8(s_desc + lane, p.desc + (size_t)g * p.C + c0 + lane);
-        const uint32_t beg = s_kb[warp * kMaxBoundaries + k], end = s_kb[warp * kMaxBoundaries + k + 1];
-        for (uint32_t i = beg + lane; i < end; i += 32) cp_async16(s_vals + (i - beg), p.vals + i);
-    }
 }
 
-template <int S, int RY, int RX, typename TIn>
-__global__ void __launch_bounds__(kThreads, 1) pconv_main(const MainParams p) {
-    constexpr int WY = Win<S, RY, RX>::WY, WX = Win<S, RY, RX>::WX;
-    constexpr int NST = 3;
-    extern __shared__ __align__(16) unsigned char smem[];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+// Fill pipeline stage k % kStages with input channel chunk k (whole warp; non-blocking): the
+// input tile by one TMA (or the fallback copy), each group's descriptors and kept weights by
+// cp.async; the stage's full barrier completes when every byte has landed.
+template <typename TIn>
+__device__ __forceinline__ void produce_chunk(const TmParams& p, const CUtensorMap* tmap, unsigned char* smem,
+                                              const uint32_t* s_kb, uint32_t full0, int k, int n0, int iy0,
+                                              int ix0, int g0, int lane) {
+    const int s = k % kStages;
+    const int nkb = p.n_chunks + 1;
+    unsigned char* st = smem + p.stage_off + (size_t)s * p.stage_bytes;
+    const uint32_t fb = full0 + 8 * s;
+    const int c0 = k * p.CK, ckv = min(p.CK, p.C - c0);
+    if (lane == 0) {
+        mbar_arrive_expect_tx(fb, p.use_tma ? p.tma_bytes : 0u);
+        if (p.use_tma) tma_load_4d(smem_u32(st), tmap, ix0, iy0, c0, n0, fb);
+    }
+    if (!p.use_tma) stage_input_fallback<TIn>(p, reinterpret_cast<float*>(st), c0, ckv, n0, iy0, ix0, lane);
+    uint64_t* sd = reinterpret_cast<uint64_t*>(st + p.desc_off);
+    for (int i = lane; i < p.WG * ckv; i += 32) {
+        const int wg = i / ckv, cl = i - wg * ckv, g = g0 + wg;
+        if (g < p.G) cp_async8(sd + wg * p.CK + cl, p.desc + (size_t)g * p.C + c0 + cl);
+    }
+    float4* sv = reinterpret_cast<float4*>(st + p.vals_off);
+    for (int wg = 0; wg < p.WG; ++wg) {
+        const uint32_t beg = s_kb[wg * nkb + k], end = s_kb[wg * nkb + k + 1];
+        for (uint32_t i = beg + lane; i < end; i += 32) cp_async16(sv + wg * p.maxk + (i - beg), p.vals + i);
+    }
+    __threadfence_block();
+    cp_async_arrive(fb);
+}
 
-    // CTA -> (spatial tile, filter chunk); filter chunk fastest so CTAs sharing a tile run together
+template <int S, typename TIn>
+__global__ void __launch_bounds__(kThreadsTM, 1)
+    pconv_tm(const TmParams p, const __grid_constant__ CUtensorMap tmap) {
+    constexpr int RY = 4, RX = 4;
+    constexpr int WY = (RY - 1) * S + 3, WX = (RX - 1) * S + 3;
+    extern __shared__ __align__(128) unsigned char smem[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    uint64_t* bar = reinterpret_cast<uint64_t*>(smem);                    // full[kStages]
+    uint32_t* s_cnt = reinterpret_cast<uint32_t*>(smem + 8 * kStages);    // releases per stage
+    uint32_t* s_tmem = s_cnt + kStages;                                   // tensor-memory base
+    uint32_t* s_issued = s_tmem + 1;                                      // chunks issued
+    uint32_t* s_kb = reinterpret_cast<uint32_t*>(smem + p.kb_off);
+    const uint32_t full0 = smem_u32(bar);
+
+    // CTA -> (spatial tile, filter chunk); the filter chunk varies fastest so CTAs that share an
+    // input tile run together and hit it in L2
     const int cta = blockIdx.x;
     const int fchunk = cta % p.n_fchunks;
     int t = cta / p.n_fchunks;
@@ -200,143 +318,174 @@ __global__ void __launch_bounds__(kThreads, 1) pconv_main(const MainParams p) {
     const int tn = t / p.tiles_y;
     const int n0 = tn * p.NB;
     const int oy0 = ty * p.BY * RY, ox0 = tx * p.BX * RX;
-    const int iy0 = oy0 * S - 1, ix0 = ox0 * S - 1;
-    const int g = fchunk * kWarps + warp;
+    const int iy0 = oy0 * S - 1, ix0 = ox0 * S - 4;     // stage origin: 1 halo row, 16-B aligned col
+    const int g0 = fchunk * p.WG;
+    const int nkb = p.n_chunks + 1;
 
-    // shared memory carve-up
-    const int vals_per_warp = kF * p.CK;
-    float* s_in = reinterpret_cast<float*>(smem);
-    float4* s_vals = reinterpret_cast<float4*>(s_in + (size_t)NST * p.stage_floats);
-    uint64_t* s_desc = reinterpret_cast<uint64_t*>(s_vals + (size_t)NST * kWarps * vals_per_warp);
-    uint32_t* s_kb = reinterpret_cast<uint32_t*>(s_desc + (size_t)NST * kWarps * p.CK);
-
-    // chunk boundaries of this warp's group in the kept-weight stream
-    if (g < p.G) {
-        for (int i = lane; i <= p.n_chunks; i += 32)
-            s_kb[warp * kMaxBoundaries + i] = p.kofs[(size_t)g * p.C + min(i * p.CK, p.C)];
+    if (!p.use_tma) {   // the fallback writes only in-image elements: zero all stages once
+        float* z = reinterpret_cast<float*>(smem + p.stage_off);
+        const int nf = (int)(kStages * p.stage_bytes / 4);
+        for (int i = threadIdx.x; i < nf; i += kThreadsTM) z[i] = 0.0f;
     }
+    for (int i = threadIdx.x; i < p.WG * nkb; i += kThreadsTM) {
+        const int wg = i / nkb, j = i - wg * nkb, g = g0 + wg;
+        s_kb[i] = g < p.G ? p.kofs[(size_t)g * p.C + min(j * p.CK, p.C)] : 0u;
+    }
+    if (warp == 0) {
+        if (lane == 0) {
+            for (int s = 0; s < kStages; ++s) {
+                mbar_init(full0 + 8 * s, 33);   // lane 0's expect-tx arrival + 32 cp.async arrivals
+                s_cnt[s] = 0;
+            }
+            *s_issued = 0;
+        }
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
+                     ::"r"(smem_u32(s_tmem)), "r"(kTmemCols) : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tbase = *s_tmem;
 
-    // lane -> block
-    const int blk = lane;
+    if (warp == 0) {   // prologue: fill every stage
+        const int first = min(kStages, p.n_chunks);
+        for (int k = 0; k < first; ++k) produce_chunk<TIn>(p, &tmap, smem, s_kb, full0, k, n0, iy0, ix0, g0, lane);
+        if (lane == 0) *s_issued = first;
+    }
+
+    const int wg = warp / p.WS, ws = warp - (warp / p.WS) * p.WS;
+    const int g = g0 + wg;
+    // tensor memory: warp w owns lanes 32*(w%4).. and columns 128*(w/4) + 16*slot ..
+    const uint32_t tw = tbase + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)(128 * (warp >> 2));
+#pragma unroll
+    for (int f = 0; f < kF; ++f) tmem_zero16(tw + 16u * f);
+
+    const int blk = ws * 32 + lane;
     const int per_img = p.BY * p.BX;
     const int img = blk / per_img;
-    const int by = (blk % per_img) / p.BX, bx = blk % p.BX;
+    const int rem = blk - img * per_img;
+    const int by = rem / p.BX, bx = rem - (rem / p.BX) * p.BX;
     const bool active = img < p.NB;
-    const int lane_off = active ? (img * p.IH + by * RY * S) * p.pitch + bx * RX * S : 0;
-    const int plane = p.NB * p.IH * p.pitch;
-
-    float acc[kF][RY * RX];
-#pragma unroll
-    for (int f = 0; f < kF; ++f)
-#pragma unroll
-        for (int i = 0; i < RY * RX; ++i) acc[f][i] = 0.0f;
-
-#pragma unroll
-    for (int s = 0; s < NST - 1; ++s) {
-        if (s < p.n_chunks)
-            stage_chunk<TIn>(p, s, s_in + (size_t)s * p.stage_floats, s_desc + (size_t)(s * kWarps + warp) * p.CK,
-                             s_vals + (size_t)(s * kWarps + warp) * vals_per_warp, s_kb, g, n0, iy0, ix0);
-        cp_commit();
-    }
+    const int plane = p.IH * p.BWb;
+    const int in_off = active ? img * p.CK * plane + by * RY * S * p.BWb + bx * RX * S + 3 : 3;
 
     for (int k = 0; k < p.n_chunks; ++k) {
-        cp_wait<NST - 2>();
-        __syncthreads();
-        {
-            const int kn = k + NST - 1, sb = kn % NST;
-            if (kn < p.n_chunks)
-                stage_chunk<TIn>(p, kn, s_in + (size_t)sb * p.stage_floats,
-                                 s_desc + (size_t)(sb * kWarps + warp) * p.CK,
-                                 s_vals + (size_t)(sb * kWarps + warp) * vals_per_warp, s_kb, g, n0, iy0, ix0);
-            cp_commit();
-        }
-        if (g >= p.G) continue;
-        const int sb = k % NST;
-        const float* s_base = s_in + (size_t)sb * p.stage_floats + lane_off;
-        const uint64_t* sd = s_desc + (size_t)(sb * kWarps + warp) * p.CK;
-        const float4* sv = s_vals + (size_t)(sb * kWarps + warp) * vals_per_warp;
-        const int ckv = min(p.CK, p.C - k * p.CK);
-        int voff = 0;
-        for (int cl = 0; cl < ckv; ++cl) {
-            uint64_t d = sd[cl];
-            const int cnt = (int)(d & 15u);
-            if (cnt == 0) continue;
-            d >>= 4;
-            float win[WY][WX];
-            const float* wp = s_base + (size_t)cl * plane;
+        const int s = k % kStages;
+        if (!mbar_wait(full0 + 8 * s, (k / kStages) & 1, p.status, kStatusFullTimeout)) break;
+        if (g < p.G) {
+            const unsigned char* st = smem + p.stage_off + (size_t)s * p.stage_bytes;
+            const float* sin0 = reinterpret_cast<const float*>(st) + in_off;
+            const uint64_t* sd = reinterpret_cast<const uint64_t*>(st + p.desc_off) + wg * p.CK;
+            const float4* sv = reinterpret_cast<const float4*>(st + p.vals_off) + wg * p.maxk;
+            const int ckv = min(p.CK, p.C - k * p.CK);
+            int voff = 0;
+            for (int cl = 0; cl < ckv; ++cl) {
+                uint64_t d = sd[cl];
+                const int cnt = (int)(d & 15u);
+                if (cnt == 0) continue;
+                d >>= 4;
+                float win[WY][WX];
+                const float* wp = sin0 + (size_t)cl * plane;
 #pragma unroll
-            for (int r = 0; r < WY; ++r) {
+                for (int r = 0; r < WY; ++r) {
+                    const float* rp = wp + r * p.BWb;
+                    win[r][0] = rp[0];
 #pragma unroll
-                for (int c = 0; c < WX; c += 4) {
-                    if (c + 4 <= WX) {
-                        const float4 v = *reinterpret_cast<const float4*>(wp + r * p.pitch + c);
+                    for (int c = 1; c + 4 <= WX; c += 4) {
+                        const float4 v = *reinterpret_cast<const float4*>(rp + c);
                         win[r][c] = v.x;
                         win[r][c + 1] = v.y;
                         win[r][c + 2] = v.z;
                         win[r][c + 3] = v.w;
-                    } else if (c + 2 <= WX) {
-                        const float2 v = *reinterpret_cast<const float2*>(wp + r * p.pitch + c);
-                        win[r][c] = v.x;
-                        win[r][c + 1] = v.y;
-                        if (c + 3 <= WX) win[r][c + 2] = wp[r * p.pitch + c + 2];
-                    } else {
-                        win[r][c] = wp[r * p.pitch + c];
                     }
+                    if constexpr ((WX - 1) % 4 != 0) win[r][WX - 1] = rp[WX - 1];
                 }
+                for (int j = 0; j < cnt; ++j) {
+                    const float4 w = sv[voff + j];
+                    const uint32_t code = (uint32_t)(d & 63u);
+                    d >>= 6;
+                    apply_kernel<S, WY, WX>(tw + 16u * (code >> 3), code & 7u, w, win);
+                }
+                voff += cnt;
             }
-            for (int j = 0; j < cnt; ++j) {
-                const float4 w = sv[voff + j];
-                const int code = (int)(d & 63u);
-                d >>= 6;
-                dispatch<S, RY, RX, WY, WX>(code, w, acc, win);
+        }
+        // release the stage; the last warp to release it refills it with chunk k + kStages
+        __syncwarp();
+        uint32_t old = 0;
+        if (lane == 0) {
+            __threadfence_block();
+            old = atomicAdd(&s_cnt[s], 1u);
+        }
+        old = __shfl_sync(0xffffffffu, old, 0);
+        if (old == kCompute - 1) {
+            if (lane == 0) s_cnt[s] = 0;
+            if (k + kStages < p.n_chunks) {
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                produce_chunk<TIn>(p, &tmap, smem, s_kb, full0, k + kStages, n0, iy0, ix0, g0, lane);
+                if (lane == 0) atomicMax(s_issued, (uint32_t)(k + kStages + 1));
             }
-            voff += cnt;
         }
     }
-    cp_wait<0>();
 
-    // epilogue: bias + ReLU + store to the original channel of every slot
-    if (g >= p.G || !active) return;
-    const int n = n0 + img;
-    if (n >= p.N) return;
-    const int oyb = oy0 + by * RY, oxb = ox0 + bx * RX;
-    using TOut = TIn;
-    TOut* y = static_cast<TOut*>(p.y);
+    // epilogue: accumulators out of tensor memory, + bias, ReLU, store to the original channel
+    {
+        const int n = n0 + img;
+        const int oyb = oy0 + by * RY, oxb = ox0 + bx * RX;
+        using TOut = TIn;
+        TOut* y = static_cast<TOut*>(p.y);
+#pragma unroll 1
+        for (int f = 0; f < kF; ++f) {
+            float a[16];
+            __syncwarp();
+            tmem_ld16(tw + 16u * f, a);
+            if (g >= p.G || !active || n >= p.N) continue;
+            const uint32_t co = p.perm[g * kF + f];
+            if (co == kPadSlot) continue;
+            const float b = p.bias ? p.bias[co] : 0.0f;
+            TOut* yc = y + ((size_t)n * p.Cout + co) * p.Ho * p.Wo;
 #pragma unroll
-    for (int f = 0; f < kF; ++f) {
-        const uint32_t co = p.perm[g * kF + f];
-        if (co == kPadSlot) continue;
-        const float b = p.bias ? p.bias[co] : 0.0f;
-        TOut* yc = y + ((size_t)n * p.Cout + co) * p.Ho * p.Wo;
+            for (int r = 0; r < RY; ++r) {
+                const int oy = oyb + r;
+                if (oy >= p.Ho) break;
+                TOut* yr = yc + (size_t)oy * p.Wo;
+                float v[RX];
 #pragma unroll
-        for (int r = 0; r < RY; ++r) {
-            const int oy = oyb + r;
-            if (oy >= p.Ho) break;
-            TOut* yr = yc + (size_t)oy * p.Wo;
-            float v[RX];
-#pragma unroll
-            for (int c = 0; c < RX; ++c) {
-                float a = acc[f][r * RX + c] + b;
-                v[c] = p.relu ? fmaxf(a, 0.0f) : a;
-            }
-            if (RX == 4 && p.vec_store && oxb + RX <= p.Wo) {
-                if constexpr (sizeof(TOut) == 4) {
-                    *reinterpret_cast<float4*>(yr + oxb) = make_float4(v[0], v[1], v[2], v[3]);
-                } else {
-                    __half2 h0 = __floats2half2_rn(v[0], v[1]);
-                    __half2 h1 = __floats2half2_rn(v[2], v[3]);
-                    uint2 u;
-                    u.x = *reinterpret_cast<unsigned*>(&h0);
-                    u.y = *reinterpret_cast<unsigned*>(&h1);
-                    *reinterpret_cast<uint2*>(yr + oxb) = u;
+                for (int c = 0; c < RX; ++c) {
+                    const float q = a[r * RX + c] + b;
+                    v[c] = p.relu ? fmaxf(q, 0.0f) : q;
                 }
-            } else {
+                if (p.vec_store && oxb + RX <= p.Wo) {
+                    if constexpr (sizeof(TOut) == 4) {
+                        *reinterpret_cast<float4*>(yr + oxb) = make_float4(v[0], v[1], v[2], v[3]);
+                    } else {
+                        __half2 h0 = __floats2half2_rn(v[0], v[1]);
+                        __half2 h1 = __floats2half2_rn(v[2], v[3]);
+                        uint2 u;
+                        u.x = *reinterpret_cast<unsigned*>(&h0);
+                        u.y = *reinterpret_cast<unsigned*>(&h1);
+                        *reinterpret_cast<uint2*>(yr + oxb) = u;
+                    }
+                } else {
 #pragma unroll
-                for (int c = 0; c < RX; ++c)
-                    if (oxb + c < p.Wo) yr[oxb + c] = from_f32<TOut>(v[c]);
+                    for (int c = 0; c < RX; ++c)
+                        if (oxb + c < p.Wo) yr[oxb + c] = from_f32<TOut>(v[c]);
+                }
             }
         }
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 0) {
+        // no copy of this CTA may still be in flight when it exits (only possible after a timeout)
+        if (lane == 0) {
+            const int issued = (int)*s_issued;
+            for (int k = max(0, issued - kStages); k < issued; ++k)
+                mbar_wait(full0 + 8 * (k % kStages), (k / kStages) & 1, p.status, kStatusDrainTimeout);
+        }
+        __syncwarp();
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tbase), "r"(kTmemCols) : "memory");
     }
 }
 
@@ -485,40 +634,75 @@ int sm_count() {
     return n;
 }
 
-struct Tile {
-    int BY, BX, NB;
+using EncodeTiledFn = PFN_cuTensorMapEncodeTiled_v12000;
+
+EncodeTiledFn encode_tiled() {
+    static const EncodeTiledFn fn = []() -> EncodeTiledFn {
+        void* f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            return nullptr;
+        return reinterpret_cast<EncodeTiledFn>(f);
+    }();
+    return fn;
+}
+
+unsigned* status_word() {
+    static std::atomic<unsigned*> cached[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return nullptr;
+    if (dev < 64 && cached[dev].load()) return cached[dev].load();
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_pp_status) != cudaSuccess) return nullptr;
+    if (dev < 64) cached[dev].store(static_cast<unsigned*>(ptr));
+    return static_cast<unsigned*>(ptr);
+}
+
+struct TileChoice {
+    int BY = 1, BX = 1, NB = 1, IH = 0, BWb = 0;
 };
 
-// Spatial tile of 32 lane-blocks that minimises the number of CTA waves, then wasted lanes.
-Tile choose_tile(int N, int Ho, int Wo, int RY, int RX, int n_fchunks) {
-    const int nby = (Ho + RY - 1) / RY, nbx = (Wo + RX - 1) / RX;
-    const long long slots = sm_count();
-    Tile best{1, 1, 1};
+// Spatial tile of at most 32*WS blocks (4x4 outputs each) minimising CTA waves, then the lanes
+// left idle; stride-1 rows need 4*BX + 5 staged columns, stride-2 rows 8*BX + 4, rounded to a
+// 16-byte multiple and padded to 4 (mod 8) floats so that rows four apart fall in other banks.
+TileChoice choose_tile(int N, int Ho, int Wo, int S, int lanes, int n_fchunks, int C) {
+    const int nby = (Ho + 3) / 4, nbx = (Wo + 3) / 4;
+    const long long sms = sm_count();
+    TileChoice best;
     long long best_waves = LLONG_MAX, best_cover = LLONG_MAX;
-    int best_bx = 0;
-    for (int bx = 1; bx <= std::min(nbx, 32); ++bx) {
-        for (int by = 1; by <= std::min(nby, 32 / bx); ++by) {
-            const int nb = std::max(1, std::min(N, 32 / (bx * by)));
+    for (int bx = 1; bx <= std::min(nbx, lanes); ++bx) {
+        for (int by = 1; by <= std::min(nby, lanes / bx); ++by) {
+            // several images per tile only when each image contributes a whole image's blocks
+            // (lanes then step through one image before the next: no bank-aligned image stride)
+            const bool whole = by == nby && bx == nbx;
+            const int nb = whole ? std::max(1, std::min(std::min(N, 256), lanes / (bx * by))) : 1;
+            const int ih = S == 1 ? 4 * by + 2 : 8 * by + 1;
+            int bw = S == 1 ? 4 * bx + 8 : 8 * bx + 4;
+            if (bw % 8 == 0) bw += 4;
+            if (bw > 256 || ih > 256) continue;
+            const int ck_min = (C + kMaxChunks - 1) / kMaxChunks;
+            if ((long long)nb * ih * bw * 4 * ck_min > 48 * 1024) continue;   // enough channels per stage
             const long long tiles = (long long)((N + nb - 1) / nb) * ((nby + by - 1) / by) * ((nbx + bx - 1) / bx);
-            const long long ctas = tiles * n_fchunks;
-            const long long waves = (ctas + slots - 1) / slots;
-            const long long cover = tiles * 32;   // lanes issued
+            const long long waves = (tiles * n_fchunks + sms - 1) / sms;
+            const long long cover = tiles * lanes;
             if (waves < best_waves || (waves == best_waves && (cover < best_cover ||
-                                                               (cover == best_cover && bx > best_bx)))) {
-                best = Tile{by, bx, nb};
+                                                               (cover == best_cover && bx > best.BX)))) {
+                best = TileChoice{by, bx, nb, ih, bw};
                 best_waves = waves;
                 best_cover = cover;
-                best_bx = bx;
             }
         }
     }
     return best;
 }
 
-template <int S, int RY, int RX, typename T>
-int launch_main(const pp_layer* L, const void* x, void* y, const float* bias, int relu, int N, int H, int W,
-                int Ho, int Wo, cudaStream_t st) {
-    MainParams p{};
+size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+template <int S, typename T>
+int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int relu, int N, int H, int W, int Ho,
+              int Wo, cudaStream_t st) {
+    TmParams p{};
     p.x = x;
     p.y = y;
     p.bias = bias;
@@ -527,6 +711,8 @@ int launch_main(const pp_layer* L, const void* x, void* y, const float* bias, in
     p.desc = reinterpret_cast<const uint64_t*>(img + L->off_desc);
     p.kofs = reinterpret_cast<const uint32_t*>(img + L->off_kofs);
     p.vals = reinterpret_cast<const float4*>(img + L->off_vals);
+    p.status = status_word();
+    if (!p.status) return PP_ERR_CUDA;
     p.N = N;
     p.C = L->cin_g;
     p.H = H;
@@ -536,46 +722,84 @@ int launch_main(const pp_layer* L, const void* x, void* y, const float* bias, in
     p.Wo = Wo;
     p.G = L->G;
     p.relu = relu;
-    p.n_fchunks = (L->G + kWarps - 1) / kWarps;
-    const Tile t = choose_tile(N, Ho, Wo, RY, RX, p.n_fchunks);
+    int wg = 1;
+    while (wg < L->G && wg < kCompute) wg *= 2;
+    p.WG = wg;
+    p.WS = kCompute / wg;
+    p.n_fchunks = (L->G + wg - 1) / wg;
+    const TileChoice t = choose_tile(N, Ho, Wo, S, 32 * p.WS, p.n_fchunks, L->cin_g);
+    if (t.IH == 0) return PP_ERR_SHAPE;
     p.BY = t.BY;
     p.BX = t.BX;
     p.NB = t.NB;
-    p.tiles_x = ((Wo + RX - 1) / RX + t.BX - 1) / t.BX;
-    p.tiles_y = ((Ho + RY - 1) / RY + t.BY - 1) / t.BY;
+    p.IH = t.IH;
+    p.BWb = t.BWb;
+    p.tiles_x = ((Wo + 3) / 4 + t.BX - 1) / t.BX;
+    p.tiles_y = ((Ho + 3) / 4 + t.BY - 1) / t.BY;
     p.tiles_n = (N + t.NB - 1) / t.NB;
-    p.IH = (t.BY * RY - 1) * S + 3;
-    p.IW = (t.BX * RX - 1) * S + 3;
-    p.pitch = (p.IW + 3) / 4 * 4;
-    // channels per stage: fill ~40 KB of input per stage, at most 32, at least 1
-    const int per_ci = p.NB * p.IH * p.pitch;
-    int ck = std::max(1, std::min(32, (40 * 1024 / 4) / std::max(per_ci, 1)));
-    ck = std::min(ck, L->cin_g);
-    p.n_chunks = (L->cin_g + ck - 1) / ck;
-    if (p.n_chunks + 1 > kMaxBoundaries) {
-        ck = (L->cin_g + kMaxBoundaries - 2) / (kMaxBoundaries - 1);
-        p.n_chunks = (L->cin_g + ck - 1) / ck;
-    }
-    constexpr int NST = 3;
-    auto smem_bytes = [&](int c) {
-        return (size_t)NST * c * per_ci * 4 + (size_t)NST * kWarps * kF * c * 16 + (size_t)NST * kWarps * c * 8 +
-               (size_t)kWarps * kMaxBoundaries * 4;
+    const int C = L->cin_g;
+    const size_t es = sizeof(T);
+    p.use_tma = es == 4 && (W * es) % 16 == 0 && reinterpret_cast<uintptr_t>(x) % 16 == 0 && encode_tiled() != nullptr;
+
+    // channels per stage: the largest that fits three stages in shared memory
+    auto maxk_for = [&](int ck) {
+        uint32_t m = 0;
+        for (int g = 0; g < L->G; ++g)
+            for (int c0 = 0; c0 < C; c0 += ck) {
+                const size_t b = (size_t)g * C;
+                m = std::max(m, L->kofs[b + std::min(c0 + ck, C)] - L->kofs[b + c0]);
+            }
+        return (int)m;
     };
-    while (ck > 1 && smem_bytes(ck) > 200 * 1024) --ck;
-    p.n_chunks = (L->cin_g + ck - 1) / ck;
-    if (p.n_chunks + 1 > kMaxBoundaries) return PP_ERR_SHAPE;
+    auto layout = [&](int ck, int maxk, size_t* stage_bytes, size_t* kb_bytes) {
+        const size_t in_b = align_up((size_t)p.NB * ck * p.IH * p.BWb * 4, 128);
+        const size_t desc_b = align_up((size_t)p.WG * ck * 8, 16);
+        const size_t vals_b = (size_t)p.WG * std::max(maxk, 1) * 16;
+        *stage_bytes = align_up(in_b + desc_b + vals_b, 128);
+        const int nch = (C + ck - 1) / ck;
+        *kb_bytes = (size_t)p.WG * (nch + 1) * 4;
+        return align_up(64 + *kb_bytes, 128) + kStages * *stage_bytes;
+    };
+    int ck = std::min(C, 64);
+    int maxk = 0;
+    size_t stage_bytes = 0, kb_bytes = 0, total = 0;
+    for (;; --ck) {
+        if (ck < 1) return PP_ERR_SHAPE;
+        if ((C + ck - 1) / ck > kMaxChunks) return PP_ERR_SHAPE;
+        maxk = maxk_for(ck);
+        total = layout(ck, maxk, &stage_bytes, &kb_bytes);
+        if (total <= 200 * 1024) break;
+    }
     p.CK = ck;
-    p.stage_floats = ck * per_ci;
-    p.vec_store = (RX == 4) && (Wo % 4 == 0) &&
-                  ((reinterpret_cast<uintptr_t>(y) % (4 * sizeof(T))) == 0);
-    const size_t smem = smem_bytes(ck);
-    if (smem > 227 * 1024) return PP_ERR_SHAPE;
-    auto kern = pconv_main<S, RY, RX, T>;
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+    p.n_chunks = (C + ck - 1) / ck;
+    p.maxk = std::max(maxk, 1);
+    p.kb_off = 64;
+    p.stage_off = (unsigned)align_up(64 + kb_bytes, 128);
+    p.stage_bytes = (unsigned)stage_bytes;
+    p.desc_off = (unsigned)align_up((size_t)p.NB * ck * p.IH * p.BWb * 4, 128);
+    p.vals_off = p.desc_off + (unsigned)align_up((size_t)p.WG * ck * 8, 16);
+    p.vec_store = (Wo % 4 == 0) && (reinterpret_cast<uintptr_t>(y) % (4 * es)) == 0;
+
+    CUtensorMap tmap;
+    std::memset(&tmap, 0, sizeof(tmap));
+    if (p.use_tma) {
+        const cuuint64_t dims[4] = {(cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)C, (cuuint64_t)N};
+        const cuuint64_t strides[3] = {(cuuint64_t)W * es, (cuuint64_t)H * W * es, (cuuint64_t)C * H * W * es};
+        const cuuint32_t box[4] = {(cuuint32_t)p.BWb, (cuuint32_t)p.IH, (cuuint32_t)ck, (cuuint32_t)p.NB};
+        const cuuint32_t estr[4] = {1, 1, 1, 1};
+        const CUresult r = encode_tiled()(&tmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<void*>(x), dims,
+                                          strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                                          CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) p.use_tma = 0;
+        p.tma_bytes = (unsigned)((size_t)p.BWb * p.IH * ck * p.NB * 4);
+    }
+    auto kern = pconv_tm<S, T>;
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)total) != cudaSuccess)
         return PP_ERR_CUDA;
     const long long ctas = (long long)p.tiles_n * p.tiles_y * p.tiles_x * p.n_fchunks;
     if (ctas > INT_MAX) return PP_ERR_SHAPE;
-    kern<<<(unsigned)ctas, kThreads, smem, st>>>(p);
+    kern<<<(unsigned)ctas, kThreadsTM, total, st>>>(p, tmap);
     return cudaGetLastError() == cudaSuccess ? PP_OK : PP_ERR_CUDA;
 }
 
@@ -669,10 +893,22 @@ int pp_conv(pp_handle h, const void* x, int dtype, int N, int H, int W, const fl
                    : launch_depthwise<float>(h, x, y, bias, relu, N, H, W, Ho, Wo, st);
     }
     if (h->stride == 1)
-        return f16 ? launch_main<1, 4, 4, __half>(h, x, y, bias, relu, N, H, W, Ho, Wo, st)
-                   : launch_main<1, 4, 4, float>(h, x, y, bias, relu, N, H, W, Ho, Wo, st);
-    return f16 ? launch_main<2, 2, 4, __half>(h, x, y, bias, relu, N, H, W, Ho, Wo, st)
-               : launch_main<2, 2, 4, float>(h, x, y, bias, relu, N, H, W, Ho, Wo, st);
+        return f16 ? launch_tm<1, __half>(h, x, y, bias, relu, N, H, W, Ho, Wo, st)
+                   : launch_tm<1, float>(h, x, y, bias, relu, N, H, W, Ho, Wo, st);
+    return f16 ? launch_tm<2, __half>(h, x, y, bias, relu, N, H, W, Ho, Wo, st)
+               : launch_tm<2, float>(h, x, y, bias, relu, N, H, W, Ho, Wo, st);
+}
+
+int pp_device_status(int clear, unsigned int* status) {
+    if (!status) return PP_ERR_NULL;
+    unsigned v = 0;
+    if (cudaMemcpyFromSymbol(&v, g_pp_status, sizeof(v)) != cudaSuccess) return PP_ERR_CUDA;
+    if (clear) {
+        const unsigned z = 0;
+        if (cudaMemcpyToSymbol(g_pp_status, &z, sizeof(z)) != cudaSuccess) return PP_ERR_CUDA;
+    }
+    *status = v;
+    return PP_OK;
 }
 
 int pp_maxpool2x2(const void* x, int dtype, int N, int C, int H, int W, void* y, void* stream) {
