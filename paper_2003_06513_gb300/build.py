@@ -24,7 +24,7 @@ NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "--expt-relaxed-constexpr", "-Xc
               "-Xcompiler", "-ffp-contract=off", "-I", os.path.join(ROOT, "include")] + ARCH
 GXX_FLAGS = ["-O2", "-std=c++17", "-fPIC", "-ffp-contract=off", "-Wall", "-I",
              os.path.join(ROOT, "include")]
-SOURCES = ["conv.cu", "pack.cpp", "layer.h"]
+SOURCES = ["conv.cu", "pack.cpp", "layer.h", "gen_dispatch.py"]
 
 
 def _nvcc() -> str:
@@ -53,10 +53,12 @@ def build(force: bool = False, verbose: bool = False, extra_nvcc=()) -> str:
             if f.read().strip() == digest:
                 return LIB
     nvcc = _nvcc()
+    subprocess.run([sys.executable, os.path.join(CSRC, "gen_dispatch.py"),
+                    os.path.join(BUILD, "pattern_dispatch.h")], check=True)
     conv_o = os.path.join(BUILD, "conv.o")
     pack_o = os.path.join(BUILD, "pack.o")
     cmds = [
-        [nvcc, "-c", os.path.join(CSRC, "conv.cu"), "-o", conv_o] + NVCC_FLAGS + list(extra_nvcc),
+        [nvcc, "-c", os.path.join(CSRC, "conv.cu"), "-o", conv_o, "-I", BUILD] + NVCC_FLAGS + list(extra_nvcc),
         ["g++", "-c", os.path.join(CSRC, "pack.cpp"), "-o", pack_o] + GXX_FLAGS,
     ]
 

@@ -29,6 +29,7 @@
 
 #include "../../include/patconv.h"
 #include "layer.h"
+#include "pattern_dispatch.h"
 
 using namespace patconv;
 
@@ -169,53 +170,6 @@ __device__ __forceinline__ void tmem_zero16(uint32_t ta) {
         "tcgen05.wait::st.sync.aligned;" ::"r"(ta), "r"(z) : "memory");
 }
 
-// One kept kernel applied to a lane's 4x4 accumulator block: the four taps of pattern P_ are
-// compile-time offsets into the input window (the 4 kept weights of §3.2); tap-outer order keeps
-// 16 independent FMAs between two dependent ones while every output still sums its taps in
-// ascending raster order.
-template <int P_, int S, int WY, int WX>
-__device__ __forceinline__ void fma_pattern(float (&a)[16], const float (&win)[WY][WX], const float4& w) {
-    constexpr int t[4] = {ktap(P_, 0), ktap(P_, 1), ktap(P_, 2), ktap(P_, 3)};
-    const float wk[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-    for (int k = 0; k < 4; ++k)
-#pragma unroll
-        for (int r = 0; r < 4; ++r)
-#pragma unroll
-            for (int c = 0; c < 4; ++c) a[r * 4 + c] = fmaf(wk[k], win[r * S + t[k] / 3][c * S + t[k] % 3], a[r * 4 + c]);
-}
-
-// Accumulators of filter slot `ta` (16 tensor-memory columns) += pattern `pat` x window.
-template <int S, int WY, int WX>
-__device__ __forceinline__ void apply_kernel(uint32_t ta, uint32_t pat, const float4& w, const float (&win)[WY][WX]) {
-    uint32_t r[16];
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n\t"
-        "tcgen05.wait::ld.sync.aligned;"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(ta) : "memory");
-    float a[16];
-#pragma unroll
-    for (int i = 0; i < 16; ++i) a[i] = __uint_as_float(r[i]);
-    switch (pat) {
-        case 0: fma_pattern<0, S, WY, WX>(a, win, w); break;
-        case 1: fma_pattern<1, S, WY, WX>(a, win, w); break;
-        case 2: fma_pattern<2, S, WY, WX>(a, win, w); break;
-        case 3: fma_pattern<3, S, WY, WX>(a, win, w); break;
-        case 4: fma_pattern<4, S, WY, WX>(a, win, w); break;
-        case 5: fma_pattern<5, S, WY, WX>(a, win, w); break;
-        case 6: fma_pattern<6, S, WY, WX>(a, win, w); break;
-        default: fma_pattern<7, S, WY, WX>(a, win, w); break;
-    }
-    asm volatile(
-        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};"
-        ::"r"(ta), "f"(a[0]), "f"(a[1]), "f"(a[2]), "f"(a[3]), "f"(a[4]), "f"(a[5]), "f"(a[6]), "f"(a[7]),
-          "f"(a[8]), "f"(a[9]), "f"(a[10]), "f"(a[11]), "f"(a[12]), "f"(a[13]), "f"(a[14]), "f"(a[15])
-        : "memory");
-    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-}
-
 // Fallback input staging when no TMA descriptor applies (row pitch not a multiple of 16 bytes,
 // or fp16 input widened to fp32 on the way): copy the in-image part of the tile; everything else
 // in the stage keeps the zero written at kernel start.
@@ -297,7 +251,6 @@ template <int S, typename TIn>
 __global__ void __launch_bounds__(kThreadsTM, 1)
     pconv_tm(const TmParams p, const __grid_constant__ CUtensorMap tmap) {
     constexpr int RY = 4, RX = 4;
-    constexpr int WY = (RY - 1) * S + 3, WX = (RX - 1) * S + 3;
     extern __shared__ __align__(128) unsigned char smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     uint64_t* bar = reinterpret_cast<uint64_t*>(smem);                    // full[kStages]
@@ -375,39 +328,14 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
         if (!mbar_wait(full0 + 8 * s, (k / kStages) & 1, p.status, kStatusFullTimeout)) break;
         if (g < p.G) {
             const unsigned char* st = smem + p.stage_off + (size_t)s * p.stage_bytes;
-            const float* sin0 = reinterpret_cast<const float*>(st) + in_off;
-            const uint64_t* sd = reinterpret_cast<const uint64_t*>(st + p.desc_off) + wg * p.CK;
-            const float4* sv = reinterpret_cast<const float4*>(st + p.vals_off) + wg * p.maxk;
+            const uint32_t win_addr = smem_u32(reinterpret_cast<const float*>(st) + in_off);
+            const uint32_t desc_addr = smem_u32(reinterpret_cast<const uint64_t*>(st + p.desc_off) + wg * p.CK);
+            const uint32_t vals_addr = smem_u32(reinterpret_cast<const float4*>(st + p.vals_off) + wg * p.maxk);
             const int ckv = min(p.CK, p.C - k * p.CK);
-            int voff = 0;
-            for (int cl = 0; cl < ckv; ++cl) {
-                uint64_t d = sd[cl];
-                const int cnt = (int)(d & 15u);
-                if (cnt == 0) continue;
-                d >>= 4;
-                float win[WY][WX];
-                const float* wp = sin0 + (size_t)cl * plane;
-#pragma unroll
-                for (int r = 0; r < WY; ++r) {
-                    const float* rp = wp + r * p.BWb;
-                    win[r][0] = rp[0];
-#pragma unroll
-                    for (int c = 1; c + 4 <= WX; c += 4) {
-                        const float4 v = *reinterpret_cast<const float4*>(rp + c);
-                        win[r][c] = v.x;
-                        win[r][c + 1] = v.y;
-                        win[r][c + 2] = v.z;
-                        win[r][c + 3] = v.w;
-                    }
-                    if constexpr ((WX - 1) % 4 != 0) win[r][WX - 1] = rp[WX - 1];
-                }
-                for (int j = 0; j < cnt; ++j) {
-                    const float4 w = sv[voff + j];
-                    const uint32_t code = (uint32_t)(d & 63u);
-                    d >>= 6;
-                    apply_kernel<S, WY, WX>(tw + 16u * (code >> 3), code & 7u, w, win);
-                }
-                voff += cnt;
+            if constexpr (S == 1) {
+                PP_STAGE_KERNELS_S1(ckv, desc_addr, vals_addr, win_addr, 4 * p.BWb, 4 * plane, tw);
+            } else {
+                PP_STAGE_KERNELS_S2(ckv, desc_addr, vals_addr, win_addr, 4 * p.BWb, 4 * plane, tw);
             }
         }
         // release the stage; the last warp to release it refills it with chunk k + kStages

@@ -1,0 +1,134 @@
+#!/usr/bin/env python3
+"""Generate pattern_dispatch.h: the channel loop of the pattern-sparse kernel as inline PTX.
+
+One macro per stride processes one pipeline stage (CK input channels) for one filter group and
+one lane's 4x4 output block.  Per input channel:
+
+    ld.shared        the group's 64-bit descriptor (count in bits 0-3, then 6-bit
+                     (slot << 3 | pattern) codes of the kept kernels, slots ascending)
+    ld.shared        the lane's input window, (4-1)*S+3 rows of (4-1)*S+3 floats; row r starts at
+                     a register advanced by one channel plane per channel, columns are immediates
+    per kept kernel:
+      ld.shared.v4   its four kept weights (consecutive in the compact storage, §3.4)
+      tcgen05.ld     the 16 accumulators of its filter slot from tensor memory
+      compare tree   three uniform branches select the body of its pattern
+      body           64 fma.rn.f32 whose tap operands are compile-time window registers (the
+                     four kept positions of the pattern, §3.2): nothing is decoded per element
+      tcgen05.st     the accumulators back
+
+Every branch is warp-uniform (bra.uni), so no convergence code surrounds the loop.  Taps are
+applied in ascending raster order for every output.  The library masks are the eight defaults
+(centre + 3 of the 4 edge neighbours; centre + one edge + its 2 flanking corners).
+
+Usage: gen_dispatch.py OUT.h
+"""
+import sys
+
+MASKS = [0x0B8, 0x0B2, 0x09A, 0x03A, 0x017, 0x059, 0x134, 0x1D0]
+STRIDES = [1, 2]          # every lane owns a 4x4 output block
+
+
+def taps(mask):
+    return [t for t in range(9) if (mask >> t) & 1]
+
+
+def macro(S):
+    RY = RX = 4
+    WY, WX = (RY - 1) * S + 3, (RX - 1) * S + 3
+    R = RY * RX
+    acc = ", ".join(f"a{i}" for i in range(R))
+    rows = ", ".join(f"rb{r}" for r in range(WY))
+    # operands: %0 channels, %1 descriptor address, %2 weights address, %3 window address of
+    # channel 0, %4 row pitch in bytes, %5 channel plane in bytes, %6 tensor-memory base
+    L = ["{",
+         ".reg .pred P;",
+         f".reg .b32 cl, cnt, code, ta, pat, va, da, t1, {rows};",
+         ".reg .b64 d, dd;",
+         f".reg .f32 x<{WY * WX}>, a<{R}>, w<4>;",
+         "mov.b32 cl, %0;",
+         "mov.b32 da, %1;",
+         "mov.b32 va, %2;",
+         "mov.b32 rb0, %3;"]
+    for r in range(1, WY):
+        L.append(f"add.u32 rb{r}, rb{r - 1}, %4;")
+    L += ["CL:",
+          "setp.eq.u32 P, cl, 0;",
+          "@P bra.uni CD;",
+          "ld.shared.u64 d, [da];",
+          "add.u32 da, da, 8;",
+          "cvt.u32.u64 cnt, d;",
+          "and.b32 cnt, cnt, 15;",
+          "setp.eq.u32 P, cnt, 0;",
+          "@P bra.uni CN;"]
+    # window: column 0 alone, then aligned groups of four
+    for r in range(WY):
+        base = r * WX
+        L.append(f"ld.shared.f32 x{base}, [rb{r}];")
+        c = 1
+        while c + 4 <= WX:
+            L.append(f"ld.shared.v4.f32 {{x{base + c}, x{base + c + 1}, x{base + c + 2}, x{base + c + 3}}}, "
+                     f"[rb{r}+{4 * c}];")
+            c += 4
+        while c < WX:
+            L.append(f"ld.shared.f32 x{base + c}, [rb{r}+{4 * c}];")
+            c += 1
+    L += ["shr.b64 dd, d, 4;",
+          "PL:",
+          "ld.shared.v4.f32 {w0, w1, w2, w3}, [va];",
+          "add.u32 va, va, 16;",
+          "cvt.u32.u64 code, dd;",
+          "shr.b64 dd, dd, 6;",
+          "and.b32 pat, code, 7;",
+          "and.b32 t1, code, 56;",
+          "shl.b32 t1, t1, 1;",
+          "add.u32 ta, %6, t1;",
+          f"tcgen05.ld.sync.aligned.32x32b.x{R}.b32 {{{acc}}}, [ta];",
+          "tcgen05.wait::ld.sync.aligned;",
+          "setp.lt.u32 P, pat, 4;", "@P bra.uni T03;",
+          "setp.lt.u32 P, pat, 6;", "@P bra.uni T45;",
+          "setp.eq.u32 P, pat, 6;", "@P bra.uni B6;", "bra.uni B7;",
+          "T45:", "setp.eq.u32 P, pat, 4;", "@P bra.uni B4;", "bra.uni B5;",
+          "T03:", "setp.lt.u32 P, pat, 2;", "@P bra.uni T01;",
+          "setp.eq.u32 P, pat, 2;", "@P bra.uni B2;", "bra.uni B3;",
+          "T01:", "setp.eq.u32 P, pat, 0;", "@P bra.uni B0;", "bra.uni B1;"]
+    for p, m in enumerate(MASKS):
+        L.append(f"B{p}:")
+        tp = taps(m)
+        for k in range(4):                   # tap-outer: 16 independent FMAs per tap
+            t = tp[k]
+            for r in range(RY):
+                for c in range(RX):
+                    wr = (r * S + t // 3) * WX + (c * S + t % 3)
+                    L.append(f"fma.rn.f32 a{r * RX + c}, w{k}, x{wr}, a{r * RX + c};")
+        if p != len(MASKS) - 1:
+            L.append("bra.uni BS;")
+    L += ["BS:",
+          f"tcgen05.st.sync.aligned.32x32b.x{R}.b32 [ta], {{{acc}}};",
+          "tcgen05.wait::st.sync.aligned;",
+          "sub.u32 cnt, cnt, 1;",
+          "setp.ne.u32 P, cnt, 0;",
+          "@P bra.uni PL;",
+          "CN:"]
+    for r in range(WY):
+        L.append(f"add.u32 rb{r}, rb{r}, %5;")
+    L += ["sub.u32 cl, cl, 1;",
+          "bra.uni CL;",
+          "CD:",
+          "}"]
+    body = "\\n\\t".join(L)
+    return (f"// stride {S}: 4x4 outputs per lane, {WY}x{WX} input window\n"
+            f"#define PP_STAGE_KERNELS_S{S}(nch, desc_addr, vals_addr, win_addr, pitch_b, plane_b, tbase) \\\n"
+            f'    asm volatile("{body}" :: "r"(nch), "r"(desc_addr), "r"(vals_addr), "r"(win_addr), '
+            f'"r"(pitch_b), "r"(plane_b), "r"(tbase) : "memory")\n')
+
+
+def main():
+    text = ["// generated by gen_dispatch.py -- do not edit", "#pragma once", ""]
+    for S in STRIDES:
+        text.append(macro(S))
+    with open(sys.argv[1], "w") as f:
+        f.write("\n".join(text))
+
+
+if __name__ == "__main__":
+    main()
