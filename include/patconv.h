@@ -128,6 +128,29 @@ int pp_bind_device(pp_handle h, void* dev_image, size_t bytes, void* stream);
 int pp_conv(pp_handle h, const void* x, int dtype, int N, int H, int W,
             const float* bias, int relu, void* y, void* stream);
 
+/* pp_conv with an optional caller-owned DEVICE workspace (16-byte aligned, no overlap with x or
+ * y).  When one pass over all input channels gives too few CTAs to fill the GPU (small images),
+ * the input channels are cut into KS contiguous ranges; each range's CTAs write fp32 partial
+ * sums into the workspace ([KS][N][Cout][Ho][Wo]) and a second kernel adds the ranges in order,
+ * adds the bias, applies ReLU and rounds to the output type.  The result is deterministic; it
+ * can differ from the single-pass sum in the last bits (fp32 summation order).  workspace ==
+ * NULL or too small for any split means a single pass.  The dense fast path only; other paths
+ * ignore the workspace.  Same errors as pp_conv, plus PP_ERR_ALIGN / PP_ERR_BUFFER for the
+ * workspace. */
+int pp_conv_ws(pp_handle h, const void* x, int dtype, int N, int H, int W, const float* bias,
+               int relu, void* y, void* workspace, size_t workspace_bytes, void* stream);
+
+/* Workspace bytes pp_conv_ws would use for this call shape with unlimited workspace (0 when it
+ * would not split).  Host-only. */
+int pp_conv_workspace_size(pp_handle h, int N, int H, int W, size_t* bytes);
+
+/* Launch plan of pp_conv_ws for a call shape and workspace size, for tests and tuning:
+ * info[0] = path (1 dense fast kernel, 2 depthwise kernel, 3 generic kernel); for path 1:
+ * info[1] channel splits KS, [2] workspace bytes used, [3] CTAs, [4..6] tile BY, BX, NB (4x4
+ * output blocks, images), [7] channels per stage, [8] filter groups and [9] spatial warps per
+ * CTA, [10] shared-memory bytes, [11] stages per CTA.  Writes min(n_info, 12) values.  Host-only. */
+int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info);
+
 /* 2x2 max-pool, stride 2, floor mode: y[n,c,i,j] = max x[n,c,2i+a,2j+b] (a,b in {0,1}).
  * The pooling between VGG blocks; x DEVICE [N][C][H][W], y DEVICE [N][C][H/2][W/2], same dtype,
  * no overlap.  Enqueue only. */

@@ -100,9 +100,30 @@ class Layer:
         s = self.stride
         return (N, self.cout, (H - 1) // s + 1, (W - 1) // s + 1)
 
+    PLAN_KEYS = ("path", "splits", "workspace_bytes", "ctas", "tile_by", "tile_bx", "tile_nb",
+                 "channels_per_stage", "filter_groups", "spatial_warps", "smem_bytes", "stages")
+
+    def plan(self, x_shape, workspace_bytes: int = 0) -> dict:
+        """Launch plan pp_conv_ws would use for input shape [N, C, H, W] (pp_conv_plan)."""
+        N, _, H, W = x_shape
+        info = (ctypes.c_int64 * 12)()
+        _lib.check("pp_conv_plan", _lib.load().pp_conv_plan(self._h, N, H, W, int(workspace_bytes),
+                                                            info, 12))
+        return dict(zip(self.PLAN_KEYS, (int(v) for v in info)))
+
+    def workspace_bytes(self, x_shape) -> int:
+        """Workspace the input-channel split would use for this input shape (0: no split)."""
+        N, _, H, W = x_shape
+        v = ctypes.c_size_t()
+        _lib.check("pp_conv_workspace_size", _lib.load().pp_conv_workspace_size(
+            self._h, N, H, W, ctypes.byref(v)))
+        return int(v.value)
+
     def conv(self, x: torch.Tensor, bias: Optional[torch.Tensor] = None, relu: bool = False,
-             out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
-        """y = ReLU?(conv3x3(x, W_hat, stride, pad 1) + bias) via pp_conv."""
+             out: Optional[torch.Tensor] = None, stream=None,
+             workspace: Optional[torch.Tensor] = None) -> torch.Tensor:
+        """y = ReLU?(conv3x3(x, W_hat, stride, pad 1) + bias) via pp_conv_ws (pp_conv when no
+        workspace tensor is given)."""
         if self._dev_buf is None:
             self.bind(x.device)
         if not x.is_cuda or x.dtype not in _DT or not x.is_contiguous() or x.dim() != 4:
@@ -122,9 +143,14 @@ class Layer:
                 raise ValueError("bias must be a contiguous CUDA float32 tensor of Cout values")
             bptr = ctypes.c_void_p(bias.data_ptr())
         N, _, H, W = x.shape
-        _lib.check("pp_conv", _lib.load().pp_conv(
+        wptr, wbytes = None, 0
+        if workspace is not None:
+            if not workspace.is_cuda or not workspace.is_contiguous():
+                raise ValueError("workspace must be a contiguous CUDA tensor")
+            wptr, wbytes = ctypes.c_void_p(workspace.data_ptr()), workspace.numel() * workspace.element_size()
+        _lib.check("pp_conv_ws", _lib.load().pp_conv_ws(
             self._h, ctypes.c_void_p(x.data_ptr()), _DT[x.dtype], N, H, W, bptr, int(bool(relu)),
-            ctypes.c_void_p(out.data_ptr()), _stream_ptr(stream, x.device)))
+            ctypes.c_void_p(out.data_ptr()), wptr, wbytes, _stream_ptr(stream, x.device)))
         return out
 
     def __del__(self):
@@ -156,8 +182,17 @@ def pp_pack(W, pattern_set: Optional[Sequence[int]] = None, keep_ratio: float = 
 
 
 def pp_conv(layer: Layer, x: torch.Tensor, bias: Optional[torch.Tensor], relu: bool,
-            y: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
-    return layer.conv(x, bias, relu, y, stream)
+            y: Optional[torch.Tensor] = None, stream=None,
+            workspace: Optional[torch.Tensor] = None) -> torch.Tensor:
+    return layer.conv(x, bias, relu, y, stream, workspace)
+
+
+def workspace_for(layers, x_shapes, device=None) -> Optional[torch.Tensor]:
+    """One device buffer large enough for the input-channel split of every (layer, shape)."""
+    n = max([lay.workspace_bytes(s) for lay, s in zip(layers, x_shapes)] + [0])
+    if n == 0:
+        return None
+    return torch.empty(n // 4 + 4, dtype=torch.float32, device=device or "cuda")
 
 
 def pp_maxpool2x2(x: torch.Tensor, out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:

@@ -108,7 +108,10 @@ struct TmParams {
     int WG, WS;                        // filter groups x spatial warps per CTA (WG * WS = 16)
     int BY, BX, NB;                    // spatial tile: BY x BX blocks (4x4 outputs) of NB images
     int tiles_x, tiles_y, tiles_n, n_fchunks;
-    int CK, n_chunks, maxk;            // channels per stage, stages, max kept kernels per group-stage
+    int CK, n_chunks, maxk;            // channels per stage, stages per CTA (max), max kept per group-stage
+    int KS, c_split;                   // input-channel splits; channels per split (multiple of CK)
+    float* ws;                         // KS > 1: fp32 partial sums [KS][N][Cout][Ho][Wo]
+    size_t ws_stride;                  // elements per split
     int IH, BWb;                       // staged rows / row width (floats) per (image, channel)
     int use_tma, vec_store;
     unsigned tma_bytes;                // bytes one TMA box delivers
@@ -222,12 +225,12 @@ __device__ __forceinline__ void stage_input_fallback(const TmParams& p, float* s
 template <typename TIn>
 __device__ __forceinline__ void produce_chunk(const TmParams& p, const CUtensorMap* tmap, unsigned char* smem,
                                               const uint32_t* s_kb, uint32_t full0, int k, int n0, int iy0,
-                                              int ix0, int g0, int lane) {
+                                              int ix0, int g0, int c_lo, int c_hi, int lane) {
     const int s = k % kStages;
     const int nkb = p.n_chunks + 1;
     unsigned char* st = smem + p.stage_off + (size_t)s * p.stage_bytes;
     const uint32_t fb = full0 + 8 * s;
-    const int c0 = k * p.CK, ckv = min(p.CK, p.C - c0);
+    const int c0 = c_lo + k * p.CK, ckv = min(p.CK, c_hi - c0);
     if (lane == 0) {
         mbar_arrive_expect_tx(fb, p.use_tma ? p.tma_bytes : 0u);
         if (p.use_tma) tma_load_4d(smem_u32(st), tmap, ix0, iy0, c0, n0, fb);
@@ -268,7 +271,11 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     const int tx = t % p.tiles_x;
     t /= p.tiles_x;
     const int ty = t % p.tiles_y;
-    const int tn = t / p.tiles_y;
+    t /= p.tiles_y;
+    const int tn = t % p.tiles_n;
+    const int ks = t / p.tiles_n;                         // input-channel split of this CTA
+    const int c_lo = ks * p.c_split, c_hi = min(p.C, c_lo + p.c_split);
+    const int nck = (c_hi - c_lo + p.CK - 1) / p.CK;       // channel chunks of this CTA
     const int n0 = tn * p.NB;
     const int oy0 = ty * p.BY * RY, ox0 = tx * p.BX * RX;
     const int iy0 = oy0 * S - 1, ix0 = ox0 * S - 4;     // stage origin: 1 halo row, 16-B aligned col
@@ -282,7 +289,7 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     }
     for (int i = threadIdx.x; i < p.WG * nkb; i += kThreadsTM) {
         const int wg = i / nkb, j = i - wg * nkb, g = g0 + wg;
-        s_kb[i] = g < p.G ? p.kofs[(size_t)g * p.C + min(j * p.CK, p.C)] : 0u;
+        s_kb[i] = g < p.G ? p.kofs[(size_t)g * p.C + min(c_lo + j * p.CK, c_hi)] : 0u;
     }
     if (warp == 0) {
         if (lane == 0) {
@@ -302,8 +309,9 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     const uint32_t tbase = *s_tmem;
 
     if (warp == 0) {   // prologue: fill every stage
-        const int first = min(kStages, p.n_chunks);
-        for (int k = 0; k < first; ++k) produce_chunk<TIn>(p, &tmap, smem, s_kb, full0, k, n0, iy0, ix0, g0, lane);
+        const int first = min(kStages, nck);
+        for (int k = 0; k < first; ++k)
+            produce_chunk<TIn>(p, &tmap, smem, s_kb, full0, k, n0, iy0, ix0, g0, c_lo, c_hi, lane);
         if (lane == 0) *s_issued = first;
     }
 
@@ -323,7 +331,7 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     const int plane = p.IH * p.BWb;
     const int in_off = active ? img * p.CK * plane + by * RY * S * p.BWb + bx * RX * S + 3 : 3;
 
-    for (int k = 0; k < p.n_chunks; ++k) {
+    for (int k = 0; k < nck; ++k) {
         const int s = k % kStages;
         if (!mbar_wait(full0 + 8 * s, (k / kStages) & 1, p.status, kStatusFullTimeout)) break;
         if (g < p.G) {
@@ -331,7 +339,7 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
             const uint32_t win_addr = smem_u32(reinterpret_cast<const float*>(st) + in_off);
             const uint32_t desc_addr = smem_u32(reinterpret_cast<const uint64_t*>(st + p.desc_off) + wg * p.CK);
             const uint32_t vals_addr = smem_u32(reinterpret_cast<const float4*>(st + p.vals_off) + wg * p.maxk);
-            const int ckv = min(p.CK, p.C - k * p.CK);
+            const int ckv = min(p.CK, c_hi - c_lo - k * p.CK);
             if constexpr (S == 1) {
                 PP_STAGE_KERNELS_S1(ckv, desc_addr, vals_addr, win_addr, 4 * p.BWb, 4 * plane, tw);
             } else {
@@ -348,9 +356,9 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
         old = __shfl_sync(0xffffffffu, old, 0);
         if (old == kCompute - 1) {
             if (lane == 0) s_cnt[s] = 0;
-            if (k + kStages < p.n_chunks) {
+            if (k + kStages < nck) {
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                produce_chunk<TIn>(p, &tmap, smem, s_kb, full0, k + kStages, n0, iy0, ix0, g0, lane);
+                produce_chunk<TIn>(p, &tmap, smem, s_kb, full0, k + kStages, n0, iy0, ix0, g0, c_lo, c_hi, lane);
                 if (lane == 0) atomicMax(s_issued, (uint32_t)(k + kStages + 1));
             }
         }
@@ -370,6 +378,24 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
             if (g >= p.G || !active || n >= p.N) continue;
             const uint32_t co = p.perm[g * kF + f];
             if (co == kPadSlot) continue;
+            if (p.KS > 1) {   // raw partial sums of this split; bias, ReLU and rounding come later
+                float* wc = p.ws + (size_t)ks * p.ws_stride + ((size_t)n * p.Cout + co) * p.Ho * p.Wo;
+#pragma unroll
+                for (int r = 0; r < RY; ++r) {
+                    const int oy = oyb + r;
+                    if (oy >= p.Ho) break;
+                    float* wr = wc + (size_t)oy * p.Wo;
+                    if ((p.Wo % 4) == 0 && oxb + RX <= p.Wo) {
+                        *reinterpret_cast<float4*>(wr + oxb) =
+                            make_float4(a[r * RX], a[r * RX + 1], a[r * RX + 2], a[r * RX + 3]);
+                    } else {
+#pragma unroll
+                        for (int c = 0; c < RX; ++c)
+                            if (oxb + c < p.Wo) wr[oxb + c] = a[r * RX + c];
+                    }
+                }
+                continue;
+            }
             const float b = p.bias ? p.bias[co] : 0.0f;
             TOut* yc = y + ((size_t)n * p.Cout + co) * p.Ho * p.Wo;
 #pragma unroll
@@ -627,9 +653,115 @@ TileChoice choose_tile(int N, int Ho, int Wo, int S, int lanes, int n_fchunks, i
 
 size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
+// Launch plan of the pattern-sparse kernel for one call shape (shared by the workspace query,
+// the plan query and the launch, so all three agree).
+struct Plan {
+    int WG = 0, WS = 0, n_fchunks = 0;
+    TileChoice tile;
+    int tiles_x = 0, tiles_y = 0, tiles_n = 0;
+    int CK = 0, n_chunks = 0, maxk = 0, KS = 1, c_split = 0;
+    size_t stage_bytes = 0, kb_bytes = 0, smem = 0;
+    long long ctas = 0;           // CTAs of one split
+    size_t ws_bytes = 0;          // workspace the chosen split needs (0 without a split)
+};
+
+int make_plan(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out) {
+    Plan pl;
+    const int S = L->stride;
+    const int Ho = (H - 1) / S + 1, Wo = (W - 1) / S + 1;
+    int wg = 1;
+    while (wg < L->G && wg < kCompute) wg *= 2;
+    pl.WG = wg;
+    pl.WS = kCompute / wg;
+    pl.n_fchunks = (L->G + wg - 1) / wg;
+    const int C = L->cin_g;
+    pl.tile = choose_tile(N, Ho, Wo, S, 32 * pl.WS, pl.n_fchunks, C);
+    if (pl.tile.IH == 0) return PP_ERR_SHAPE;
+    pl.tiles_x = ((Wo + 3) / 4 + pl.tile.BX - 1) / pl.tile.BX;
+    pl.tiles_y = ((Ho + 3) / 4 + pl.tile.BY - 1) / pl.tile.BY;
+    pl.tiles_n = (N + pl.tile.NB - 1) / pl.tile.NB;
+    pl.ctas = (long long)pl.tiles_n * pl.tiles_y * pl.tiles_x * pl.n_fchunks;
+
+    // channels per stage: the largest that fits three stages in shared memory
+    auto maxk_for = [&](int ck) {
+        uint32_t m = 0;
+        for (int g = 0; g < L->G; ++g)
+            for (int c0 = 0; c0 < C; c0 += ck) {
+                const size_t b = (size_t)g * C;
+                m = std::max(m, L->kofs[b + std::min(c0 + ck, C)] - L->kofs[b + c0]);
+            }
+        return (int)m;
+    };
+    auto layout = [&](int ck, int maxk, size_t* stage_bytes, size_t* kb_bytes) {
+        const size_t in_b = align_up((size_t)pl.tile.NB * ck * pl.tile.IH * pl.tile.BWb * 4, 128);
+        const size_t desc_b = align_up((size_t)pl.WG * ck * 8, 16);
+        const size_t vals_b = (size_t)pl.WG * std::max(maxk, 1) * 16;
+        *stage_bytes = align_up(in_b + desc_b + vals_b, 128);
+        const int nch = (C + ck - 1) / ck;
+        *kb_bytes = (size_t)pl.WG * (nch + 1) * 4;
+        return align_up(64 + *kb_bytes, 128) + kStages * *stage_bytes;
+    };
+    int ck = std::min(C, 64);
+    for (;; --ck) {
+        if (ck < 1) return PP_ERR_SHAPE;
+        if ((C + ck - 1) / ck > kMaxChunks) return PP_ERR_SHAPE;
+        pl.maxk = maxk_for(ck);
+        pl.smem = layout(ck, pl.maxk, &pl.stage_bytes, &pl.kb_bytes);
+        if (pl.smem <= 200 * 1024) break;
+    }
+    pl.CK = ck;
+    pl.maxk = std::max(pl.maxk, 1);
+    const int nck_total = (C + ck - 1) / ck;
+
+    // input-channel split: when one split gives too few CTAs for the SMs, cut the channel range
+    // into KS parts (whole chunks each) if the caller's workspace holds the partial sums.
+    // Cost in channel-stage units: waves x (chunks per split + start-up) + a reduction term.
+    const size_t out_elems = (size_t)N * L->cout * Ho * Wo;
+    const long long sms = sm_count();
+    int best_ks = 1;
+    double best_cost = 1e300;
+    for (int ksp = 1; ksp <= std::min(8, nck_total); ++ksp) {
+        const int per = (nck_total + ksp - 1) / ksp;
+        const int used = (nck_total + per - 1) / per;
+        if (used != ksp) continue;                       // every split must get chunks
+        if (ksp > 1 && ws_avail < (size_t)ksp * out_elems * 4) break;
+        const long long waves = (pl.ctas * ksp + sms - 1) / sms;
+        const double cost = (double)waves * (per + 2.0) + (ksp > 1 ? 0.5 * ksp : 0.0);
+        if (cost < best_cost - 1e-9) {
+            best_cost = cost;
+            best_ks = ksp;
+        }
+    }
+    pl.KS = best_ks;
+    const int per = (nck_total + best_ks - 1) / best_ks;
+    pl.c_split = per * ck;
+    pl.n_chunks = std::min(per, nck_total);
+    pl.ws_bytes = best_ks > 1 ? (size_t)best_ks * out_elems * 4 : 0;
+    *out = pl;
+    return PP_OK;
+}
+
+// Sum the KS partial planes in split order, + bias, ReLU, round to the output type.
+template <typename T>
+__global__ void splitk_reduce(const float* __restrict__ ws, T* __restrict__ y, const float* __restrict__ bias,
+                              int KS, size_t stride, int Cout, int HoWo, int relu) {
+    const size_t total = stride;
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total; i += (size_t)gridDim.x * blockDim.x) {
+        float a = ws[i];
+        for (int k = 1; k < KS; ++k) a += ws[(size_t)k * stride + i];
+        const int co = (int)((i / (size_t)HoWo) % (size_t)Cout);
+        a += bias ? bias[co] : 0.0f;
+        y[i] = from_f32<T>(relu ? fmaxf(a, 0.0f) : a);
+    }
+}
+
 template <int S, typename T>
 int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int relu, int N, int H, int W, int Ho,
-              int Wo, cudaStream_t st) {
+              int Wo, void* ws, size_t ws_bytes, cudaStream_t st) {
+    Plan pl;
+    const int rc = make_plan(L, N, H, W, ws ? ws_bytes : 0, &pl);
+    if (rc != PP_OK) return rc;
+    if (pl.KS > 1 && reinterpret_cast<uintptr_t>(ws) % 16 != 0) return PP_ERR_ALIGN;
     TmParams p{};
     p.x = x;
     p.y = y;
@@ -650,62 +782,32 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
     p.Wo = Wo;
     p.G = L->G;
     p.relu = relu;
-    int wg = 1;
-    while (wg < L->G && wg < kCompute) wg *= 2;
-    p.WG = wg;
-    p.WS = kCompute / wg;
-    p.n_fchunks = (L->G + wg - 1) / wg;
-    const TileChoice t = choose_tile(N, Ho, Wo, S, 32 * p.WS, p.n_fchunks, L->cin_g);
-    if (t.IH == 0) return PP_ERR_SHAPE;
-    p.BY = t.BY;
-    p.BX = t.BX;
-    p.NB = t.NB;
-    p.IH = t.IH;
-    p.BWb = t.BWb;
-    p.tiles_x = ((Wo + 3) / 4 + t.BX - 1) / t.BX;
-    p.tiles_y = ((Ho + 3) / 4 + t.BY - 1) / t.BY;
-    p.tiles_n = (N + t.NB - 1) / t.NB;
+    p.WG = pl.WG;
+    p.WS = pl.WS;
+    p.n_fchunks = pl.n_fchunks;
+    p.BY = pl.tile.BY;
+    p.BX = pl.tile.BX;
+    p.NB = pl.tile.NB;
+    p.IH = pl.tile.IH;
+    p.BWb = pl.tile.BWb;
+    p.tiles_x = pl.tiles_x;
+    p.tiles_y = pl.tiles_y;
+    p.tiles_n = pl.tiles_n;
+    p.CK = pl.CK;
+    p.n_chunks = pl.n_chunks;
+    p.maxk = pl.maxk;
+    p.KS = pl.KS;
+    p.c_split = pl.c_split;
+    p.ws = static_cast<float*>(ws);
+    p.ws_stride = (size_t)N * L->cout * Ho * Wo;
     const int C = L->cin_g;
     const size_t es = sizeof(T);
     p.use_tma = es == 4 && (W * es) % 16 == 0 && reinterpret_cast<uintptr_t>(x) % 16 == 0 && encode_tiled() != nullptr;
-
-    // channels per stage: the largest that fits three stages in shared memory
-    auto maxk_for = [&](int ck) {
-        uint32_t m = 0;
-        for (int g = 0; g < L->G; ++g)
-            for (int c0 = 0; c0 < C; c0 += ck) {
-                const size_t b = (size_t)g * C;
-                m = std::max(m, L->kofs[b + std::min(c0 + ck, C)] - L->kofs[b + c0]);
-            }
-        return (int)m;
-    };
-    auto layout = [&](int ck, int maxk, size_t* stage_bytes, size_t* kb_bytes) {
-        const size_t in_b = align_up((size_t)p.NB * ck * p.IH * p.BWb * 4, 128);
-        const size_t desc_b = align_up((size_t)p.WG * ck * 8, 16);
-        const size_t vals_b = (size_t)p.WG * std::max(maxk, 1) * 16;
-        *stage_bytes = align_up(in_b + desc_b + vals_b, 128);
-        const int nch = (C + ck - 1) / ck;
-        *kb_bytes = (size_t)p.WG * (nch + 1) * 4;
-        return align_up(64 + *kb_bytes, 128) + kStages * *stage_bytes;
-    };
-    int ck = std::min(C, 64);
-    int maxk = 0;
-    size_t stage_bytes = 0, kb_bytes = 0, total = 0;
-    for (;; --ck) {
-        if (ck < 1) return PP_ERR_SHAPE;
-        if ((C + ck - 1) / ck > kMaxChunks) return PP_ERR_SHAPE;
-        maxk = maxk_for(ck);
-        total = layout(ck, maxk, &stage_bytes, &kb_bytes);
-        if (total <= 200 * 1024) break;
-    }
-    p.CK = ck;
-    p.n_chunks = (C + ck - 1) / ck;
-    p.maxk = std::max(maxk, 1);
     p.kb_off = 64;
-    p.stage_off = (unsigned)align_up(64 + kb_bytes, 128);
-    p.stage_bytes = (unsigned)stage_bytes;
-    p.desc_off = (unsigned)align_up((size_t)p.NB * ck * p.IH * p.BWb * 4, 128);
-    p.vals_off = p.desc_off + (unsigned)align_up((size_t)p.WG * ck * 8, 16);
+    p.stage_off = (unsigned)align_up(64 + pl.kb_bytes, 128);
+    p.stage_bytes = (unsigned)pl.stage_bytes;
+    p.desc_off = (unsigned)align_up((size_t)p.NB * p.CK * p.IH * p.BWb * 4, 128);
+    p.vals_off = p.desc_off + (unsigned)align_up((size_t)p.WG * p.CK * 8, 16);
     p.vec_store = (Wo % 4 == 0) && (reinterpret_cast<uintptr_t>(y) % (4 * es)) == 0;
 
     CUtensorMap tmap;
@@ -713,22 +815,29 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
     if (p.use_tma) {
         const cuuint64_t dims[4] = {(cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)C, (cuuint64_t)N};
         const cuuint64_t strides[3] = {(cuuint64_t)W * es, (cuuint64_t)H * W * es, (cuuint64_t)C * H * W * es};
-        const cuuint32_t box[4] = {(cuuint32_t)p.BWb, (cuuint32_t)p.IH, (cuuint32_t)ck, (cuuint32_t)p.NB};
+        const cuuint32_t box[4] = {(cuuint32_t)p.BWb, (cuuint32_t)p.IH, (cuuint32_t)p.CK, (cuuint32_t)p.NB};
         const cuuint32_t estr[4] = {1, 1, 1, 1};
         const CUresult r = encode_tiled()(&tmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<void*>(x), dims,
                                           strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
                                           CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
                                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         if (r != CUDA_SUCCESS) p.use_tma = 0;
-        p.tma_bytes = (unsigned)((size_t)p.BWb * p.IH * ck * p.NB * 4);
+        p.tma_bytes = (unsigned)((size_t)p.BWb * p.IH * p.CK * p.NB * 4);
     }
     auto kern = pconv_tm<S, T>;
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)total) != cudaSuccess)
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem) != cudaSuccess)
         return PP_ERR_CUDA;
-    const long long ctas = (long long)p.tiles_n * p.tiles_y * p.tiles_x * p.n_fchunks;
+    const long long ctas = pl.ctas * pl.KS;
     if (ctas > INT_MAX) return PP_ERR_SHAPE;
-    kern<<<(unsigned)ctas, kThreadsTM, total, st>>>(p, tmap);
-    return cudaGetLastError() == cudaSuccess ? PP_OK : PP_ERR_CUDA;
+    kern<<<(unsigned)ctas, kThreadsTM, pl.smem, st>>>(p, tmap);
+    if (cudaGetLastError() != cudaSuccess) return PP_ERR_CUDA;
+    if (pl.KS > 1) {
+        const size_t total = p.ws_stride;
+        const int blocks = (int)std::max<size_t>(1, std::min<size_t>((total + 255) / 256, (size_t)sm_count() * 16));
+        splitk_reduce<T><<<blocks, 256, 0, st>>>(p.ws, static_cast<T*>(y), bias, pl.KS, total, L->cout, Ho * Wo, relu);
+        if (cudaGetLastError() != cudaSuccess) return PP_ERR_CUDA;
+    }
+    return PP_OK;
 }
 
 template <typename T>
@@ -793,8 +902,10 @@ int pp_bind_device(pp_handle h, void* dev_image, size_t bytes, void* stream) {
     return PP_OK;
 }
 
-int pp_conv(pp_handle h, const void* x, int dtype, int N, int H, int W, const float* bias, int relu, void* y,
-            void* stream) {
+namespace {
+
+int validate_conv(pp_handle h, const void* x, int dtype, int N, int H, int W, const float* bias, int relu,
+                  const void* y) {
     if (!h) return PP_ERR_NULL;
     if (!h->dev) return PP_ERR_NOT_BOUND;
     if (dtype != PP_F32 && dtype != PP_F16) return PP_ERR_DTYPE;
@@ -805,11 +916,21 @@ int pp_conv(pp_handle h, const void* x, int dtype, int N, int H, int W, const fl
     const int C = h->depthwise ? h->cout : h->cin_g;
     const int Ho = (H - 1) / h->stride + 1, Wo = (W - 1) / h->stride + 1;
     const size_t es = dtype == PP_F32 ? 4 : 2;
-    const size_t xb = (size_t)N * C * H * W * es, yb = (size_t)N * h->cout * Ho * Wo * es;
     if ((size_t)N * C * H * W >= (1ull << 40) || (size_t)N * h->cout * Ho * Wo >= (1ull << 40)) return PP_ERR_SHAPE;
+    const size_t xb = (size_t)N * C * H * W * es, yb = (size_t)N * h->cout * Ho * Wo * es;
     if (reinterpret_cast<uintptr_t>(x) % es || reinterpret_cast<uintptr_t>(y) % es) return PP_ERR_ALIGN;
     if (bias && reinterpret_cast<uintptr_t>(bias) % 4) return PP_ERR_ALIGN;
     if (overlaps(x, xb, y, yb)) return PP_ERR_BUFFER;
+    return PP_OK;
+}
+
+}  // namespace
+
+int pp_conv_ws(pp_handle h, const void* x, int dtype, int N, int H, int W, const float* bias, int relu, void* y,
+               void* workspace, size_t workspace_bytes, void* stream) {
+    const int v = validate_conv(h, x, dtype, N, H, W, bias, relu, y);
+    if (v != PP_OK || N == 0) return v;
+    const int Ho = (H - 1) / h->stride + 1, Wo = (W - 1) / h->stride + 1;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const bool f16 = dtype == PP_F16;
     if (!h->fast) {
@@ -820,11 +941,59 @@ int pp_conv(pp_handle h, const void* x, int dtype, int N, int H, int W, const fl
         return f16 ? launch_depthwise<__half>(h, x, y, bias, relu, N, H, W, Ho, Wo, st)
                    : launch_depthwise<float>(h, x, y, bias, relu, N, H, W, Ho, Wo, st);
     }
+    if (workspace) {
+        const size_t es = f16 ? 2 : 4;
+        const int C = h->cin_g;
+        if (overlaps(workspace, workspace_bytes, x, (size_t)N * C * H * W * es) ||
+            overlaps(workspace, workspace_bytes, y, (size_t)N * h->cout * Ho * Wo * es))
+            return PP_ERR_BUFFER;
+    }
     if (h->stride == 1)
-        return f16 ? launch_tm<1, __half>(h, x, y, bias, relu, N, H, W, Ho, Wo, st)
-                   : launch_tm<1, float>(h, x, y, bias, relu, N, H, W, Ho, Wo, st);
-    return f16 ? launch_tm<2, __half>(h, x, y, bias, relu, N, H, W, Ho, Wo, st)
-               : launch_tm<2, float>(h, x, y, bias, relu, N, H, W, Ho, Wo, st);
+        return f16 ? launch_tm<1, __half>(h, x, y, bias, relu, N, H, W, Ho, Wo, workspace, workspace_bytes, st)
+                   : launch_tm<1, float>(h, x, y, bias, relu, N, H, W, Ho, Wo, workspace, workspace_bytes, st);
+    return f16 ? launch_tm<2, __half>(h, x, y, bias, relu, N, H, W, Ho, Wo, workspace, workspace_bytes, st)
+               : launch_tm<2, float>(h, x, y, bias, relu, N, H, W, Ho, Wo, workspace, workspace_bytes, st);
+}
+
+int pp_conv(pp_handle h, const void* x, int dtype, int N, int H, int W, const float* bias, int relu, void* y,
+            void* stream) {
+    return pp_conv_ws(h, x, dtype, N, H, W, bias, relu, y, nullptr, 0, stream);
+}
+
+int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info) {
+    if (!h || !info) return PP_ERR_NULL;
+    if (N < 1 || H < 1 || W < 1 || n_info < 1) return PP_ERR_SHAPE;
+    int64_t v[12] = {0};
+    if (!h->fast || h->depthwise) {
+        v[0] = h->fast ? 2 : 3;   // depthwise kernel / generic kernel: no plan, no workspace
+    } else {
+        Plan pl;
+        const int rc = make_plan(h, N, H, W, workspace_bytes, &pl);
+        if (rc != PP_OK) return rc;
+        v[0] = 1;
+        v[1] = pl.KS;
+        v[2] = (int64_t)pl.ws_bytes;
+        v[3] = pl.ctas * pl.KS;
+        v[4] = pl.tile.BY;
+        v[5] = pl.tile.BX;
+        v[6] = pl.tile.NB;
+        v[7] = pl.CK;
+        v[8] = pl.WG;
+        v[9] = pl.WS;
+        v[10] = (int64_t)pl.smem;
+        v[11] = pl.n_chunks;
+    }
+    for (int i = 0; i < n_info && i < 12; ++i) info[i] = v[i];
+    return PP_OK;
+}
+
+int pp_conv_workspace_size(pp_handle h, int N, int H, int W, size_t* bytes) {
+    if (!h || !bytes) return PP_ERR_NULL;
+    int64_t info[3];
+    const int rc = pp_conv_plan(h, N, H, W, (size_t)-1, info, 3);
+    if (rc != PP_OK) return rc;
+    *bytes = info[0] == 1 ? (size_t)info[2] : 0;
+    return PP_OK;
 }
 
 int pp_device_status(int clear, unsigned int* status) {

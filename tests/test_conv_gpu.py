@@ -25,7 +25,7 @@ def _np_dt(dt):
 
 
 def run_gpu(W, x, b, keep, stride=1, relu=True, depthwise=False, dtype=torch.float32, masks=None,
-            guard=0, to_host=True):
+            guard=0, to_host=True, ws=False, ws_bytes=None):
     """Pack + bind + pp_conv; x host array; returns the output (host float64 unless
     ``to_host=False``) and the layer."""
     layer = api.pp_pack(W, masks, keep, W.shape[0] if depthwise else 1, stride)
@@ -40,7 +40,12 @@ def run_gpu(W, x, b, keep, stride=1, relu=True, depthwise=False, dtype=torch.flo
         y = buf[guard:guard + n].view(shape)
     else:
         y = torch.empty(shape, dtype=dtype, device=dev)
-    layer.conv(xt, bt, relu, y)
+    wt = None
+    if ws:
+        nb = layer.workspace_bytes(x.shape) if ws_bytes is None else ws_bytes
+        if nb:
+            wt = torch.full((nb // 4,), float("nan"), dtype=torch.float32, device=dev)
+    layer.conv(xt, bt, relu, y, workspace=wt)
     torch.cuda.synchronize()
     if guard:
         g = torch.cat([buf[:guard], buf[guard + n:]])
@@ -158,11 +163,13 @@ def test_maxpool_exact(dtype):
 
 # --------------------------------------------------------------------------- workloads
 
-def _sampled_check(L, n, dtype=torch.float32, samples=(0, -1)):
-    """Full-batch launch (the benchmark's launch configuration), oracle on sampled images."""
+def _sampled_check(L, n, dtype=torch.float32, samples=(0, -1), ws=True):
+    """Full-batch launch with the workspace the benchmark gives it (its launch configuration),
+    oracle on sampled images."""
     x = WL.layer_input(L, n, relu=not L.depthwise, dtype=_np_dt(dtype))
     W, b = WL.weights(L), WL.bias(L)
-    y, _ = run_gpu(W, x, b, L.keep, L.stride, True, L.depthwise, dtype, guard=256, to_host=False)
+    y, _ = run_gpu(W, x, b, L.keep, L.stride, True, L.depthwise, dtype, guard=256, to_host=False,
+                   ws=ws)
     assert bool(torch.isfinite(y).all())
     idx = [s % n for s in samples]
     ref, den = oracle(W, x[idx], b, L.keep, L.stride, True, L.depthwise)
@@ -204,3 +211,56 @@ def test_vgg16_chained_network():
             assert np.array_equal(p.cpu().numpy(), OC.maxpool2x2(y.cpu().numpy()))
             y = p
         x = y
+
+
+# --------------------------------------------------------------------------- channel split
+
+def _split_case():
+    L = WL.vgg16()[10]                                    # 512 -> 512 at 14x14
+    return L, WL.weights(L), WL.bias(L), WL.layer_input(L, 32)
+
+
+def test_split_is_planned_for_small_images():
+    L, W, b, x = _split_case()
+    lay = api.pp_pack(W, None, L.keep)
+    plan = lay.plan(x.shape, lay.workspace_bytes(x.shape))
+    assert plan["path"] == 1 and plan["splits"] > 1
+    assert lay.plan(x.shape, 0)["splits"] == 1
+    big = api.pp_pack(WL.weights(WL.vgg16()[1]), None, 0.3)
+    assert big.plan((32, 64, 224, 224), 1 << 34)["splits"] == 1
+
+
+def test_split_matches_oracle_single_pass_and_is_deterministic():
+    L, W, b, x = _split_case()
+    y_split, lay = run_gpu(W, x, b, L.keep, ws=True)
+    y_split2, _ = run_gpu(W, x, b, L.keep, ws=True)
+    y_one, _ = run_gpu(W, x, b, L.keep, ws=False)
+    assert np.array_equal(y_split, y_split2)
+    ref, den = oracle(W, x[[0, 31]], b, L.keep)
+    assert OC.max_norm_err(y_split[[0, 31]], ref, den) <= 1e-4
+    d = np.abs(y_split - y_one) / np.maximum(np.abs(y_one), 1e-3)
+    assert float(np.max(d)) < 1e-3                       # only fp32 summation order differs
+
+
+def test_split_with_small_workspace_and_fp16():
+    L, W, b, x = _split_case()
+    lay = api.pp_pack(W, None, L.keep)
+    need = lay.workspace_bytes(x.shape)
+    out_bytes = 32 * 512 * 14 * 14 * 4
+    assert need >= 2 * out_bytes
+    # room for two splits only: still correct
+    y2, _ = run_gpu(W, x, b, L.keep, ws=True, ws_bytes=2 * out_bytes)
+    ref, den = oracle(W, x[[5]], b, L.keep)
+    assert OC.max_norm_err(y2[[5]], ref, den) <= 1e-4
+    # too small for any split: single pass
+    y1, _ = run_gpu(W, x, b, L.keep, ws=True, ws_bytes=out_bytes)
+    assert OC.max_norm_err(y1[[5]], ref, den) <= 1e-4
+    xh = x.astype(np.float16)
+    yh, _ = run_gpu(W, xh, b, L.keep, ws=True, dtype=torch.float16)
+    ref, den = oracle(W, xh[[3]], b, L.keep)
+    assert OC.max_norm_err(yh[[3]], ref, den) <= 2e-3
+
+
+@pytest.mark.parametrize("idx", [13, 14, 15])
+def test_resnet50_split_layers_without_workspace(idx):
+    _sampled_check(WL.resnet50_3x3()[idx], 64, ws=False)
