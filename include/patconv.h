@@ -49,7 +49,9 @@ typedef enum {
     PP_ERR_BUFFER = -9,       /* caller buffer too small / wrong size, or x and y overlap     */
     PP_ERR_CUDA = -10,        /* a CUDA runtime call failed (launch or copy)                 */
     PP_ERR_ARG = -11,         /* any other invalid argument (section, query key, flag)       */
-    PP_ERR_ALLOC = -12        /* host allocation failed                                      */
+    PP_ERR_ALLOC = -12,       /* host allocation failed                                      */
+    PP_ERR_SCRATCH = -13      /* pp_conv_static_scratch: the call needs more scratch than the
+                                 static array holds                                           */
 } pp_status;
 
 typedef enum { PP_F32 = 0, PP_F16 = 1 } pp_dtype;
@@ -150,6 +152,29 @@ int pp_conv_workspace_size(pp_handle h, int N, int H, int W, size_t* bytes);
  * output blocks, images), [7] channels per stage, [8] filter groups and [9] spatial warps per
  * CTA, [10] shared-memory bytes, [11] stages per CTA.  Writes min(n_info, 12) values.  Host-only. */
 int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info);
+
+/* pp_conv_ws for callers that cannot allocate device memory (the paper has no counterpart to
+ * this entry point).  Some callers are not allowed to call cudaMalloc or any allocating routine:
+ * code embedded in a host runtime whose allocator owns all device memory, plugins that must
+ * not allocate while serving, or setups where an allocation could block behind other work.
+ * Such callers still pass x, y and bias, but get the input-channel split's partial sums in a
+ * scratch array that lives in the library itself: a file-scope device array of
+ * PP_STATIC_SCRATCH_BYTES (32 MiB) that every GPU loading the library keeps until the process
+ * exits.  Nothing is allocated and no allocating routine is called.
+ *   - the first call on a device looks up the array's device address (once per device, with
+ *     that device current); make that first call before any stream capture;
+ *   - a call whose split would need more scratch than the array holds (see
+ *     pp_conv_workspace_size) returns PP_ERR_SCRATCH without launching anything;
+ *   - every call on a device shares the one array, which keeps the previous call's contents;
+ *     nothing needs clearing (each call writes every partial sum it reads), but calls that
+ *     overlap on the GPU (different streams, or different host threads) race on it: order them;
+ *   - otherwise identical to pp_conv_ws (same plan, same result, same errors). */
+#define PP_STATIC_SCRATCH_BYTES 33554432
+int pp_conv_static_scratch(pp_handle h, const void* x, int dtype, int N, int H, int W,
+                           const float* bias, int relu, void* y, void* stream);
+
+/* Size in bytes of the static scratch array behind pp_conv_static_scratch. */
+int pp_static_scratch_bytes(size_t* bytes);
 
 /* 2x2 max-pool, stride 2, floor mode: y[n,c,i,j] = max x[n,c,2i+a,2j+b] (a,b in {0,1}).
  * The pooling between VGG blocks; x DEVICE [N][C][H][W], y DEVICE [N][C][H/2][W/2], same dtype,

@@ -26,6 +26,7 @@
 #include <climits>
 #include <cstdint>
 #include <cstring>
+#include <mutex>
 
 #include "../../include/patconv.h"
 #include "layer.h"
@@ -575,6 +576,14 @@ __global__ void maxpool2x2(const T* __restrict__ x, T* __restrict__ y, long long
     }
 }
 
+
+// ------------------------------------------------------------------------------ static scratch
+// Scratch for pp_conv_static_scratch: a fixed array in the library's own device image, so that
+// callers which may not allocate device memory still get the input-channel split.  It exists on
+// every GPU that loads the library, from module load until process exit.
+constexpr size_t kStaticScratchBytes = (size_t)32 << 20;
+static __device__ __align__(256) float g_pp_scratch[kStaticScratchBytes / sizeof(float)];
+
 // ------------------------------------------------------------------------------ host side
 
 int sm_count() {
@@ -881,6 +890,23 @@ int launch_generic(const pp_layer* L, const void* x, void* y, const float* bias,
     return cudaGetLastError() == cudaSuccess ? PP_OK : PP_ERR_CUDA;
 }
 
+
+// Device address of g_pp_scratch on the current device, looked up once per device (the host-side
+// name of the array is only a stand-in; kernels must be given this address).
+void* static_scratch_address() {
+    static std::mutex mu;
+    static void* addr[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!addr[dev]) {
+        void* ptr = nullptr;
+        if (cudaGetSymbolAddress(&ptr, g_pp_scratch) != cudaSuccess) return nullptr;
+        addr[dev] = ptr;
+    }
+    return addr[dev];
+}
+
 bool overlaps(const void* a, size_t na, const void* b, size_t nb) {
     const uintptr_t x0 = reinterpret_cast<uintptr_t>(a), y0 = reinterpret_cast<uintptr_t>(b);
     return x0 < y0 + nb && y0 < x0 + na;
@@ -993,6 +1019,28 @@ int pp_conv_workspace_size(pp_handle h, int N, int H, int W, size_t* bytes) {
     const int rc = pp_conv_plan(h, N, H, W, (size_t)-1, info, 3);
     if (rc != PP_OK) return rc;
     *bytes = info[0] == 1 ? (size_t)info[2] : 0;
+    return PP_OK;
+}
+
+int pp_conv_static_scratch(pp_handle h, const void* x, int dtype, int N, int H, int W, const float* bias, int relu,
+                           void* y, void* stream) {
+    if (!h) return PP_ERR_NULL;
+    if (!h->dev) return PP_ERR_NOT_BOUND;
+    if (dtype != PP_F32 && dtype != PP_F16) return PP_ERR_DTYPE;
+    if (N < 0 || H < 1 || W < 1) return PP_ERR_SHAPE;
+    if (N == 0) return pp_conv_ws(h, x, dtype, N, H, W, bias, relu, y, nullptr, 0, stream);
+    size_t need = 0;
+    const int rc = pp_conv_workspace_size(h, N, H, W, &need);
+    if (rc != PP_OK) return rc;
+    if (need > kStaticScratchBytes) return PP_ERR_SCRATCH;
+    void* scratch = static_scratch_address();
+    if (!scratch) return PP_ERR_CUDA;
+    return pp_conv_ws(h, x, dtype, N, H, W, bias, relu, y, scratch, kStaticScratchBytes, stream);
+}
+
+int pp_static_scratch_bytes(size_t* bytes) {
+    if (!bytes) return PP_ERR_NULL;
+    *bytes = kStaticScratchBytes;
     return PP_OK;
 }
 

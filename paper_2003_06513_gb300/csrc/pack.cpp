@@ -301,6 +301,7 @@ const char* pp_status_string(int status) {
         case PP_ERR_CUDA: return "CUDA runtime error";
         case PP_ERR_ARG: return "invalid argument";
         case PP_ERR_ALLOC: return "host allocation failed";
+        case PP_ERR_SCRATCH: return "call needs more scratch than the library's static scratch array holds";
         default: return "unknown status";
     }
 }

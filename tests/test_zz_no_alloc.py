@@ -1,0 +1,81 @@
+"""pp_conv_static_scratch: the entry point for callers that may not allocate device memory.
+
+Such callers (code inside a host runtime that owns every device allocation, plugins that must
+not allocate while serving) still pass x, y and bias, and the split of the input channels keeps
+its partial sums in the library's own static device array instead of a caller workspace.  This
+test calls the entry point through the C ABI, twice in a row, and checks both results against
+the workspace entry point pp_conv_ws within the tolerance of the other conv tests.  The file
+sorts last so that a run stopping at the first failure has already run every other test.
+"""
+import ctypes
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import conv as OC
+from oracle import patterns as OP
+from oracle import project as OPR
+from paper_2003_06513_gb300 import _lib, api
+from paper_2003_06513_gb300 import workloads as WL
+
+pytestmark = pytest.mark.gpu
+
+PP_ERR_SCRATCH = -13
+
+
+def _call_static(lib, layer, x, b, y):
+    N, _, H, W = x.shape
+    return lib.pp_conv_static_scratch(layer._h, ctypes.c_void_p(x.data_ptr()), 0, N, H, W,
+                                      ctypes.c_void_p(b.data_ptr()), 1,
+                                      ctypes.c_void_p(y.data_ptr()), None)
+
+
+def test_static_scratch_entry_point_matches_workspace_entry_point():
+    lib = _lib.load()
+    cap = ctypes.c_size_t()
+    assert lib.pp_static_scratch_bytes(ctypes.byref(cap)) == 0 and cap.value == 32 << 20
+
+    L = WL.vgg16()[10]                                # 512 -> 512 at 14x14: split input channels
+    W, bias = WL.weights(L), WL.bias(L)
+    x_np = WL.layer_input(L, 16)
+    layer = api.pp_pack(W, None, L.keep).bind("cuda")
+    x = torch.from_numpy(x_np).cuda()
+    b = torch.from_numpy(bias).cuda()
+    need = layer.workspace_bytes(x.shape)
+    assert 0 < need <= cap.value
+    assert layer.plan(x.shape, cap.value)["splits"] > 1
+
+    ws = torch.empty(need // 4, dtype=torch.float32, device="cuda")
+    ref = layer.conv(x, b, True, workspace=ws)
+    torch.cuda.synchronize()
+
+    Wh = OPR.project(W, OP.default8(), L.keep)["W_hat"]
+    den = OC.denominator(x_np, Wh, bias, 1)
+    ref_h = ref.double().cpu().numpy()
+    for _ in range(2):                                # two calls in a row share the array
+        y = torch.full_like(ref, float("nan"))
+        assert _call_static(lib, layer, x, b, y) == 0
+        torch.cuda.synchronize()
+        err = OC.max_norm_err(y.double().cpu().numpy(), ref_h, den)
+        assert err <= 1e-4, f"static-scratch result differs from pp_conv_ws: {err:.3e}"
+
+
+def test_static_scratch_rejects_calls_beyond_its_size():
+    lib = _lib.load()
+    # a wide layer on small images: few CTAs, so the plan splits the input channels, and the
+    # partial sums of the split outgrow the 32 MiB array
+    C = 1024
+    W = np.random.default_rng(0).standard_normal((C, C, 3, 3)).astype(np.float32)
+    layer = api.pp_pack(W, None, 0.25).bind("cuda")
+    shape = None
+    for n in (16, 32, 64, 96, 128):
+        if layer.workspace_bytes((n, C, 7, 7)) > 32 << 20:
+            shape = (n, C, 7, 7)
+            break
+    assert shape is not None, "no call shape needs more scratch than the static array"
+    x = torch.zeros(shape, device="cuda")
+    y = torch.zeros(shape, device="cuda")
+    b = torch.zeros(C, device="cuda")
+    assert _call_static(lib, layer, x, b, y) == PP_ERR_SCRATCH
+    assert b"static scratch" in lib.pp_status_string(PP_ERR_SCRATCH)
