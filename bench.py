@@ -44,6 +44,9 @@ def parse():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0, help="oracle sample budget")
+    ap.add_argument("--profile-layer", type=int, default=None,
+                    help="run only VGG-16 layer IDX (0-based) --steps times at --batch (for ncu)")
+    ap.add_argument("--batch", type=int, default=BATCH, help="batch of --profile-layer")
     return ap.parse_args()
 
 
@@ -230,17 +233,21 @@ def hbm_peak():
 
 
 def traffic_record():
-    """Per-launch DRAM bytes of pconv_main from the committed ncu summary, or None when the
-    kernel source changed since the counters were taken."""
-    path = os.path.join(ROOT, "profiles", "pconv_main_vgg16_traffic.json")
+    """Per-launch DRAM bytes of pconv_tm on this workload from the committed ncu summary, or
+    None when the kernel source changed since the counters were taken."""
+    path = os.path.join(ROOT, "profiles", "pconv_tm_vgg16_b32_traffic.txt")
     src = os.path.join(ROOT, "paper_2003_06513_gb300", "csrc", "conv.cu")
     try:
+        rec = {}
         with open(path) as f:
-            rec = json.load(f)
+            for line in f:
+                if ":" in line and not line.startswith("#"):
+                    k, v = line.split(":", 1)
+                    rec[k.strip()] = v.strip()
         with open(src, "rb") as f:
             sha = hashlib.sha256(f.read()).hexdigest()
         if rec.get("conv_cu_sha256") == sha:
-            return rec
+            return {"dram_bytes_per_launch": float(rec["dram_bytes_per_launch"])}
     except Exception:
         pass
     return None
@@ -398,8 +405,36 @@ def our_arm(args, rank, world, local_rank):
         dist.destroy_process_group()
 
 
+def profile_layer(args):
+    """One VGG-16 layer alone at a chosen batch, for profiler captures on small cases."""
+    import torch
+    from paper_2003_06513_gb300 import api
+    from paper_2003_06513_gb300 import workloads as WL
+    L = WL.vgg16()[args.profile_layer]
+    lay = api.pp_pack(WL.weights(L), None, L.keep).bind("cuda")
+    x = torch.from_numpy(WL.layer_input(L, args.batch)).cuda()
+    b = torch.from_numpy(WL.bias(L)).cuda()
+    ws_n = lay.workspace_bytes(x.shape)
+    ws = torch.empty(max(ws_n // 4, 1), device="cuda") if ws_n else None
+    y = lay.conv(x, b, True, workspace=ws)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        lay.conv(x, b, True, y, workspace=ws)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / max(args.steps, 1)
+    flops = 8.0 * lay.beta * args.batch * L.ho * L.wo
+    print(json.dumps({"layer": L.name, "batch": args.batch, "ms": ms, "useful_tflops": flops / ms / 1e9,
+                      "plan": lay.plan(x.shape, ws_n)}))
+
+
 def main():
     args = parse()
+    if args.profile_layer is not None:
+        profile_layer(args)
+        return
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
