@@ -68,7 +68,9 @@ typedef enum { PP_F32 = 0, PP_F16 = 1 } pp_dtype;
  *   DENSE  f32[Cout][Cin_g][9] projected weights with zeros in place
  *   IMAGE  the device image: PERM | DESC | KOFS | VALS, each starting at a multiple of 256 B.
  * Filter slot order (filter kernel reorder, §3.4): filters sorted by kept count descending, then
- * by their pattern-index sequence over ci (pruned = 15) ascending, then by original index. */
+ * by their pattern-index sequence over ci (pruned = 15) ascending, then by original index; the
+ * j-th filter of that order takes slot r = j / G of group g = j % G (g = G-1 - j % G when r is
+ * odd), so every group holds a similar number of kept kernels. */
 typedef enum {
     PP_SEC_HEADER = 0, PP_SEC_PID = 1, PP_SEC_PERM = 2, PP_SEC_DESC = 3,
     PP_SEC_KOFS = 4, PP_SEC_VALS = 5, PP_SEC_DENSE = 6, PP_SEC_IMAGE = 7

@@ -10,9 +10,10 @@ so that the two can be compared bit for bit.
 Specification (F = 8 filters per group, G = ceil(Cout / F), K = Cin_g kernels per filter):
 
 * filter order: filters sorted by (kept-kernel count descending, pattern-id sequence over ci
-  ascending with a pruned kernel counted as 15, original index ascending); slot j of the sorted
-  order holds filter perm[j]; group g owns slots 8g .. 8g+7; missing slots are padding
-  (perm = 0xFFFFFFFF);
+  ascending with a pruned kernel counted as 15, original index ascending); the j-th filter of
+  that order goes to group g = j mod G in round r = j div G (g = G-1 - (j mod G) when r is odd:
+  snake order, so every group gets a similar number of kept kernels) and slot r, i.e.
+  perm[8g + r]; group g owns perm[8g .. 8g+7]; missing slots are padding (perm = 0xFFFFFFFF);
 * header  u32[16]: magic 'PPK1' (0x314B5050), version 1, Cout, Cin_g, groups, stride,
   n_patterns, beta, F, G, the masks two per word (low half first) in 4 words, 0, 0;
 * pid     i8 [Cout][Cin_g]: pattern index, -1 = pruned, original filter order;
@@ -64,7 +65,10 @@ def build(W: np.ndarray, pid: np.ndarray, masks: Sequence[int], groups: int, str
     G = (cout + F - 1) // F
     order = filter_order(pid)
     perm = np.full(G * F, PAD, dtype=np.uint32)
-    perm[:cout] = order
+    for j, co in enumerate(order):
+        r, pos = divmod(j, G)
+        g = pos if r % 2 == 0 else G - 1 - pos
+        perm[g * F + r] = co
 
     desc = np.zeros(G * cin_g, dtype=np.uint64)
     kofs = np.zeros(G * cin_g + 1, dtype=np.uint32)
@@ -76,10 +80,9 @@ def build(W: np.ndarray, pid: np.ndarray, masks: Sequence[int], groups: int, str
             word = 0
             c = 0
             for f in range(F):
-                j = g * F + f
-                if j >= cout:
+                if perm[g * F + f] == PAD:
                     continue
-                co = order[j]
+                co = int(perm[g * F + f])
                 p = int(pid[co, ci])
                 if p < 0:
                     continue

@@ -94,7 +94,7 @@ constexpr uint32_t kTmemCols = 512;                // 16 warps x 8 slots x 16 ac
 // Device status word: a wait that ran out of time records its code here and the kernel returns
 // early instead of hanging (read back by pp_device_status).
 __device__ unsigned int g_pp_status;
-enum : unsigned { kStatusFullTimeout = 1u, kStatusDrainTimeout = 4u };
+enum : unsigned { kStatusFullTimeout = 1u, kStatusEmptyTimeout = 2u, kStatusDrainTimeout = 4u };
 
 struct TmParams {
     const void* x;
@@ -149,6 +149,13 @@ __device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity, unsigned*
         }
     }
 }
+__device__ __forceinline__ void mbar_arrive(uint32_t a) {
+    asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(a) : "memory");
+}
+// mbar_wait by a whole warp with one outcome for all its lanes
+__device__ __forceinline__ bool mbar_wait_warp(uint32_t a, uint32_t parity, unsigned* status, unsigned code) {
+    return __all_sync(0xffffffffu, mbar_wait(a, parity, status, code));
+}
 __device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map, int x, int y, int c, int n,
                                             uint32_t mbar) {
     asm volatile(
@@ -175,79 +182,84 @@ __device__ __forceinline__ void tmem_zero16(uint32_t ta) {
 }
 
 // Fallback input staging when no TMA descriptor applies (row pitch not a multiple of 16 bytes,
-// or fp16 input widened to fp32 on the way): copy the in-image part of the tile; everything else
-// in the stage keeps the zero written at kernel start.
+// or fp16 input widened to fp32 on the way): thread tid copies elements tid, tid + 512, ... of the
+// in-image part of the tile; everything else in the stage keeps the zero written at kernel start.
 template <typename TIn>
-__device__ __forceinline__ void stage_input_fallback(const TmParams& p, float* s_in, int c0, int ckv, int n0,
-                                                     int iy0, int ix0, int lane) {
+__device__ __forceinline__ void stage_input_share(const TmParams& p, float* s_in, int c0, int ckv, int n0,
+                                                  int iy0, int ix0, int tid) {
     const TIn* x = static_cast<const TIn*>(p.x);
     const int ry0 = max(0, iy0), ry1 = min(p.H, iy0 + p.IH);
     const int rx0 = max(0, ix0), rx1 = min(p.W, ix0 + p.BWb);
     const int nr = ry1 - ry0, nc = rx1 - rx0;
     if (nr <= 0 || nc <= 0) return;
-    int nimg = min(p.NB, p.N - n0);
-    const int planes = nimg * ckv;
+    const int nimg = min(p.NB, p.N - n0);
     // fp32 rows whose global start and length are even go as 8-byte pairs; the staged column of
     // image column ix is ix - ix0 with ix0 a multiple of 4, so the shared side is 8-byte aligned too
     const bool pairs = sizeof(TIn) == 4 && (p.W % 2 == 0) && (rx0 % 2 == 0) && (nc % 2 == 0);
     const int units = pairs ? nc / 2 : nc;                  // copy units per row
-    const int per_plane = nr * units;
-    const int total = planes * per_plane;
-    // unit e -> (plane, row, unit-in-row), advanced incrementally by 32 per step
-    int pl = lane / per_plane, rem = lane - pl * per_plane;
-    int r = rem / units, u = rem - r * units;
-    const int step_pl = 32 / per_plane, step_rem = 32 - step_pl * per_plane;
-    for (int e = lane; e < total; e += 32) {
-        const int img = pl / ckv, cl = pl - (pl / ckv) * ckv;
+    // element e = ((img * ckv + cl) * nr + r) * units + u as digits (img, cl, r, u); adding the
+    // thread count digit by digit needs at most one carry per digit
+    int q = tid / units;
+    int u = tid - q * units;
+    int r = q % nr;
+    q /= nr;
+    int cl = q % ckv, img = q / ckv;
+    q = kThreadsTM / units;
+    const int su = kThreadsTM - q * units, sr = q % nr;
+    q /= nr;
+    const int scl = q % ckv, simg = q / ckv;
+    const size_t HW = (size_t)p.H * p.W;
+    while (img < nimg) {
         const int iy = ry0 + r, ix = rx0 + (pairs ? 2 * u : u);
-        const TIn* src = x + (((size_t)(n0 + img) * p.C + c0 + cl) * p.H + iy) * p.W + ix;
-        float* dst = s_in + (((size_t)img * p.CK + cl) * p.IH + (iy - iy0)) * p.BWb + (ix - ix0);
+        const TIn* src = x + ((size_t)(n0 + img) * p.C + c0 + cl) * HW + (size_t)iy * p.W + ix;
+        float* dst = s_in + ((img * p.CK + cl) * p.IH + (iy - iy0)) * p.BWb + (ix - ix0);
         if constexpr (sizeof(TIn) == 4) {
             if (pairs) cp_async8(dst, src);
             else cp_async4(dst, src, true);
         } else {
             *dst = to_f32<TIn>(*src);
         }
-        pl += step_pl;
-        u += step_rem;
-        while (u >= units) {
-            u -= units;
-            if (++r == nr) {
-                r = 0;
-                ++pl;
-            }
-        }
+        u += su;
+        if (u >= units) { u -= units; ++r; }
+        r += sr;
+        if (r >= nr) { r -= nr; ++cl; }
+        cl += scl;
+        if (cl >= ckv) { cl -= ckv; ++img; }
+        img += simg;
     }
 }
 
-// Fill pipeline stage k % kStages with input channel chunk k (whole warp; non-blocking): the
-// input tile by one TMA (or the fallback copy), each group's descriptors and kept weights by
-// cp.async; the stage's full barrier completes when every byte has landed.
+// This thread's share of filling pipeline stage k % kStages with input channel chunk k
+// (non-blocking): warp 0 lane 0 issues the input tile's TMA, or every thread copies its share of
+// the tile; the warps of filter group wg copy that group's descriptors and kept weights.  The
+// stage's full barrier completes when all 512 threads have arrived and every byte has landed.
 template <typename TIn>
-__device__ __forceinline__ void produce_chunk(const TmParams& p, const CUtensorMap* tmap, unsigned char* smem,
-                                              const uint32_t* s_kb, uint32_t full0, int k, int n0, int iy0,
-                                              int ix0, int g0, int c_lo, int c_hi, int lane) {
+__device__ __forceinline__ void fill_share(const TmParams& p, const CUtensorMap* tmap, unsigned char* smem,
+                                           const uint32_t* s_kb, uint32_t full0, int k, int n0, int iy0,
+                                           int ix0, int g0, int c_lo, int c_hi, int warp, int lane) {
     const int s = k % kStages;
     const int nkb = p.n_chunks + 1;
     unsigned char* st = smem + p.stage_off + (size_t)s * p.stage_bytes;
     const uint32_t fb = full0 + 8 * s;
     const int c0 = c_lo + k * p.CK, ckv = min(p.CK, c_hi - c0);
-    if (lane == 0) {
+    if (warp == 0 && lane == 0) {
         mbar_arrive_expect_tx(fb, p.use_tma ? p.tma_bytes : 0u);
-        if (p.use_tma) tma_load_4d(smem_u32(st), tmap, ix0, iy0, c0, n0, fb);
+        if (p.use_tma) {
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            tma_load_4d(smem_u32(st), tmap, ix0, iy0, c0, n0, fb);
+        }
     }
-    if (!p.use_tma) stage_input_fallback<TIn>(p, reinterpret_cast<float*>(st), c0, ckv, n0, iy0, ix0, lane);
-    uint64_t* sd = reinterpret_cast<uint64_t*>(st + p.desc_off);
-    for (int i = lane; i < p.WG * ckv; i += 32) {
-        const int wg = i / ckv, cl = i - wg * ckv, g = g0 + wg;
-        if (g < p.G) cp_async8(sd + wg * p.CK + cl, p.desc + (size_t)g * p.C + c0 + cl);
-    }
-    float4* sv = reinterpret_cast<float4*>(st + p.vals_off);
-    for (int wg = 0; wg < p.WG; ++wg) {
+    if (!p.use_tma) stage_input_share<TIn>(p, reinterpret_cast<float*>(st), c0, ckv, n0, iy0, ix0, warp * 32 + lane);
+    const int wg = warp / p.WS, ws = warp - wg * p.WS, g = g0 + wg;
+    if (g < p.G) {
+        uint64_t* sd = reinterpret_cast<uint64_t*>(st + p.desc_off) + wg * p.CK;
+        for (int cl = ws * 32 + lane; cl < ckv; cl += p.WS * 32)
+            cp_async8(sd + cl, p.desc + (size_t)g * p.C + c0 + cl);
+        float4* sv = reinterpret_cast<float4*>(st + p.vals_off) + wg * p.maxk;
         const uint32_t beg = s_kb[wg * nkb + k], end = s_kb[wg * nkb + k + 1];
-        for (uint32_t i = beg + lane; i < end; i += 32) cp_async16(sv + wg * p.maxk + (i - beg), p.vals + i);
+        for (uint32_t i = beg + ws * 32 + lane; i < end; i += p.WS * 32) cp_async16(sv + (i - beg), p.vals + i);
     }
-    __threadfence_block();
+    __threadfence_block();   // orders the fp16 path's plain shared stores before the arrival
     cp_async_arrive(fb);
 }
 
@@ -257,12 +269,13 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     constexpr int RY = 4, RX = 4;
     extern __shared__ __align__(128) unsigned char smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    uint64_t* bar = reinterpret_cast<uint64_t*>(smem);                    // full[kStages]
-    uint32_t* s_cnt = reinterpret_cast<uint32_t*>(smem + 8 * kStages);    // releases per stage
-    uint32_t* s_tmem = s_cnt + kStages;                                   // tensor-memory base
-    uint32_t* s_issued = s_tmem + 1;                                      // chunks issued
+    // header: full[kStages] (stage filled), empty[kStages] (stage read by all 16 warps), the
+    // tensor-memory base and the number of chunks whose fill warp 0 has issued
+    uint64_t* bar = reinterpret_cast<uint64_t*>(smem);
+    uint32_t* s_tmem = reinterpret_cast<uint32_t*>(smem + 16 * kStages);
+    uint32_t* s_issued = s_tmem + 1;
     uint32_t* s_kb = reinterpret_cast<uint32_t*>(smem + p.kb_off);
-    const uint32_t full0 = smem_u32(bar);
+    const uint32_t full0 = smem_u32(bar), empty0 = full0 + 8 * kStages;
 
     // CTA -> (spatial tile, filter chunk); the filter chunk varies fastest so CTAs that share an
     // input tile run together and hit it in L2
@@ -295,8 +308,8 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     if (warp == 0) {
         if (lane == 0) {
             for (int s = 0; s < kStages; ++s) {
-                mbar_init(full0 + 8 * s, 33);   // lane 0's expect-tx arrival + 32 cp.async arrivals
-                s_cnt[s] = 0;
+                mbar_init(full0 + 8 * s, kThreadsTM + 1);   // 512 cp.async arrivals + the expect-tx one
+                mbar_init(empty0 + 8 * s, kCompute);        // one arrival per warp
             }
             *s_issued = 0;
         }
@@ -309,11 +322,11 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tbase = *s_tmem;
 
-    if (warp == 0) {   // prologue: fill every stage
+    {   // prologue: every thread's share of the first kStages chunks
         const int first = min(kStages, nck);
         for (int k = 0; k < first; ++k)
-            produce_chunk<TIn>(p, &tmap, smem, s_kb, full0, k, n0, iy0, ix0, g0, c_lo, c_hi, lane);
-        if (lane == 0) *s_issued = first;
+            fill_share<TIn>(p, &tmap, smem, s_kb, full0, k, n0, iy0, ix0, g0, c_lo, c_hi, warp, lane);
+        if (threadIdx.x == 0) *s_issued = first;
     }
 
     const int wg = warp / p.WS, ws = warp - (warp / p.WS) * p.WS;
@@ -334,7 +347,7 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
 
     for (int k = 0; k < nck; ++k) {
         const int s = k % kStages;
-        if (!mbar_wait(full0 + 8 * s, (k / kStages) & 1, p.status, kStatusFullTimeout)) break;
+        if (!mbar_wait_warp(full0 + 8 * s, (k / kStages) & 1, p.status, kStatusFullTimeout)) break;
         if (g < p.G) {
             const unsigned char* st = smem + p.stage_off + (size_t)s * p.stage_bytes;
             const uint32_t win_addr = smem_u32(reinterpret_cast<const float*>(st) + in_off);
@@ -347,21 +360,16 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
                 PP_STAGE_KERNELS_S2(ckv, desc_addr, vals_addr, win_addr, 4 * p.BWb, 4 * plane, tw);
             }
         }
-        // release the stage; the last warp to release it refills it with chunk k + kStages
+        // release the stage, then take this warp's share of filling chunk k + kStages - 1 into the
+        // stage chunk k - 1 used, once all 16 warps have released that one
         __syncwarp();
-        uint32_t old = 0;
-        if (lane == 0) {
-            __threadfence_block();
-            old = atomicAdd(&s_cnt[s], 1u);
-        }
-        old = __shfl_sync(0xffffffffu, old, 0);
-        if (old == kCompute - 1) {
-            if (lane == 0) s_cnt[s] = 0;
-            if (k + kStages < nck) {
-                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                produce_chunk<TIn>(p, &tmap, smem, s_kb, full0, k + kStages, n0, iy0, ix0, g0, c_lo, c_hi, lane);
-                if (lane == 0) atomicMax(s_issued, (uint32_t)(k + kStages + 1));
-            }
+        if (lane == 0) mbar_arrive(empty0 + 8 * s);
+        const int j = k + kStages - 1;
+        if (k >= 1 && j < nck) {
+            if (!mbar_wait_warp(empty0 + 8 * (j % kStages), ((k - 1) / kStages) & 1, p.status, kStatusEmptyTimeout))
+                break;
+            fill_share<TIn>(p, &tmap, smem, s_kb, full0, j, n0, iy0, ix0, g0, c_lo, c_hi, warp, lane);
+            if (threadIdx.x == 0) *s_issued = j + 1;
         }
     }
 
@@ -429,10 +437,11 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
             }
         }
     }
+    asm volatile("cp.async.wait_all;" ::: "memory");   // this thread's copies (only after a timeout)
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
     if (warp == 0) {
-        // no copy of this CTA may still be in flight when it exits (only possible after a timeout)
+        // no tensor copy of this CTA may still be in flight when it exits (only after a timeout)
         if (lane == 0) {
             const int issued = (int)*s_issued;
             for (int k = max(0, issued - kStages); k < issued; ++k)
@@ -521,16 +530,18 @@ __global__ void pconv_generic(const T* __restrict__ x, T* __restrict__ y, const 
                               const uint32_t* perm, const uint64_t* desc, const uint32_t* kofs,
                               const float4* vals, TapTable taps, int N, int C, int cin_g, int dw, int H,
                               int W, int Cout, int Ho, int Wo, int S, int relu) {
-    const long long total = (long long)N * Cout * Ho * Wo;
+    const int nslot = (Cout + kF - 1) / kF * kF;   // padding slots may sit anywhere in a group
+    const long long total = (long long)N * nslot * Ho * Wo;
     for (long long o = blockIdx.x * (long long)blockDim.x + threadIdx.x; o < total;
          o += (long long)gridDim.x * blockDim.x) {
         const int ox = (int)(o % Wo);
         long long r = o / Wo;
         const int oy = (int)(r % Ho);
         r /= Ho;
-        const int slot = (int)(r % Cout);
-        const int n = (int)(r / Cout);
+        const int slot = (int)(r % nslot);
+        const int n = (int)(r / nslot);
         const uint32_t co = perm[slot];
+        if (co == kPadSlot) continue;
         const int g = slot / kF, f = slot % kF;
         float a = 0.0f;
         for (int ci = 0; ci < cin_g; ++ci) {

@@ -6,8 +6,9 @@
 //  * connectivity pruning (§4.4, C'_n: at most beta nonzero kernels): the beta kernels with the
 //    largest retained energy survive, ties to the lower flat index;
 //  * filter kernel reorder and compressed weight storage (§3.4): filters sorted by
-//    (kept count desc, pattern sequence asc, index asc), cut into groups of 8; per (group, ci) a
-//    64-bit descriptor of (slot, pattern) codes; 4 fp32 values per kept kernel.
+//    (kept count desc, pattern sequence asc, index asc) and dealt to groups of 8 in snake order
+//    (balanced kept counts per group); per (group, ci) a 64-bit descriptor of (slot, pattern)
+//    codes; 4 fp32 values per kept kernel.
 //
 // Built with -ffp-contract=off: every float64 operation below rounds on its own.
 #include <algorithm>
@@ -98,10 +99,17 @@ int build(pp_layer* L, const float* W, double keep) {
         return a < b;
     });
 
+    // deal the sorted filters over the G groups in snake order (round r fills slot r of every
+    // group, alternating direction), so that every group gets a similar number of kept kernels:
+    // one warp processes one group, and the warps of a CTA then finish their channels together
     const int G = (cout + kF - 1) / kF;
     L->G = G;
     L->perm.assign((size_t)G * kF, kPadSlot);
-    for (int j = 0; j < cout; ++j) L->perm[j] = (uint32_t)fo[j];
+    for (int j = 0; j < cout; ++j) {
+        const int round = j / G, pos = j % G;
+        const int g = (round % 2 == 0) ? pos : G - 1 - pos;
+        L->perm[(size_t)g * kF + round] = (uint32_t)fo[j];
+    }
 
     // 4. compressed weight storage
     L->desc.assign((size_t)G * cin_g, 0);
@@ -115,9 +123,9 @@ int build(pp_layer* L, const float* W, double keep) {
             uint64_t word = 0;
             unsigned c = 0;
             for (int f = 0; f < kF; ++f) {
-                const int j = g * kF + f;
-                if (j >= cout) continue;
-                const int co = fo[j];
+                const uint32_t co_u = L->perm[(size_t)g * kF + f];
+                if (co_u == kPadSlot) continue;
+                const int co = (int)co_u;
                 const int p = L->pid[(size_t)co * cin_g + ci];
                 if (p < 0) continue;
                 word |= (uint64_t)((unsigned)(f << 3) | (unsigned)p) << (4 + 6 * c);

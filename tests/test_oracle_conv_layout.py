@@ -160,10 +160,16 @@ def test_layout_decodes_to_projection(cout, cin, keep, dw):
     # structure of the sections
     G = (cout + 7) // 8
     perm = s["perm"]
-    assert sorted(perm[:cout].tolist()) == list(range(cout))
-    assert (perm[cout:] == L.PAD).all()
-    counts = [int(np.count_nonzero(r["pid"][co] >= 0)) for co in perm[:cout]]
-    assert counts == sorted(counts, reverse=True)          # filter kernel reorder by length
+    real = perm[perm != L.PAD]
+    assert sorted(real.tolist()) == list(range(cout)) and perm.size == 8 * G
+    # filter kernel reorder: filters in kept-count order, dealt to groups in snake order, so
+    # group totals differ by at most the largest single filter's count
+    count = np.count_nonzero(r["pid"] >= 0, axis=1)
+    order = L.filter_order(r["pid"])
+    assert [count[c] for c in order] == sorted(count, reverse=True)
+    totals = [sum(int(count[c]) for c in perm[8 * g:8 * g + 8] if c != L.PAD) for g in range(G)]
+    if cout % G == 0 or cout < G:
+        assert max(totals) - min(totals) <= int(count.max())
     assert (np.diff(s["kofs"].astype(np.int64)) >= 0).all() and s["kofs"][-1] == r["beta"]
     assert s["vals"].shape == (r["beta"], 4)
     assert s["image"].size % 256 == 0
