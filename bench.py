@@ -47,12 +47,21 @@ def parse():
     ap.add_argument("--profile-layer", type=int, default=None,
                     help="run only VGG-16 layer IDX (0-based) --steps times at --batch (for ncu)")
     ap.add_argument("--batch", type=int, default=BATCH, help="batch of --profile-layer")
+    ap.add_argument("--workload", choices=["vgg16", "single", "resnet50", "mobilenet"], default="vgg16",
+                    help="vgg16: the headline step; the others time each layer of that config alone "
+                         "and report it against its roofline")
+    ap.add_argument("--sweep", action="store_true", help="single-layer roofline sweep (288 points)")
+    ap.add_argument("--sweep-out", default=None, help="also write the sweep as a markdown table here")
+    ap.add_argument("--no-dense-context", action="store_true", help="skip the cuDNN dense context")
     return ap.parse_args()
 
 
-def conv_cost(beta, cin, cout, h, w, ho, wo, n, G, es=4):
+def conv_cost(beta, cin, cout, h, w, ho, wo, n, G, es=4, cin_g=None):
+    """Useful FLOP (8 per kept kernel per output pixel) and algorithmic bytes (input and output
+    activations once, the packed weight image once, the bias) of one pattern-sparse conv."""
+    cin_g = cin if cin_g is None else cin_g
     flops = 8.0 * beta * n * ho * wo
-    image = 4 * G * 8 + 8 * G * cin + 4 * (G * cin + 1) + 16 * beta
+    image = 4 * G * 8 + 8 * G * cin_g + 4 * (G * cin_g + 1) + 16 * beta
     bytes_ = es * (n * cin * h * w + n * cout * ho * wo) + image + 4 * cout
     return flops, float(bytes_)
 
@@ -286,9 +295,9 @@ def our_arm(args, rank, world, local_rank):
     bufA = torch.empty(big, dtype=torch.float32, device=dev)
     bufB = torch.empty(big, dtype=torch.float32, device=dev)
     out_final = torch.empty((BATCH, 512, 7, 7), dtype=torch.float32, device=dev)
-    stream = torch.cuda.current_stream(dev)
 
     def step(x, ev=None):
+        stream = torch.cuda.current_stream(dev)    # the capture stream while a graph records
         cur = x
         bufs = (bufA, bufB)
         j = 0
@@ -326,6 +335,7 @@ def our_arm(args, rank, world, local_rank):
     evs = [[[torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)]
             for _ in layers] for _ in range(K)]
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    stream = torch.cuda.current_stream(dev)
     with ClockSampler(dev.index) as clk:
         barrier()
         t0.record(stream)
@@ -335,6 +345,25 @@ def our_arm(args, rank, world, local_rank):
         barrier()
     elapsed_ms = t0.elapsed_time(t1)
     conv_ms = [[evs[k][i][0].elapsed_time(evs[k][i][1]) for i in range(len(layers))] for k in range(K)]
+
+    # the same step captured once in a CUDA graph and replayed (no per-launch host work)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        step(x0)
+    for _ in range(3):
+        graph.replay()
+    barrier()
+    g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    g0.record(stream)
+    for _ in range(K):
+        graph.replay()
+    g1.record(stream)
+    barrier()
+    graph_ms = g0.elapsed_time(g1) / K
+
+    dense = None
+    if not args.no_dense_context:
+        dense = dense_context(packed, biases, layers, x0, K, barrier)
 
     # e2e: input from pinned host memory and the final feature map back, inside the timed region
     host_in = torch.from_numpy(WL.vgg16_image(BATCH)).pin_memory()
@@ -354,10 +383,10 @@ def our_arm(args, rank, world, local_rank):
     barrier()
     e2e_ms = e0.elapsed_time(e1) / Ke
 
-    t = torch.tensor([elapsed_ms, e2e_ms], device=dev, dtype=torch.float64)
+    t = torch.tensor([elapsed_ms, e2e_ms, graph_ms], device=dev, dtype=torch.float64)
     if dist is not None:
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    elapsed_ms, e2e_ms = float(t[0]), float(t[1])
+    elapsed_ms, e2e_ms, graph_ms = float(t[0]), float(t[1]), float(t[2])
 
     if rank == 0:
         props = torch.cuda.get_device_properties(dev)
@@ -370,7 +399,8 @@ def our_arm(args, rank, world, local_rank):
         tot_conv_ms = sum(statistics.mean(conv_ms[k][i] for k in range(K)) for i in range(len(layers)))
         achieved = sum(flops) / (tot_conv_ms * 1e-3)
         roof_ms = sum(max(f / peak, b / hbm) for f, b in zip(flops, bytes_)) * 1e3
-        ms_step = elapsed_ms / K
+        eager_ms = elapsed_ms / K
+        ms_step = min(eager_ms, graph_ms)      # the faster of stream launches and graph replay
         img_s = world * BATCH / (ms_step * 1e-3)
         trec = traffic_record()
         line = {
@@ -388,6 +418,8 @@ def our_arm(args, rank, world, local_rank):
                          "traffic": (trec or {}).get("dram_bytes_per_launch"),
                          "algorithmic_bytes_per_launch": sum(bytes_) / len(bytes_),
                          "hbm_peak_gbs": hbm / 1e9, "hbm_peak_kind": hbm_kind},
+            "timing": {"eager_ms_per_step": eager_ms, "graph_ms_per_step": graph_ms,
+                       "value_from": "graph" if graph_ms <= eager_ms else "eager"},
             "per_layer_ms": [round(v, 4) for v in per_layer_ms],
             "e2e": {"value": world * BATCH / (e2e_ms * 1e-3), "unit": "img/s",
                     "h2d_bytes_per_step": int(host_in.numel() * 4),
@@ -395,6 +427,11 @@ def our_arm(args, rank, world, local_rank):
             "gpu_launches": K * launches_per_step,
             "clocks": clocks,
         }
+        if dense is not None:
+            line["cudnn_dense_context"] = {"value": world * BATCH / (dense * 1e-3), "unit": "img/s",
+                                           "ms_per_step": dense,
+                                           "what": "torch conv2d (cuDNN) on the zero-filled projected "
+                                                   "weights + bias + ReLU, max_pool2d; fp32, TF32 off"}
         if world == 1 and not args.no_cpu_baseline:
             n, dt, thr = oracle_forward_images(args.cpu_seconds, max_images=BATCH)
             line["cpu_baseline"] = {"value": n / dt, "unit": "img/s", "cores": thr, "kind": "oracle",
@@ -403,6 +440,157 @@ def our_arm(args, rank, world, local_rank):
     if dist is not None:
         dist.barrier()
         dist.destroy_process_group()
+
+
+def dense_context(packed, biases, layers, x0, K, barrier):
+    """ms per step of the same network as dense fp32 convolutions (cuDNN) on the zero-filled
+    projected weights: the dense work the pattern-sparse path avoids, for context."""
+    import torch
+    import torch.nn.functional as F
+    torch.backends.cudnn.allow_tf32 = False
+    torch.backends.cuda.matmul.allow_tf32 = False
+    torch.backends.cudnn.benchmark = True
+    dev = x0.device
+    dense = [torch.from_numpy(lay.export("dense").reshape(L.cout, L.cin_g, 3, 3)).to(dev)
+             for lay, L in zip(packed, layers)]
+
+    def dstep(x):
+        for L, Wd, b in zip(layers, dense, biases):
+            x = F.relu(F.conv2d(x, Wd, b, stride=L.stride, padding=1))
+            if L.pool_after:
+                x = F.max_pool2d(x, 2)
+        return x
+
+    with torch.no_grad():
+        for _ in range(3):
+            dstep(x0)
+        barrier()
+        st = torch.cuda.current_stream(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        Kd = max(3, min(K, 20))
+        e0.record(st)
+        for _ in range(Kd):
+            dstep(x0)
+        e1.record(st)
+        barrier()
+    return e0.elapsed_time(e1) / Kd
+
+
+def _peaks(dev):
+    import torch
+    props = torch.cuda.get_device_properties(dev)
+    peak, mhz = fp32_peak(props, {})
+    hbm, kind = hbm_peak()
+    return peak, hbm, kind, f"{props.multi_processor_count} SMs x 128 FP32 lanes x 2 x {mhz:.0f} MHz"
+
+
+def _time_layer(lay, x, b, relu, ws, K):
+    """Median ms of K launches of one layer (CUDA events on the current stream, after 3 warm-ups)."""
+    import torch
+    y = lay.conv(x, b, relu, workspace=ws)
+    for _ in range(2):
+        lay.conv(x, b, relu, y, workspace=ws)
+    torch.cuda.synchronize()
+    st = torch.cuda.current_stream()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    for e0, e1 in evs:
+        e0.record(st)
+        lay.conv(x, b, relu, y, workspace=ws)
+        e1.record(st)
+    torch.cuda.synchronize()
+    return statistics.median(e0.elapsed_time(e1) for e0, e1 in evs)
+
+
+def layer_suite(args):
+    """Every layer of one config timed alone (inputs resident, larger than L2 where the config is)
+    and set against its own roofline min(FP32 peak, AI x HBM bandwidth)."""
+    import numpy as np
+    import torch
+    from paper_2003_06513_gb300 import api
+    from paper_2003_06513_gb300 import workloads as WL
+    which = args.workload
+    if which == "single":
+        layers, batch, dt = [WL.single_layer()], 1, "f32"
+    elif which == "resnet50":
+        layers, batch, dt = WL.resnet50_3x3(), 64, "f32"
+    else:
+        layers, batch, dt = WL.mobilenet_v2_dw(), 128, "f16"
+    tdt, ndt, es = (torch.float16, np.float16, 2) if dt == "f16" else (torch.float32, np.float32, 4)
+    peak, hbm, hbm_kind, basis = _peaks(0)
+    K = max(args.steps, 5)
+    rows, tot_ms, tot_roof, tot_flops = [], 0.0, 0.0, 0.0
+    with ClockSampler(0) as clk:
+        for L in layers:
+            lay = api.pp_pack(WL.weights(L), None, L.keep, groups=L.cout if L.depthwise else 1,
+                              stride=L.stride).bind("cuda")
+            x = torch.from_numpy(WL.layer_input(L, batch, dtype=ndt)).cuda()
+            b = torch.from_numpy(WL.bias(L)).cuda()
+            nb = lay.workspace_bytes(x.shape)
+            ws = torch.empty(max(nb // 4, 1), device="cuda") if nb else None
+            ms = _time_layer(lay, x, b, True, ws, K)
+            G = (L.cout + 7) // 8
+            fl, by = conv_cost(lay.beta, L.cin, L.cout, L.h, L.w, L.ho, L.wo, batch, G, es, L.cin_g)
+            roof = max(fl / peak, by / hbm) * 1e3
+            rows.append({"layer": L.name, "shape": [batch, L.cin, L.h, L.w, L.cout, L.stride], "ms": round(ms, 5),
+                         "useful_tflops": fl / ms / 1e9, "gbs": by / ms / 1e6,
+                         "bound": "alu" if fl / peak >= by / hbm else "hbm", "roofline_frac": roof / ms,
+                         "plan_path": lay.plan(x.shape, nb)["path"]})
+            tot_ms += ms
+            tot_roof += roof
+            tot_flops += fl
+            del x, ws
+    line = {"metric": METRIC, "workload": which, "value": tot_flops / (tot_ms * 1e-3) / 1e9, "unit": "GFLOP/s",
+            "higher_is_better": True, "n_gpus": 1, "steps": K, "dtype": dt, "batch": batch,
+            "data": "synthetic (seeded He-normal weights, N(0,1) or post-ReLU inputs)",
+            "sum_layer_ms": tot_ms,
+            "roofline": {"frac": tot_roof / tot_ms, "fp32_peak_tflops": peak / 1e12, "peak_basis": basis,
+                         "hbm_gbs": hbm / 1e9, "hbm_kind": hbm_kind,
+                         "note": "time-weighted: sum of per-layer roofline times / sum of measured times"},
+            "per_layer": rows, "clocks": clk.summary()}
+    print(json.dumps(line), flush=True)
+
+
+def sweep_run(args):
+    """Single-layer sweep: useful GFLOP/s against arithmetic intensity for every point."""
+    import torch
+    from paper_2003_06513_gb300 import api
+    from paper_2003_06513_gb300 import workloads as WL
+    peak, hbm, hbm_kind, basis = _peaks(0)
+    K = max(3, min(args.steps, 10))
+    out = []
+    with ClockSampler(0) as clk:
+        for L, n, dt in WL.sweep():
+            tdt, es = (torch.float16, 2) if dt == "f16" else (torch.float32, 4)
+            lay = api.pp_pack(WL.weights(L), None, L.keep).bind("cuda")
+            g = torch.Generator(device="cuda")
+            g.manual_seed(L.x_seed)
+            x = torch.randn((n, L.cin, L.h, L.w), generator=g, device="cuda").to(tdt)
+            b = torch.from_numpy(WL.bias(L)).cuda()
+            nb = lay.workspace_bytes(x.shape)
+            ws = torch.empty(max(nb // 4, 1), device="cuda") if nb else None
+            ms = _time_layer(lay, x, b, True, ws, K)
+            fl, by = conv_cost(lay.beta, L.cin, L.cout, L.h, L.w, L.ho, L.wo, n, (L.cout + 7) // 8, es)
+            roof = max(fl / peak, by / hbm) * 1e3
+            rec = {"c": L.cin, "hw": L.h, "n": n, "keep": L.keep, "io": dt, "ms": ms, "ai": fl / by,
+                   "useful_gflops": fl / ms / 1e6, "bound": "alu" if fl / peak >= by / hbm else "hbm",
+                   "roofline_frac": roof / ms}
+            out.append(rec)
+            print(json.dumps(rec), flush=True)
+            del x, ws
+    clocks = clk.summary()
+    if args.sweep_out:
+        with open(args.sweep_out, "w") as f:
+            f.write("# Single-layer roofline sweep: pattern-sparse 3x3 conv, stride 1, 8 patterns\n\n")
+            f.write("Command: `python bench.py --sweep --steps %d --sweep-out %s`\n\n" % (args.steps, args.sweep_out))
+            f.write(f"Peaks: FP32 {peak / 1e12:.1f} TFLOP/s ({basis}); HBM {hbm / 1e9:.0f} GB/s ({hbm_kind}). "
+                    f"Clocks: {json.dumps(clocks)}\n\n")
+            f.write("Inputs N(0,1) generated on the device from the point's seed; weights seeded He-normal. "
+                    "ms = median of %d launches. AI = useful FLOP / algorithmic bytes.\n\n" % K)
+            f.write("| C | HxW | N | keep | io | ms | AI (FLOP/B) | useful GFLOP/s | bound | roofline frac |\n")
+            f.write("|---:|---:|---:|---:|:--|---:|---:|---:|:--|---:|\n")
+            for r in out:
+                f.write(f"| {r['c']} | {r['hw']} | {r['n']} | {r['keep']} | {r['io']} | {r['ms']:.4f} | "
+                        f"{r['ai']:.1f} | {r['useful_gflops']:.0f} | {r['bound']} | {r['roofline_frac']:.3f} |\n")
 
 
 def profile_layer(args):
@@ -434,6 +622,12 @@ def main():
     args = parse()
     if args.profile_layer is not None:
         profile_layer(args)
+        return
+    if args.sweep:
+        sweep_run(args)
+        return
+    if args.workload != "vgg16" and args.impl == "ours":
+        layer_suite(args)
         return
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))

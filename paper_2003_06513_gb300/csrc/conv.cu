@@ -775,6 +775,24 @@ __global__ void splitk_reduce(const float* __restrict__ ws, T* __restrict__ y, c
     }
 }
 
+// Raise the kernel's dynamic shared-memory limit to the device's opt-in maximum once per device
+// (a launch needs at most that), so that later calls, including ones under stream capture, make
+// no attribute call.
+template <int S, typename T>
+bool allow_max_smem(size_t need) {
+    static std::atomic<int> done[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+    if (done[dev].load(std::memory_order_acquire)) return true;
+    int optin = 0;
+    if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess) return false;
+    if ((size_t)optin < need) return false;
+    if (cudaFuncSetAttribute(pconv_tm<S, T>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin) != cudaSuccess)
+        return false;
+    done[dev].store(1, std::memory_order_release);
+    return true;
+}
+
 template <int S, typename T>
 int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int relu, int N, int H, int W, int Ho,
               int Wo, void* ws, size_t ws_bytes, cudaStream_t st) {
@@ -845,8 +863,7 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
         p.tma_bytes = (unsigned)((size_t)p.BWb * p.IH * p.CK * p.NB * 4);
     }
     auto kern = pconv_tm<S, T>;
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem) != cudaSuccess)
-        return PP_ERR_CUDA;
+    if (!allow_max_smem<S, T>(pl.smem)) return PP_ERR_CUDA;
     const long long ctas = pl.ctas * pl.KS;
     if (ctas > INT_MAX) return PP_ERR_SHAPE;
     kern<<<(unsigned)ctas, kThreadsTM, pl.smem, st>>>(p, tmap);
