@@ -36,22 +36,6 @@ using namespace patconv;
 
 namespace {
 
-// ------------------------------------------------------------------------------ constants
-
-// k-th tap (ascending raster order) of pattern p of the compiled library (kDefaultMasks).
-__host__ __device__ constexpr int ktap(int p, int k) {
-    const unsigned m = p == 0 ? 0x0B8u : p == 1 ? 0x0B2u : p == 2 ? 0x09Au : p == 3 ? 0x03Au
-                     : p == 4 ? 0x017u : p == 5 ? 0x059u : p == 6 ? 0x134u : 0x1D0u;
-    int n = 0;
-    for (int t = 0; t < 9; ++t) {
-        if ((m >> t) & 1u) {
-            if (n == k) return t;
-            ++n;
-        }
-    }
-    return -1;
-}
-
 // ------------------------------------------------------------------------------ helpers
 
 __device__ __forceinline__ void cp_async4(void* smem, const void* gmem, bool valid) {
@@ -455,65 +439,206 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
 
 // ------------------------------------------------------------------------------ depthwise
 
-// One warp per (image, slot): channel co = perm[slot] convolves its own plane with its one
-// pattern (warp-uniform, compile-time taps).  Each lane produces outputs strided by 32.
-template <int S, int P_, typename T>
-__device__ __forceinline__ void dw_plane(const T* xp, T* yp, int H, int W, int Ho, int Wo, float4 w,
-                                         float b, int relu, int lane) {
-    constexpr int t0 = ktap(P_, 0), t1 = ktap(P_, 1), t2 = ktap(P_, 2), t3 = ktap(P_, 3);
-    const float wv[4] = {w.x, w.y, w.z, w.w};
-    constexpr int tt[4] = {t0, t1, t2, t3};
-    const int total = Ho * Wo;
-    for (int o = lane; o < total; o += 32) {
-        const int oy = o / Wo, ox = o % Wo;
-        float a = 0.0f;
+// Depthwise layers (one kernel per channel, as in MobileNet-V2) move 2-4 bytes per 8 useful
+// FLOP, so HBM bandwidth bounds them, not the FMA pipe.  The kernel is shaped for bandwidth:
+// every thread produces kDwVW consecutive outputs of one output row, reading the three input rows
+// it needs with 16-byte loads where rows are 16-byte aligned; the halo columns are single loads
+// that hit the neighbouring threads' lines in L1.  Each CTA first expands the four kept weights
+// of every plane it covers to the nine taps (zeros at the pruned taps, from the layer's own
+// masks) in shared memory, so every lane runs the same branch-free code even where one warp
+// covers planes of different patterns.
+constexpr int kDwThreads = 256;
+constexpr int kDwVW = 8;                   // outputs per thread along a row
+constexpr int kDwItemsPerCta = 2048;       // (plane, row, column group) items per CTA
+constexpr int kDwMaxPlanes = kDwThreads;   // planes per CTA (one decoding thread each)
+
+struct DwParams {
+    const void* x;
+    void* y;
+    const float* bias;
+    const uint32_t* perm;
+    const uint64_t* desc;
+    const uint32_t* kofs;
+    const float4* vals;
+    int N, C, H, W, Ho, Wo, relu;
+    int NS;                 // slots (G * 8): the planes of one image, in slot order
+    int NGX;                // column groups per output row
+    int ipp;                // items per plane: Ho * NGX
+    int ppc;                // planes per CTA (small planes), else 1
+    int tiles;              // CTAs per plane (large planes), else 1
+    uint16_t masks[kMaxPatterns];
+};
+
+template <typename T>
+__device__ __forceinline__ float ld_f32(const T* p) { return to_f32<T>(*p); }
+
+// NV consecutive elements (NV a multiple of 8, 16-byte aligned) widened to fp32
+template <int NV>
+__device__ __forceinline__ void ld_vec(const float* src, float* dst) {
+#pragma unroll
+    for (int i = 0; i < NV; i += 4) {
+        const float4 v = *reinterpret_cast<const float4*>(src + i);
+        dst[i] = v.x;
+        dst[i + 1] = v.y;
+        dst[i + 2] = v.z;
+        dst[i + 3] = v.w;
+    }
+}
+template <int NV>
+__device__ __forceinline__ void ld_vec(const __half* src, float* dst) {
+#pragma unroll
+    for (int i = 0; i < NV; i += 8) {
+        const uint4 u = *reinterpret_cast<const uint4*>(src + i);
+        const __half2* h = reinterpret_cast<const __half2*>(&u);
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-            const int iy = oy * S + tt[k] / 3 - 1, ix = ox * S + tt[k] % 3 - 1;
-            if (iy >= 0 && iy < H && ix >= 0 && ix < W) a = fmaf(wv[k], to_f32<T>(xp[(size_t)iy * W + ix]), a);
+            const float2 f = __half22float2(h[k]);
+            dst[i + 2 * k] = f.x;
+            dst[i + 2 * k + 1] = f.y;
         }
-        a += b;
-        yp[o] = from_f32<T>(relu ? fmaxf(a, 0.0f) : a);
     }
 }
 
-template <int S, typename T>
-__global__ void __launch_bounds__(256) pconv_depthwise(const T* __restrict__ x, T* __restrict__ y,
-                                                       const float* __restrict__ bias, const uint32_t* perm,
-                                                       const uint64_t* desc, const uint32_t* kofs,
-                                                       const float4* vals, int C, int H, int W, int Ho,
-                                                       int Wo, int G, int relu) {
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int g = blockIdx.x % G, n = blockIdx.x / G;
-    const int slot = g * kF + warp;
-    const uint32_t co = perm[slot];
-    if (co == kPadSlot) return;
-    uint64_t d = desc[g];
-    const int cnt = (int)(d & 15u);
-    d >>= 4;
-    int pat = -1, j = 0;
-    for (int e = 0; e < cnt; ++e) {
-        const int code = (int)((d >> (6 * e)) & 63u);
-        if ((code >> 3) == warp) { pat = code & 7; j = e; }
+template <int S, typename T, bool VIN, bool VOUT>
+__global__ void __launch_bounds__(kDwThreads) pconv_depthwise(const __grid_constant__ DwParams p) {
+    constexpr int NIN = (kDwVW - 1) * S + 3;     // input columns one thread reads per row
+    const T* x = static_cast<const T*>(p.x);
+    T* y = static_cast<T*>(p.y);
+    const int tid = threadIdx.x;
+    const long long planes = (long long)p.N * p.NS;
+    // this CTA's items: planes [pl0, pl0 + ppc) x all items, or items [it0, it0 + count) of plane pl0
+    long long pl0;
+    int it0, count;
+    if (p.tiles > 1) {
+        pl0 = blockIdx.x / p.tiles;
+        it0 = (blockIdx.x % p.tiles) * kDwItemsPerCta;
+        count = min(kDwItemsPerCta, p.ipp - it0);
+    } else {
+        pl0 = (long long)blockIdx.x * p.ppc;
+        it0 = 0;
+        count = (int)min((long long)p.ppc, planes - pl0) * p.ipp;
     }
-    const float b = bias ? bias[co] : 0.0f;
-    const T* xp = x + ((size_t)n * C + co) * H * W;
-    T* yp = y + ((size_t)n * C + co) * Ho * Wo;
-    if (pat < 0) {   // pruned kernel: the output is sigma(bias)
-        const float v = relu ? fmaxf(b, 0.0f) : b;
-        for (int o = lane; o < Ho * Wo; o += 32) yp[o] = from_f32<T>(v);
-        return;
+
+    // the CTA's planes: thread t < np decodes plane pl0 + t (its channel, nine taps and bias)
+    __shared__ float s_w[kDwMaxPlanes][10];
+    __shared__ int s_co[kDwMaxPlanes];
+    const int np = p.tiles > 1 ? 1 : (int)min((long long)p.ppc, planes - pl0);
+    if (tid < np) {
+        const long long plane = pl0 + tid;
+        const int n = (int)(plane / p.NS), s = (int)(plane - (long long)n * p.NS);
+        const uint32_t co = p.perm[s];
+        float w9[9] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        float b = 0.0f;
+        if (co != kPadSlot) {
+            const int g = s >> 3, f = s & 7;
+            const uint64_t d = p.desc[g];
+            const int cnt = (int)(d & 15u);
+            int pat = -1;
+            uint32_t k0 = p.kofs[g];
+            for (int j = 0; j < cnt; ++j) {
+                const int code = (int)((d >> (4 + 6 * j)) & 63u);
+                if ((code >> 3) == f) { pat = code & 7; k0 += j; }
+            }
+            // a pruned kernel has no entry: all nine taps zero, the output is the bias
+            const float4 v = pat >= 0 ? p.vals[k0] : make_float4(0.f, 0.f, 0.f, 0.f);
+            const unsigned m = pat >= 0 ? p.masks[pat] : 0u;
+            int k = 0;
+#pragma unroll
+            for (int t = 0; t < 9; ++t) {
+                const bool on = (m >> t) & 1u;
+                const float vk = k == 0 ? v.x : k == 1 ? v.y : k == 2 ? v.z : v.w;
+                w9[t] = on ? vk : 0.0f;
+                k += on ? 1 : 0;
+            }
+            b = p.bias ? p.bias[co] : 0.0f;
+        }
+#pragma unroll
+        for (int t = 0; t < 9; ++t) s_w[tid][t] = w9[t];
+        s_w[tid][9] = b;
+        s_co[tid] = co == kPadSlot ? -1 : (int)co;
     }
-    const float4 w = vals[kofs[g] + j];
-    switch (pat) {
-        case 0: dw_plane<S, 0, T>(xp, yp, H, W, Ho, Wo, w, b, relu, lane); break;
-        case 1: dw_plane<S, 1, T>(xp, yp, H, W, Ho, Wo, w, b, relu, lane); break;
-        case 2: dw_plane<S, 2, T>(xp, yp, H, W, Ho, Wo, w, b, relu, lane); break;
-        case 3: dw_plane<S, 3, T>(xp, yp, H, W, Ho, Wo, w, b, relu, lane); break;
-        case 4: dw_plane<S, 4, T>(xp, yp, H, W, Ho, Wo, w, b, relu, lane); break;
-        case 5: dw_plane<S, 5, T>(xp, yp, H, W, Ho, Wo, w, b, relu, lane); break;
-        case 6: dw_plane<S, 6, T>(xp, yp, H, W, Ho, Wo, w, b, relu, lane); break;
-        default: dw_plane<S, 7, T>(xp, yp, H, W, Ho, Wo, w, b, relu, lane); break;
+    __syncthreads();
+
+    // item e = pl * ipp + it0 + oy * NGX + gx as digits (pl, oy, gx), stepped by the thread count
+    // with at most one carry per digit
+    const int e = it0 + tid;
+    int pl = e / p.ipp;
+    const int rem = e - pl * p.ipp;
+    int oy = rem / p.NGX, gx = rem - (rem / p.NGX) * p.NGX;
+    int st = kDwThreads;
+    const int s_pl = st / p.ipp;
+    st -= s_pl * p.ipp;
+    const int s_oy = st / p.NGX, s_gx = st - (st / p.NGX) * p.NGX;
+
+    for (int i = tid; i < count; i += kDwThreads) {
+        const int co = s_co[pl];
+        if (co >= 0) {
+            const int n = (int)((pl0 + pl) / p.NS);
+            const T* xp = x + ((size_t)n * p.C + co) * p.H * p.W;
+            T* yp = y + ((size_t)n * p.C + co) * p.Ho * p.Wo;
+            float w9[9];
+#pragma unroll
+            for (int t = 0; t < 9; ++t) w9[t] = s_w[pl][t];
+            const float b = s_w[pl][9];
+            const int c0 = kDwVW * gx;            // first output column of this thread
+            const int ic = c0 * S - 1;            // first input column it reads
+            float acc[kDwVW];
+#pragma unroll
+            for (int j = 0; j < kDwVW; ++j) acc[j] = b;
+#pragma unroll
+            for (int dy = 0; dy < 3; ++dy) {
+                const int iy = oy * S - 1 + dy;
+                if (iy < 0 || iy >= p.H) continue;
+                const T* row = xp + (size_t)iy * p.W;
+                float r[NIN];
+                if (VIN && ic + 1 + kDwVW * S <= p.W) {
+                    // columns ic+1 .. ic+kDwVW*S as 16-byte vectors, the halo columns alone
+                    ld_vec<kDwVW * S>(row + ic + 1, r + 1);
+                    r[0] = ic >= 0 ? ld_f32(row + ic) : 0.0f;
+                    if (S == 1) r[NIN - 1] = ic + NIN - 1 < p.W ? ld_f32(row + ic + NIN - 1) : 0.0f;
+                } else {
+#pragma unroll
+                    for (int c = 0; c < NIN; ++c) {
+                        const int xc = ic + c;
+                        r[c] = (xc >= 0 && xc < p.W) ? ld_f32(row + xc) : 0.0f;
+                    }
+                }
+#pragma unroll
+                for (int j = 0; j < kDwVW; ++j)
+#pragma unroll
+                    for (int dx = 0; dx < 3; ++dx) acc[j] = fmaf(w9[3 * dy + dx], r[j * S + dx], acc[j]);
+            }
+            T* out = yp + (size_t)oy * p.Wo + c0;
+            if (VOUT && c0 + kDwVW <= p.Wo) {
+                if constexpr (sizeof(T) == 4) {
+                    float v[kDwVW];
+#pragma unroll
+                    for (int j = 0; j < kDwVW; ++j) v[j] = p.relu ? fmaxf(acc[j], 0.0f) : acc[j];
+                    float4* o4 = reinterpret_cast<float4*>(out);
+                    o4[0] = make_float4(v[0], v[1], v[2], v[3]);
+                    o4[1] = make_float4(v[4], v[5], v[6], v[7]);
+                } else {
+                    uint4 u;
+                    __half2* h = reinterpret_cast<__half2*>(&u);
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        const float a0 = p.relu ? fmaxf(acc[2 * k], 0.0f) : acc[2 * k];
+                        const float a1 = p.relu ? fmaxf(acc[2 * k + 1], 0.0f) : acc[2 * k + 1];
+                        h[k] = __floats2half2_rn(a0, a1);
+                    }
+                    *reinterpret_cast<uint4*>(out) = u;
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < kDwVW; ++j)
+                    if (c0 + j < p.Wo) out[j] = from_f32<T>(p.relu ? fmaxf(acc[j], 0.0f) : acc[j]);
+            }
+        }
+        gx += s_gx;
+        if (gx >= p.NGX) { gx -= p.NGX; ++oy; }
+        oy += s_oy;
+        if (oy >= p.Ho) { oy -= p.Ho; ++pl; }
+        pl += s_pl;
     }
 }
 
@@ -877,25 +1002,57 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
     return PP_OK;
 }
 
+template <int S, typename T>
+int launch_depthwise_s(const DwParams& p, unsigned ctas, bool vin, bool vout, cudaStream_t st) {
+    if (vin && vout) pconv_depthwise<S, T, true, true><<<ctas, kDwThreads, 0, st>>>(p);
+    else if (vin) pconv_depthwise<S, T, true, false><<<ctas, kDwThreads, 0, st>>>(p);
+    else if (vout) pconv_depthwise<S, T, false, true><<<ctas, kDwThreads, 0, st>>>(p);
+    else pconv_depthwise<S, T, false, false><<<ctas, kDwThreads, 0, st>>>(p);
+    return cudaGetLastError() == cudaSuccess ? PP_OK : PP_ERR_CUDA;
+}
+
 template <typename T>
 int launch_depthwise(const pp_layer* L, const void* x, void* y, const float* bias, int relu, int N, int H, int W,
                      int Ho, int Wo, cudaStream_t st) {
     const unsigned char* img = static_cast<const unsigned char*>(L->dev);
-    const auto* perm = reinterpret_cast<const uint32_t*>(img + L->off_perm);
-    const auto* desc = reinterpret_cast<const uint64_t*>(img + L->off_desc);
-    const auto* kofs = reinterpret_cast<const uint32_t*>(img + L->off_kofs);
-    const auto* vals = reinterpret_cast<const float4*>(img + L->off_vals);
-    const long long blocks = (long long)N * L->G;
-    if (blocks > INT_MAX) return PP_ERR_SHAPE;
-    if (L->stride == 1)
-        pconv_depthwise<1, T><<<(unsigned)blocks, 256, 0, st>>>(static_cast<const T*>(x), static_cast<T*>(y), bias,
-                                                                 perm, desc, kofs, vals, L->cout, H, W, Ho, Wo,
-                                                                 L->G, relu);
-    else
-        pconv_depthwise<2, T><<<(unsigned)blocks, 256, 0, st>>>(static_cast<const T*>(x), static_cast<T*>(y), bias,
-                                                                 perm, desc, kofs, vals, L->cout, H, W, Ho, Wo,
-                                                                 L->G, relu);
-    return cudaGetLastError() == cudaSuccess ? PP_OK : PP_ERR_CUDA;
+    DwParams p{};
+    p.x = x;
+    p.y = y;
+    p.bias = bias;
+    p.perm = reinterpret_cast<const uint32_t*>(img + L->off_perm);
+    p.desc = reinterpret_cast<const uint64_t*>(img + L->off_desc);
+    p.kofs = reinterpret_cast<const uint32_t*>(img + L->off_kofs);
+    p.vals = reinterpret_cast<const float4*>(img + L->off_vals);
+    p.N = N;
+    p.C = L->cout;
+    p.H = H;
+    p.W = W;
+    p.Ho = Ho;
+    p.Wo = Wo;
+    p.relu = relu;
+    p.NS = L->G * kF;
+    p.NGX = (Wo + kDwVW - 1) / kDwVW;
+    for (int i = 0; i < kMaxPatterns; ++i) p.masks[i] = i < L->n_patterns ? L->masks[i] : 0;
+    const long long ipp = (long long)Ho * p.NGX;
+    const long long planes = (long long)N * p.NS;
+    if (ipp > INT_MAX / 2) return PP_ERR_SHAPE;
+    p.ipp = (int)ipp;
+    long long ctas;
+    if (ipp > kDwItemsPerCta) {
+        p.tiles = (int)((ipp + kDwItemsPerCta - 1) / kDwItemsPerCta);
+        p.ppc = 1;
+        ctas = planes * p.tiles;
+    } else {
+        p.tiles = 1;
+        p.ppc = (int)std::min<long long>(kDwItemsPerCta / ipp, kDwMaxPlanes);
+        ctas = (planes + p.ppc - 1) / p.ppc;
+    }
+    if (ctas > INT_MAX) return PP_ERR_SHAPE;
+    const size_t es = sizeof(T);
+    const bool vin = ((size_t)W * es) % 16 == 0 && reinterpret_cast<uintptr_t>(x) % 16 == 0;
+    const bool vout = ((size_t)Wo * es) % 16 == 0 && reinterpret_cast<uintptr_t>(y) % 16 == 0;
+    return L->stride == 1 ? launch_depthwise_s<1, T>(p, (unsigned)ctas, vin, vout, st)
+                          : launch_depthwise_s<2, T>(p, (unsigned)ctas, vin, vout, st);
 }
 
 template <typename T>
@@ -987,13 +1144,13 @@ int pp_conv_ws(pp_handle h, const void* x, int dtype, int N, int H, int W, const
     const int Ho = (H - 1) / h->stride + 1, Wo = (W - 1) / h->stride + 1;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const bool f16 = dtype == PP_F16;
+    if (h->depthwise) {   // any pattern library: the kernel expands each channel's taps itself
+        return f16 ? launch_depthwise<__half>(h, x, y, bias, relu, N, H, W, Ho, Wo, st)
+                   : launch_depthwise<float>(h, x, y, bias, relu, N, H, W, Ho, Wo, st);
+    }
     if (!h->fast) {
         return f16 ? launch_generic<__half>(h, x, y, bias, relu, N, H, W, Ho, Wo, st)
                    : launch_generic<float>(h, x, y, bias, relu, N, H, W, Ho, Wo, st);
-    }
-    if (h->depthwise) {
-        return f16 ? launch_depthwise<__half>(h, x, y, bias, relu, N, H, W, Ho, Wo, st)
-                   : launch_depthwise<float>(h, x, y, bias, relu, N, H, W, Ho, Wo, st);
     }
     if (workspace) {
         const size_t es = f16 ? 2 : 4;
@@ -1019,7 +1176,7 @@ int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64
     if (N < 1 || H < 1 || W < 1 || n_info < 1) return PP_ERR_SHAPE;
     int64_t v[12] = {0};
     if (!h->fast || h->depthwise) {
-        v[0] = h->fast ? 2 : 3;   // depthwise kernel / generic kernel: no plan, no workspace
+        v[0] = h->depthwise ? 2 : 3;   // depthwise kernel / generic kernel: no plan, no workspace
     } else {
         Plan pl;
         const int rc = make_plan(h, N, H, W, workspace_bytes, &pl);

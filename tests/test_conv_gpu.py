@@ -143,6 +143,22 @@ def test_depthwise(dtype, stride):
     check(Wd, x, b, 0.5, stride, depthwise=True, dtype=dtype)     # pruned channels -> sigma(b)
 
 
+@pytest.mark.parametrize("dtype", [torch.float32, torch.float16])
+@pytest.mark.parametrize("N,C,H,W,stride", [(1, 8, 160, 160, 1),    # one plane over two CTAs
+                                            (1, 8, 160, 160, 2),
+                                            (2, 16, 32, 48, 1),     # 16-byte rows in both dtypes
+                                            (2, 16, 32, 48, 2),
+                                            (3, 40, 7, 7, 1),       # many small planes per CTA
+                                            (2, 24, 14, 14, 2)])
+def test_depthwise_vector_and_tiled(dtype, N, C, H, W, stride):
+    rng = np.random.default_rng(C * 7 + H)
+    Wd = (rng.standard_normal((C, 1, 3, 3)) * np.sqrt(2 / 9)).astype(np.float32)
+    x = rnd((N, C, H, W), H + W, dtype=_np_dt(dtype))
+    b = (rng.standard_normal(C) * 0.1).astype(np.float32)
+    check(Wd, x, b, 1.0, stride, depthwise=True, dtype=dtype, guard=64)
+    check(Wd, x, b, 0.7, stride, relu=False, depthwise=True, dtype=dtype, guard=64)
+
+
 def test_deterministic_and_zero_batch():
     L = WL.single_layer()
     x = WL.layer_input(L, 2)
