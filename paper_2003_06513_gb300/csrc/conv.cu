@@ -520,7 +520,7 @@ __global__ void __launch_bounds__(kDwThreads) pconv_depthwise(const __grid_const
     }
 
     // the CTA's planes: thread t < np decodes plane pl0 + t (its channel, nine taps and bias)
-    __shared__ float s_w[kDwMaxPlanes][10];
+    __shared__ float s_w[kDwMaxPlanes][11];
     __shared__ int s_co[kDwMaxPlanes];
     const int np = p.tiles > 1 ? 1 : (int)min((long long)p.ppc, planes - pl0);
     if (tid < np) {
@@ -529,6 +529,7 @@ __global__ void __launch_bounds__(kDwThreads) pconv_depthwise(const __grid_const
         const uint32_t co = p.perm[s];
         float w9[9] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
         float b = 0.0f;
+        unsigned mask_of_slot = 0;
         if (co != kPadSlot) {
             const int g = s >> 3, f = s & 7;
             const uint64_t d = p.desc[g];
@@ -542,6 +543,7 @@ __global__ void __launch_bounds__(kDwThreads) pconv_depthwise(const __grid_const
             // a pruned kernel has no entry: all nine taps zero, the output is the bias
             const float4 v = pat >= 0 ? p.vals[k0] : make_float4(0.f, 0.f, 0.f, 0.f);
             const unsigned m = pat >= 0 ? p.masks[pat] : 0u;
+            mask_of_slot = m;
             int k = 0;
 #pragma unroll
             for (int t = 0; t < 9; ++t) {
@@ -555,6 +557,7 @@ __global__ void __launch_bounds__(kDwThreads) pconv_depthwise(const __grid_const
 #pragma unroll
         for (int t = 0; t < 9; ++t) s_w[tid][t] = w9[t];
         s_w[tid][9] = b;
+        s_w[tid][10] = __uint_as_float(co == kPadSlot ? 0u : mask_of_slot);
         s_co[tid] = co == kPadSlot ? -1 : (int)co;
     }
     __syncthreads();
@@ -580,6 +583,7 @@ __global__ void __launch_bounds__(kDwThreads) pconv_depthwise(const __grid_const
 #pragma unroll
             for (int t = 0; t < 9; ++t) w9[t] = s_w[pl][t];
             const float b = s_w[pl][9];
+            const unsigned m = __float_as_uint(s_w[pl][10]);
             const int c0 = kDwVW * gx;            // first output column of this thread
             const int ic = c0 * S - 1;            // first input column it reads
             float acc[kDwVW];
@@ -604,9 +608,11 @@ __global__ void __launch_bounds__(kDwThreads) pconv_depthwise(const __grid_const
                     }
                 }
 #pragma unroll
-                for (int j = 0; j < kDwVW; ++j)
+                for (int dx = 0; dx < 3; ++dx) {
+                    if (!((m >> (3 * dy + dx)) & 1u)) continue;   // pruned tap
 #pragma unroll
-                    for (int dx = 0; dx < 3; ++dx) acc[j] = fmaf(w9[3 * dy + dx], r[j * S + dx], acc[j]);
+                    for (int j = 0; j < kDwVW; ++j) acc[j] = fmaf(w9[3 * dy + dx], r[j * S + dx], acc[j]);
+                }
             }
             T* out = yp + (size_t)oy * p.Wo + c0;
             if (VOUT && c0 + kDwVW <= p.Wo) {
@@ -640,6 +646,214 @@ __global__ void __launch_bounds__(kDwThreads) pconv_depthwise(const __grid_const
         if (oy >= p.Ho) { oy -= p.Ho; ++pl; }
         pl += s_pl;
     }
+}
+
+// Staged variant (16-byte aligned x): tiles in channel order, so that a tile's input is one
+// contiguous run of memory: npl consecutive channels of one image as whole planes, or one
+// channel's band of output rows (npl == 1).  A persistent CTA copies its next tile into shared
+// memory with 16-byte cp.async (at the run's own alignment phase) while it computes the current
+// one, keeping HBM busy whatever the row width; the slot of every channel comes from an inverse
+// of the filter permutation built once per CTA.
+struct DwStagedParams {
+    const void* x;
+    void* y;
+    const float* bias;
+    const uint32_t* perm;
+    const uint64_t* desc;
+    const uint32_t* kofs;
+    const float4* vals;
+    int N, C, H, W, Ho, Wo, relu;
+    int NS, NGX;
+    int npl, rb, n_cg, n_bands;   // tile: npl channels x rb output rows; channel groups; bands
+    int n_tiles;
+    long long total_in;           // elements of x
+    int buf_elems;                // elements per staging buffer
+    unsigned off_w, off_buf;      // shared-memory layout: inverse permutation | taps | 2 buffers
+    uint16_t masks[kMaxPatterns];
+};
+
+template <int S, typename T, bool VIN, bool VOUT>
+__global__ void __launch_bounds__(kDwThreads) pconv_depthwise_staged(const __grid_constant__ DwStagedParams p) {
+    constexpr int VE = 16 / (int)sizeof(T);      // elements per 16-byte copy
+    constexpr int NIN = (kDwVW - 1) * S + 3;
+    extern __shared__ __align__(16) unsigned char dsm[];
+    int* s_inv = reinterpret_cast<int*>(dsm);
+    float* s_w = reinterpret_cast<float*>(dsm + p.off_w);
+    T* bufs = reinterpret_cast<T*>(dsm + p.off_buf);
+    const T* x = static_cast<const T*>(p.x);
+    T* y = static_cast<T*>(p.y);
+    const int tid = threadIdx.x;
+
+    for (int s = tid; s < p.NS; s += kDwThreads) {
+        const uint32_t co = p.perm[s];
+        if (co != kPadSlot) s_inv[co] = s;
+    }
+
+    struct Tile {
+        int n, c0, np, oy0, nro, iy_lo, nri;
+        long long g0;       // first input element of the run
+    };
+    auto tile_of = [&](int t) {
+        Tile u;
+        const int band = t % p.n_bands;
+        const int q = t / p.n_bands;
+        const int cg = q % p.n_cg;
+        u.n = q / p.n_cg;
+        u.c0 = cg * p.npl;
+        u.np = min(p.npl, p.C - u.c0);
+        u.oy0 = band * p.rb;
+        u.nro = min(p.rb, p.Ho - u.oy0);
+        u.iy_lo = max(0, u.oy0 * S - 1);
+        const int iy_hi = min(p.H - 1, (u.oy0 + u.nro - 1) * S + 1);
+        u.nri = iy_hi - u.iy_lo + 1;
+        u.g0 = ((long long)u.n * p.C + u.c0) * p.H * p.W + (long long)u.iy_lo * p.W;
+        return u;
+    };
+    // issue the copy of tile t's run into buffer b: whole 16-byte blocks from the block holding
+    // its first element (plain loads for a block that reaches past the end of x)
+    auto load = [&](const Tile& u, int b) {
+        T* buf = bufs + (size_t)b * p.buf_elems;
+        const long long len = (long long)u.np * u.nri * p.W;
+        const long long v_lo = u.g0 / VE, v_hi = (u.g0 + len - 1) / VE;
+        for (long long v = v_lo + tid; v <= v_hi; v += kDwThreads) {
+            const long long ge = v * VE;
+            T* dst = buf + (ge - v_lo * VE);
+            if (ge + VE <= p.total_in) {
+                cp_async16(dst, x + ge);
+            } else {
+                for (int k = 0; k < VE; ++k)
+                    if (ge + k < p.total_in) dst[k] = x[ge + k];
+            }
+        }
+    };
+    // thread t < np: taps and bias of the tile's channel c0 + t
+    auto decode = [&](const Tile& u) {
+        if (tid < u.np) {
+            const int s = s_inv[u.c0 + tid];
+            const int g = s >> 3, f = s & 7;
+            const uint64_t d = p.desc[g];
+            const int cnt = (int)(d & 15u);
+            int pat = -1;
+            uint32_t k0 = p.kofs[g];
+            for (int j = 0; j < cnt; ++j) {
+                const int code = (int)((d >> (4 + 6 * j)) & 63u);
+                if ((code >> 3) == f) { pat = code & 7; k0 += j; }
+            }
+            const float4 v = pat >= 0 ? p.vals[k0] : make_float4(0.f, 0.f, 0.f, 0.f);
+            const unsigned m = pat >= 0 ? p.masks[pat] : 0u;
+            int k = 0;
+#pragma unroll
+            for (int t = 0; t < 9; ++t) {
+                const bool on = (m >> t) & 1u;
+                const float vk = k == 0 ? v.x : k == 1 ? v.y : k == 2 ? v.z : v.w;
+                s_w[tid * 11 + t] = on ? vk : 0.0f;
+                k += on ? 1 : 0;
+            }
+            s_w[tid * 11 + 9] = p.bias ? p.bias[u.c0 + tid] : 0.0f;
+            s_w[tid * 11 + 10] = __uint_as_float(m);
+        }
+    };
+    auto compute = [&](const Tile& u, int b) {
+        const T* buf = bufs + (size_t)b * p.buf_elems;
+        const int off0 = (int)(u.g0 - (u.g0 / VE) * VE);   // buffer index of the run's first element
+        const int per_pl = u.nro * p.NGX;
+        const int items = u.np * per_pl;
+        int pl = tid / per_pl;
+        const int rem = tid - pl * per_pl;
+        int oyl = rem / p.NGX, gx = rem - (rem / p.NGX) * p.NGX;
+        int st = kDwThreads;
+        const int s_pl = st / per_pl;
+        st -= s_pl * per_pl;
+        const int s_oy = st / p.NGX, s_gx = st - (st / p.NGX) * p.NGX;
+        int cur = -1;
+        float w9[9], bv = 0.0f;
+        unsigned m = 0;
+        for (int i = tid; i < items; i += kDwThreads) {
+            if (pl != cur) {
+                cur = pl;
+#pragma unroll
+                for (int t = 0; t < 9; ++t) w9[t] = s_w[pl * 11 + t];
+                bv = s_w[pl * 11 + 9];
+                m = __float_as_uint(s_w[pl * 11 + 10]);
+            }
+            const int oy = u.oy0 + oyl;
+            const int c0 = kDwVW * gx, ic = c0 * S - 1;
+            float acc[kDwVW];
+#pragma unroll
+            for (int j = 0; j < kDwVW; ++j) acc[j] = bv;
+#pragma unroll
+            for (int dy = 0; dy < 3; ++dy) {
+                const int iy = oy * S - 1 + dy;
+                if (iy < 0 || iy >= p.H) continue;
+                const T* row = buf + off0 + (pl * u.nri + iy - u.iy_lo) * p.W;
+                float r[NIN];
+                if (VIN && ic + 1 + kDwVW * S <= p.W) {   // rows 16-byte aligned in the buffer too
+                    ld_vec<kDwVW * S>(row + ic + 1, r + 1);
+                    r[0] = ic >= 0 ? ld_f32(row + ic) : 0.0f;
+                    if (S == 1) r[NIN - 1] = ic + NIN - 1 < p.W ? ld_f32(row + ic + NIN - 1) : 0.0f;
+                } else {
+#pragma unroll
+                    for (int c = 0; c < NIN; ++c) {
+                        const int xc = ic + c;
+                        r[c] = (xc >= 0 && xc < p.W) ? ld_f32(row + xc) : 0.0f;
+                    }
+                }
+#pragma unroll
+                for (int dx = 0; dx < 3; ++dx) {
+                    if (!((m >> (3 * dy + dx)) & 1u)) continue;   // pruned tap
+#pragma unroll
+                    for (int j = 0; j < kDwVW; ++j) acc[j] = fmaf(w9[3 * dy + dx], r[j * S + dx], acc[j]);
+                }
+            }
+            T* out = y + (((size_t)u.n * p.C + u.c0 + pl) * p.Ho + oy) * p.Wo + c0;
+            if (VOUT && c0 + kDwVW <= p.Wo) {
+                if constexpr (sizeof(T) == 4) {
+                    float v[kDwVW];
+#pragma unroll
+                    for (int j = 0; j < kDwVW; ++j) v[j] = p.relu ? fmaxf(acc[j], 0.0f) : acc[j];
+                    float4* o4 = reinterpret_cast<float4*>(out);
+                    o4[0] = make_float4(v[0], v[1], v[2], v[3]);
+                    o4[1] = make_float4(v[4], v[5], v[6], v[7]);
+                } else {
+                    uint4 q;
+                    __half2* h = reinterpret_cast<__half2*>(&q);
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        const float a0 = p.relu ? fmaxf(acc[2 * k], 0.0f) : acc[2 * k];
+                        const float a1 = p.relu ? fmaxf(acc[2 * k + 1], 0.0f) : acc[2 * k + 1];
+                        h[k] = __floats2half2_rn(a0, a1);
+                    }
+                    *reinterpret_cast<uint4*>(out) = q;
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < kDwVW; ++j)
+                    if (c0 + j < p.Wo) out[j] = from_f32<T>(p.relu ? fmaxf(acc[j], 0.0f) : acc[j]);
+            }
+            gx += s_gx;
+            if (gx >= p.NGX) { gx -= p.NGX; ++oyl; }
+            oyl += s_oy;
+            if (oyl >= u.nro) { oyl -= u.nro; ++pl; }
+            pl += s_pl;
+        }
+    };
+
+    int t = blockIdx.x;
+    if (t < p.n_tiles) load(tile_of(t), 0);
+    asm volatile("cp.async.commit_group;" ::: "memory");
+    __syncthreads();                                   // s_inv complete
+    for (int k = 0; t < p.n_tiles; ++k, t += gridDim.x) {
+        const Tile u = tile_of(t);
+        const int tn = t + (int)gridDim.x;
+        if (tn < p.n_tiles) load(tile_of(tn), (k + 1) & 1);
+        asm volatile("cp.async.commit_group;" ::: "memory");
+        decode(u);
+        asm volatile("cp.async.wait_group 1;" ::: "memory");
+        __syncthreads();                               // tile t staged, its taps decoded
+        compute(u, k & 1);
+        __syncthreads();                               // buffer k & 1 and the taps free again
+    }
+    asm volatile("cp.async.wait_all;" ::: "memory");
 }
 
 // ------------------------------------------------------------------------------ generic path
@@ -1011,9 +1225,112 @@ int launch_depthwise_s(const DwParams& p, unsigned ctas, bool vin, bool vout, cu
     return cudaGetLastError() == cudaSuccess ? PP_OK : PP_ERR_CUDA;
 }
 
+template <int S, typename T, bool VIN, bool VOUT>
+bool dw_staged_smem(size_t need) {
+    static std::atomic<int> done[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+    if (done[dev].load(std::memory_order_acquire)) return true;
+    int optin = 0;
+    if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess) return false;
+    if ((size_t)optin < need) return false;
+    if (cudaFuncSetAttribute(pconv_depthwise_staged<S, T, VIN, VOUT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             optin) != cudaSuccess)
+        return false;
+    done[dev].store(1, std::memory_order_release);
+    return true;
+}
+
+template <int S, typename T, bool VIN, bool VOUT>
+int launch_dw_staged(const DwStagedParams& p, size_t smem, cudaStream_t st) {
+    if (!dw_staged_smem<S, T, VIN, VOUT>(smem)) return PP_ERR_CUDA;
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, pconv_depthwise_staged<S, T, VIN, VOUT>, kDwThreads,
+                                                      smem) != cudaSuccess || per_sm < 1)
+        return PP_ERR_CUDA;
+    const long long ctas = std::min<long long>(p.n_tiles, (long long)sm_count() * per_sm);
+    pconv_depthwise_staged<S, T, VIN, VOUT><<<(unsigned)ctas, kDwThreads, smem, st>>>(p);
+    return cudaGetLastError() == cudaSuccess ? PP_OK : PP_ERR_CUDA;
+}
+
+template <int S, typename T>
+int launch_dw_staged_s(const DwStagedParams& p, size_t smem, bool vin, bool vout, cudaStream_t st) {
+    if (vin && vout) return launch_dw_staged<S, T, true, true>(p, smem, st);
+    if (vin) return launch_dw_staged<S, T, true, false>(p, smem, st);
+    if (vout) return launch_dw_staged<S, T, false, true>(p, smem, st);
+    return launch_dw_staged<S, T, false, false>(p, smem, st);
+}
+
+constexpr size_t kDwStageBytes = 16384;   // one staging buffer of the staged depthwise kernel
+
+// Tile shape and shared-memory layout of the staged depthwise kernel; false when it does not
+// apply (x not 16-byte aligned, a plane row wider than a buffer, too many channels to invert).
+template <typename T>
+bool dw_staged_plan(const pp_layer* L, const void* x, int N, int H, int W, int Ho, DwStagedParams* p,
+                    size_t* smem) {
+    const int S = L->stride;
+    const long long es = sizeof(T), VE = 16 / es;
+    const long long budget = kDwStageBytes / es;
+    // rows that are 16-byte aligned already load as vectors straight from global memory
+    if (reinterpret_cast<uintptr_t>(x) % 16 != 0 || ((size_t)W * es) % 16 == 0 || L->cout > 8192) return false;
+    const long long plane = (long long)H * W;
+    if (plane <= budget) {
+        p->npl = (int)std::min<long long>({(long long)L->cout, budget / plane, (long long)kDwMaxPlanes});
+        p->rb = Ho;
+        p->n_bands = 1;
+    } else {
+        const long long rows_in = budget / W;
+        if (rows_in < 3) return false;
+        p->npl = 1;
+        p->rb = (int)((rows_in - 3) / S + 1);
+        p->n_bands = (Ho + p->rb - 1) / p->rb;
+    }
+    p->n_cg = (L->cout + p->npl - 1) / p->npl;
+    const long long n_tiles = (long long)N * p->n_cg * p->n_bands;
+    if (n_tiles > INT_MAX) return false;
+    p->n_tiles = (int)n_tiles;
+    const long long max_rows = p->n_bands == 1 ? H : std::min<long long>(H, (long long)(p->rb - 1) * S + 3);
+    const long long max_len = (long long)p->npl * max_rows * W;
+    p->buf_elems = (int)((max_len + 2 * VE + VE - 1) / VE * VE);
+    p->total_in = (long long)N * L->cout * H * W;
+    p->off_w = (unsigned)align_up((size_t)L->cout * 4, 16);
+    p->off_buf = (unsigned)align_up(p->off_w + (size_t)kDwMaxPlanes * 11 * 4, 16);
+    *smem = p->off_buf + 2 * (size_t)p->buf_elems * es;
+    return true;
+}
+
 template <typename T>
 int launch_depthwise(const pp_layer* L, const void* x, void* y, const float* bias, int relu, int N, int H, int W,
                      int Ho, int Wo, cudaStream_t st) {
+    {
+        const unsigned char* img = static_cast<const unsigned char*>(L->dev);
+        DwStagedParams q{};
+        size_t smem = 0;
+        if (dw_staged_plan<T>(L, x, N, H, W, Ho, &q, &smem)) {
+            q.x = x;
+            q.y = y;
+            q.bias = bias;
+            q.perm = reinterpret_cast<const uint32_t*>(img + L->off_perm);
+            q.desc = reinterpret_cast<const uint64_t*>(img + L->off_desc);
+            q.kofs = reinterpret_cast<const uint32_t*>(img + L->off_kofs);
+            q.vals = reinterpret_cast<const float4*>(img + L->off_vals);
+            q.N = N;
+            q.C = L->cout;
+            q.H = H;
+            q.W = W;
+            q.Ho = Ho;
+            q.Wo = Wo;
+            q.relu = relu;
+            q.NS = L->G * kF;
+            q.NGX = (Wo + kDwVW - 1) / kDwVW;
+            for (int i = 0; i < kMaxPatterns; ++i) q.masks[i] = i < L->n_patterns ? L->masks[i] : 0;
+            const size_t es = sizeof(T);
+            const bool vin = ((size_t)W * es) % 16 == 0;
+            const bool vout = ((size_t)Wo * es) % 16 == 0 && reinterpret_cast<uintptr_t>(y) % 16 == 0;
+            return L->stride == 1 ? launch_dw_staged_s<1, T>(q, smem, vin, vout, st)
+                                  : launch_dw_staged_s<2, T>(q, smem, vin, vout, st);
+        }
+    }
     const unsigned char* img = static_cast<const unsigned char*>(L->dev);
     DwParams p{};
     p.x = x;

@@ -149,7 +149,9 @@ def test_depthwise(dtype, stride):
                                             (2, 16, 32, 48, 1),     # 16-byte rows in both dtypes
                                             (2, 16, 32, 48, 2),
                                             (3, 40, 7, 7, 1),       # many small planes per CTA
-                                            (2, 24, 14, 14, 2)])
+                                            (2, 24, 14, 14, 2),
+                                            (1, 4, 9, 2100, 1),     # rows too wide to stage whole
+                                            (1, 4, 9, 2100, 2)])
 def test_depthwise_vector_and_tiled(dtype, N, C, H, W, stride):
     rng = np.random.default_rng(C * 7 + H)
     Wd = (rng.standard_normal((C, 1, 3, 3)) * np.sqrt(2 / 9)).astype(np.float32)
@@ -157,6 +159,25 @@ def test_depthwise_vector_and_tiled(dtype, N, C, H, W, stride):
     b = (rng.standard_normal(C) * 0.1).astype(np.float32)
     check(Wd, x, b, 1.0, stride, depthwise=True, dtype=dtype, guard=64)
     check(Wd, x, b, 0.7, stride, relu=False, depthwise=True, dtype=dtype, guard=64)
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.float16])
+def test_depthwise_unaligned_input(dtype):
+    """x 8 bytes off a 16-byte boundary: the direct (unstaged) depthwise kernel."""
+    rng = np.random.default_rng(31)
+    C, H, W = 12, 20, 24
+    Wd = (rng.standard_normal((C, 1, 3, 3)) * np.sqrt(2 / 9)).astype(np.float32)
+    x = rnd((2, C, H, W), 32, dtype=_np_dt(dtype))
+    b = (rng.standard_normal(C) * 0.1).astype(np.float32)
+    layer = api.pp_pack(Wd, None, 1.0, C, 1).bind("cuda")
+    off = 8 // x.itemsize
+    flat = torch.empty(x.size + off, dtype=dtype, device="cuda")
+    xt = flat[off:].view(x.shape)
+    xt.copy_(torch.from_numpy(x))
+    assert xt.data_ptr() % 16 == 8
+    y = layer.conv(xt, torch.from_numpy(b).cuda(), True)
+    ref, den = oracle(Wd, x, b, 1.0, 1, True, True)
+    assert OC.max_norm_err(y.double().cpu().numpy(), ref, den) <= TOL[dtype]
 
 
 def test_deterministic_and_zero_batch():
