@@ -50,8 +50,9 @@ typedef enum {
     PP_ERR_CUDA = -10,        /* a CUDA runtime call failed (launch or copy)                 */
     PP_ERR_ARG = -11,         /* any other invalid argument (section, query key, flag)       */
     PP_ERR_ALLOC = -12,       /* host allocation failed                                      */
-    PP_ERR_SCRATCH = -13      /* pp_conv_static_scratch: the call needs more scratch than the
+    PP_ERR_SCRATCH = -13,     /* pp_conv_static_scratch: the call needs more scratch than the
                                  static array holds                                           */
+    PP_ERR_PATH = -14         /* the layer's kernel does not offer the requested fusion        */
 } pp_status;
 
 typedef enum { PP_F32 = 0, PP_F16 = 1 } pp_dtype;
@@ -143,6 +144,19 @@ int pp_conv(pp_handle h, const void* x, int dtype, int N, int H, int W,
  * workspace. */
 int pp_conv_ws(pp_handle h, const void* x, int dtype, int N, int H, int W, const float* bias,
                int relu, void* y, void* workspace, size_t workspace_bytes, void* stream);
+
+/* pp_conv_ws followed by a 2x2 max-pool with stride 2, fused into the conv's epilogue: y is
+ * DEVICE [N][Cout][Ho/2][Wo/2] (floor: an odd last output row or column is dropped) and holds
+ * max over each 2x2 window of sigma(conv + bias).  The forward pass of a layer is sigma(WX + b)
+ * (§4.1); the pooling that follows VGG's blocks is the network's, not the paper's method, and is
+ * fused here so that the full-resolution map never reaches memory.  Each lane of the kernel owns
+ * a 4x4 output block whose origin is even, so every pooling window lies inside one lane.  With a
+ * workspace split the partial sums stay full-resolution in the workspace (same size as for
+ * pp_conv_ws) and the reduction pools.  Dense layers on the compiled pattern library only
+ * (pp_query PP_Q_FAST_PATH == 1); others return PP_ERR_PATH.  Ho and Wo must be at least 2
+ * (PP_ERR_SHAPE).  Otherwise the errors of pp_conv_ws. */
+int pp_conv_pool_ws(pp_handle h, const void* x, int dtype, int N, int H, int W, const float* bias,
+                    int relu, void* y, void* workspace, size_t workspace_bytes, void* stream);
 
 /* Workspace bytes pp_conv_ws would use for this call shape with unlimited workspace (0 when it
  * would not split).  Host-only. */

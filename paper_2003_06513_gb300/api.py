@@ -121,9 +121,9 @@ class Layer:
 
     def conv(self, x: torch.Tensor, bias: Optional[torch.Tensor] = None, relu: bool = False,
              out: Optional[torch.Tensor] = None, stream=None,
-             workspace: Optional[torch.Tensor] = None) -> torch.Tensor:
-        """y = ReLU?(conv3x3(x, W_hat, stride, pad 1) + bias) via pp_conv_ws (pp_conv when no
-        workspace tensor is given)."""
+             workspace: Optional[torch.Tensor] = None, pool2x2: bool = False) -> torch.Tensor:
+        """y = ReLU?(conv3x3(x, W_hat, stride, pad 1) + bias) via pp_conv_ws; with ``pool2x2``
+        the 2x2/2 max-pool of that map, fused into the conv (pp_conv_pool_ws)."""
         if self._dev_buf is None:
             self.bind(x.device)
         if not x.is_cuda or x.dtype not in _DT or not x.is_contiguous() or x.dim() != 4:
@@ -132,6 +132,8 @@ class Layer:
         if x.shape[1] != cin:
             raise ValueError(f"x has {x.shape[1]} channels, layer expects {cin}")
         shape = self.out_shape(tuple(x.shape))
+        if pool2x2:
+            shape = shape[:2] + (shape[2] // 2, shape[3] // 2)
         if out is None:
             out = torch.empty(shape, dtype=x.dtype, device=x.device)
         if tuple(out.shape) != shape or out.dtype != x.dtype or not out.is_contiguous() or not out.is_cuda:
@@ -148,7 +150,8 @@ class Layer:
             if not workspace.is_cuda or not workspace.is_contiguous():
                 raise ValueError("workspace must be a contiguous CUDA tensor")
             wptr, wbytes = ctypes.c_void_p(workspace.data_ptr()), workspace.numel() * workspace.element_size()
-        _lib.check("pp_conv_ws", _lib.load().pp_conv_ws(
+        name = "pp_conv_pool_ws" if pool2x2 else "pp_conv_ws"
+        _lib.check(name, getattr(_lib.load(), name)(
             self._h, ctypes.c_void_p(x.data_ptr()), _DT[x.dtype], N, H, W, bptr, int(bool(relu)),
             ctypes.c_void_p(out.data_ptr()), wptr, wbytes, _stream_ptr(stream, x.device)))
         return out

@@ -99,6 +99,7 @@ struct TmParams {
     size_t ws_stride;                  // elements per split
     int IH, BWb;                       // staged rows / row width (floats) per (image, channel)
     int use_tma, vec_store;
+    int pool, vec_pool;                // fused 2x2/2 max-pool of the output; pair stores of it
     unsigned tma_bytes;                // bytes one TMA box delivers
     unsigned kb_off, stage_off, stage_bytes, desc_off, vals_off;   // shared-memory layout
 };
@@ -390,6 +391,37 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
                 continue;
             }
             const float b = p.bias ? p.bias[co] : 0.0f;
+            if (p.pool) {   // 2x2/2 max-pool inside the lane's 4x4 block (block origins are even)
+                const int Hp = p.Ho >> 1, Wp = p.Wo >> 1;
+                const int py0 = oyb >> 1, px0 = oxb >> 1;
+                TOut* yc = y + ((size_t)n * p.Cout + co) * Hp * Wp;
+#pragma unroll
+                for (int r = 0; r < 2; ++r) {
+                    const int py = py0 + r;
+                    if (py >= Hp) break;
+                    float v[2];
+#pragma unroll
+                    for (int c = 0; c < 2; ++c) {
+                        const float m = fmaxf(fmaxf(a[2 * r * RX + 2 * c], a[2 * r * RX + 2 * c + 1]),
+                                              fmaxf(a[(2 * r + 1) * RX + 2 * c], a[(2 * r + 1) * RX + 2 * c + 1]));
+                        const float q = m + b;   // max(a) + b == max(a + b) in fp32: rounding is monotonic
+                        v[c] = p.relu ? fmaxf(q, 0.0f) : q;
+                    }
+                    TOut* yr = yc + (size_t)py * Wp + px0;
+                    if (p.vec_pool && px0 + 2 <= Wp) {
+                        if constexpr (sizeof(TOut) == 4) {
+                            *reinterpret_cast<float2*>(yr) = make_float2(v[0], v[1]);
+                        } else {
+                            *reinterpret_cast<__half2*>(yr) = __floats2half2_rn(v[0], v[1]);
+                        }
+                    } else {
+#pragma unroll
+                        for (int c = 0; c < 2; ++c)
+                            if (px0 + c < Wp) yr[c] = from_f32<TOut>(v[c]);
+                    }
+                }
+                continue;
+            }
             TOut* yc = y + ((size_t)n * p.Cout + co) * p.Ho * p.Wo;
 #pragma unroll
             for (int r = 0; r < RY; ++r) {
@@ -1114,6 +1146,33 @@ __global__ void splitk_reduce(const float* __restrict__ ws, T* __restrict__ y, c
     }
 }
 
+// Split-K reduction with the fused 2x2/2 max-pool: each pooled output sums the KS partial planes
+// at its four positions (split order), takes the maximum, adds the bias and applies ReLU.
+template <typename T>
+__global__ void splitk_reduce_pool(const float* __restrict__ ws, T* __restrict__ y, const float* __restrict__ bias,
+                                   int KS, size_t stride, int Cout, int Ho, int Wo, int relu) {
+    const int Hp = Ho >> 1, Wp = Wo >> 1;
+    const size_t total = stride / ((size_t)Ho * Wo) * Hp * Wp;
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total; i += (size_t)gridDim.x * blockDim.x) {
+        const int px = (int)(i % Wp);
+        const size_t r = i / Wp;
+        const int py = (int)(r % Hp);
+        const size_t plane = r / Hp;                       // n * Cout + co
+        const size_t base = (plane * Ho + 2 * py) * Wo + 2 * px;
+        float q[4];
+        const size_t off[4] = {0, 1, (size_t)Wo, (size_t)Wo + 1};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            float a = ws[base + off[j]];
+            for (int k = 1; k < KS; ++k) a += ws[(size_t)k * stride + base + off[j]];
+            q[j] = a;
+        }
+        const int co = (int)(plane % (size_t)Cout);
+        float a = fmaxf(fmaxf(q[0], q[1]), fmaxf(q[2], q[3])) + (bias ? bias[co] : 0.0f);
+        y[i] = from_f32<T>(relu ? fmaxf(a, 0.0f) : a);
+    }
+}
+
 // Raise the kernel's dynamic shared-memory limit to the device's opt-in maximum once per device
 // (a launch needs at most that), so that later calls, including ones under stream capture, make
 // no attribute call.
@@ -1134,7 +1193,7 @@ bool allow_max_smem(size_t need) {
 
 template <int S, typename T>
 int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int relu, int N, int H, int W, int Ho,
-              int Wo, void* ws, size_t ws_bytes, cudaStream_t st) {
+              int Wo, void* ws, size_t ws_bytes, cudaStream_t st, int pool = 0) {
     Plan pl;
     const int rc = make_plan(L, N, H, W, ws ? ws_bytes : 0, &pl);
     if (rc != PP_OK) return rc;
@@ -1186,6 +1245,8 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
     p.desc_off = (unsigned)align_up((size_t)p.NB * p.CK * p.IH * p.BWb * 4, 128);
     p.vals_off = p.desc_off + (unsigned)align_up((size_t)p.WG * p.CK * 8, 16);
     p.vec_store = (Wo % 4 == 0) && (reinterpret_cast<uintptr_t>(y) % (4 * es)) == 0;
+    p.pool = pool;
+    p.vec_pool = ((Wo >> 1) % 2 == 0) && (reinterpret_cast<uintptr_t>(y) % (2 * es)) == 0;
 
     CUtensorMap tmap;
     std::memset(&tmap, 0, sizeof(tmap));
@@ -1210,7 +1271,12 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
     if (pl.KS > 1) {
         const size_t total = p.ws_stride;
         const int blocks = (int)std::max<size_t>(1, std::min<size_t>((total + 255) / 256, (size_t)sm_count() * 16));
-        splitk_reduce<T><<<blocks, 256, 0, st>>>(p.ws, static_cast<T*>(y), bias, pl.KS, total, L->cout, Ho * Wo, relu);
+        if (pool)
+            splitk_reduce_pool<T><<<blocks, 256, 0, st>>>(p.ws, static_cast<T*>(y), bias, pl.KS, total, L->cout, Ho, Wo,
+                                                          relu);
+        else
+            splitk_reduce<T><<<blocks, 256, 0, st>>>(p.ws, static_cast<T*>(y), bias, pl.KS, total, L->cout, Ho * Wo,
+                                                     relu);
         if (cudaGetLastError() != cudaSuccess) return PP_ERR_CUDA;
     }
     return PP_OK;
@@ -1433,7 +1499,7 @@ int pp_bind_device(pp_handle h, void* dev_image, size_t bytes, void* stream) {
 namespace {
 
 int validate_conv(pp_handle h, const void* x, int dtype, int N, int H, int W, const float* bias, int relu,
-                  const void* y) {
+                  const void* y, int pool = 0) {
     if (!h) return PP_ERR_NULL;
     if (!h->dev) return PP_ERR_NOT_BOUND;
     if (dtype != PP_F32 && dtype != PP_F16) return PP_ERR_DTYPE;
@@ -1445,7 +1511,8 @@ int validate_conv(pp_handle h, const void* x, int dtype, int N, int H, int W, co
     const int Ho = (H - 1) / h->stride + 1, Wo = (W - 1) / h->stride + 1;
     const size_t es = dtype == PP_F32 ? 4 : 2;
     if ((size_t)N * C * H * W >= (1ull << 40) || (size_t)N * h->cout * Ho * Wo >= (1ull << 40)) return PP_ERR_SHAPE;
-    const size_t xb = (size_t)N * C * H * W * es, yb = (size_t)N * h->cout * Ho * Wo * es;
+    const size_t xb = (size_t)N * C * H * W * es;
+    const size_t yb = pool ? (size_t)N * h->cout * (Ho / 2) * (Wo / 2) * es : (size_t)N * h->cout * Ho * Wo * es;
     if (reinterpret_cast<uintptr_t>(x) % es || reinterpret_cast<uintptr_t>(y) % es) return PP_ERR_ALIGN;
     if (bias && reinterpret_cast<uintptr_t>(bias) % 4) return PP_ERR_ALIGN;
     if (overlaps(x, xb, y, yb)) return PP_ERR_BUFFER;
@@ -1486,6 +1553,28 @@ int pp_conv_ws(pp_handle h, const void* x, int dtype, int N, int H, int W, const
 int pp_conv(pp_handle h, const void* x, int dtype, int N, int H, int W, const float* bias, int relu, void* y,
             void* stream) {
     return pp_conv_ws(h, x, dtype, N, H, W, bias, relu, y, nullptr, 0, stream);
+}
+
+int pp_conv_pool_ws(pp_handle h, const void* x, int dtype, int N, int H, int W, const float* bias, int relu,
+                    void* y, void* workspace, size_t workspace_bytes, void* stream) {
+    if (h && (h->depthwise || !h->fast)) return PP_ERR_PATH;
+    const int v = validate_conv(h, x, dtype, N, H, W, bias, relu, y, 1);
+    if (v != PP_OK || N == 0) return v;
+    const int Ho = (H - 1) / h->stride + 1, Wo = (W - 1) / h->stride + 1;
+    if (Ho < 2 || Wo < 2) return PP_ERR_SHAPE;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const bool f16 = dtype == PP_F16;
+    if (workspace) {
+        const size_t es = f16 ? 2 : 4;
+        if (overlaps(workspace, workspace_bytes, x, (size_t)N * h->cin_g * H * W * es) ||
+            overlaps(workspace, workspace_bytes, y, (size_t)N * h->cout * (Ho / 2) * (Wo / 2) * es))
+            return PP_ERR_BUFFER;
+    }
+    if (h->stride == 1)
+        return f16 ? launch_tm<1, __half>(h, x, y, bias, relu, N, H, W, Ho, Wo, workspace, workspace_bytes, st, 1)
+                   : launch_tm<1, float>(h, x, y, bias, relu, N, H, W, Ho, Wo, workspace, workspace_bytes, st, 1);
+    return f16 ? launch_tm<2, __half>(h, x, y, bias, relu, N, H, W, Ho, Wo, workspace, workspace_bytes, st, 1)
+               : launch_tm<2, float>(h, x, y, bias, relu, N, H, W, Ho, Wo, workspace, workspace_bytes, st, 1);
 }
 
 int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info) {

@@ -310,6 +310,7 @@ const char* pp_status_string(int status) {
         case PP_ERR_ARG: return "invalid argument";
         case PP_ERR_ALLOC: return "host allocation failed";
         case PP_ERR_SCRATCH: return "call needs more scratch than the library's static scratch array holds";
+        case PP_ERR_PATH: return "the layer's kernel does not offer this fusion (dense layers of the compiled pattern library only)";
         default: return "unknown status";
     }
 }

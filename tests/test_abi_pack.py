@@ -12,6 +12,7 @@ from conftest import ROOT
 from oracle import layout as OL
 from oracle import patterns as OP
 from oracle import project as OPR
+from paper_2003_06513_gb300 import api
 from paper_2003_06513_gb300 import workloads as WL
 
 PP_ERR = {"NULL": -1, "SHAPE": -2, "PATTERN": -3, "KEEP": -4, "NONFINITE": -5, "ALIGN": -6,
@@ -174,3 +175,16 @@ def test_pack_counts_and_compression():
         dense = layer.export("dense")
         assert np.count_nonzero(dense) == 4 * layer.beta
         assert 9 * 64 * 64 / np.count_nonzero(dense) == rate
+
+
+def test_conv_pool_rejections_without_gpu(lib):
+    """pp_conv_pool_ws refuses layers whose kernel has no fused pooling (depthwise, other
+    libraries) and unbound handles, before touching the GPU."""
+    rng = np.random.default_rng(3)
+    Wd = rng.standard_normal((8, 1, 3, 3)).astype(np.float32)
+    dw = api.pp_pack(Wd, None, 1.0, 8, 1)
+    assert lib.pp_conv_pool_ws(dw._h, None, 0, 1, 8, 8, None, 1, None, None, 0, None) == -14
+    assert b"fusion" in lib.pp_status_string(-14)
+    Wt = rng.standard_normal((8, 4, 3, 3)).astype(np.float32)
+    dense = api.pp_pack(Wt, None, 0.5)
+    assert lib.pp_conv_pool_ws(dense._h, None, 0, 1, 8, 8, None, 1, None, None, 0, None) == -8   # not bound

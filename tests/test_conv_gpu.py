@@ -250,6 +250,85 @@ def test_vgg16_chained_network():
         x = y
 
 
+# --------------------------------------------------------------------------- fused max-pool
+
+def _pool_ref(W, x, b, keep, stride, relu):
+    """Oracle conv, then the oracle's 2x2/2 max-pool; the denominator of a pooled output is the
+    largest denominator in its window (max is 1-Lipschitz in the max norm)."""
+    ref, den = oracle(W, x, b, keep, stride, relu)
+    return OC.maxpool2x2(ref), OC.maxpool2x2(den)
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.float16])
+@pytest.mark.parametrize("N,Cin,Cout,H,W,stride,relu", [(2, 16, 24, 16, 16, 1, True),
+                                                        (1, 8, 13, 15, 13, 1, True),     # odd: floor
+                                                        (2, 8, 16, 17, 18, 2, False),
+                                                        (3, 5, 9, 6, 34, 1, False)])
+def test_conv_pool_fused(dtype, N, Cin, Cout, H, W, stride, relu):
+    rng = np.random.default_rng(Cin * 11 + H)
+    Wt = (rng.standard_normal((Cout, Cin, 3, 3)) * np.sqrt(2 / (9 * Cin))).astype(np.float32)
+    x = rnd((N, Cin, H, W), H * 3 + W, dtype=_np_dt(dtype))
+    b = (rng.standard_normal(Cout) * 0.1).astype(np.float32)
+    layer = api.pp_pack(Wt, None, 0.5, 1, stride).bind("cuda")
+    y = layer.conv(torch.from_numpy(x).cuda(), torch.from_numpy(b).cuda(), relu, pool2x2=True)
+    ref, den = _pool_ref(Wt, x, b, 0.5, stride, relu)
+    assert tuple(y.shape) == ref.shape
+    assert OC.max_norm_err(y.double().cpu().numpy(), ref, den) <= TOL[dtype]
+
+
+def test_conv_pool_fused_with_split_equals_unfused_pool():
+    """Small images with a workspace: the split path pools in its reduction; the result equals
+    pp_conv_ws followed by the library's max-pool bit for bit (same sums, same order)."""
+    L = WL.vgg16()[12]                                     # 512 -> 512 at 14x14, pooled
+    W, b = WL.weights(L), WL.bias(L)
+    x = torch.from_numpy(WL.layer_input(L, 16)).cuda()
+    bt = torch.from_numpy(b).cuda()
+    layer = api.pp_pack(W, None, L.keep).bind("cuda")
+    nb = layer.workspace_bytes(x.shape)
+    assert nb > 0 and layer.plan(x.shape, nb)["splits"] > 1
+    ws = torch.full((nb // 4,), float("nan"), device="cuda")
+    fused = layer.conv(x, bt, True, workspace=ws, pool2x2=True)
+    plain = api.pp_maxpool2x2(layer.conv(x, bt, True, workspace=ws))
+    assert torch.equal(fused, plain)
+    ref, den = _pool_ref(W, x[:2].cpu().numpy(), b, L.keep, 1, True)
+    assert OC.max_norm_err(fused[:2].double().cpu().numpy(), ref, den) <= 1e-4
+
+
+@pytest.mark.parametrize("idx", [i for i, L in enumerate(WL.vgg16()) if L.pool_after])
+def test_vgg16_pool_layer_fused_batch32(idx):
+    """The benchmark's launch configuration of each VGG-16 block end: batch 32, workspace,
+    fused pooling; oracle on two sampled images."""
+    L = WL.vgg16()[idx]
+    x = WL.layer_input(L, 32)
+    W, b = WL.weights(L), WL.bias(L)
+    layer = api.pp_pack(W, None, L.keep).bind("cuda")
+    xt = torch.from_numpy(x).cuda()
+    nb = layer.workspace_bytes(xt.shape)
+    ws = torch.empty(max(nb // 4, 1), device="cuda") if nb else None
+    y = layer.conv(xt, torch.from_numpy(b).cuda(), True, workspace=ws, pool2x2=True)
+    ref, den = _pool_ref(W, x[[0, 31]], b, L.keep, 1, True)
+    assert OC.max_norm_err(y[[0, 31]].double().cpu().numpy(), ref, den) <= 1e-4
+
+
+def test_vgg16_chained_network_fused_pool():
+    """The 13-layer stack with the pooling fused into each block's last conv, batch 2."""
+    x = torch.from_numpy(WL.vgg16_image(2)).cuda()
+    for L in WL.vgg16():
+        W, b = WL.weights(L), WL.bias(L)
+        layer = api.pp_pack(W, None, L.keep).bind("cuda")
+        y = layer.conv(x, torch.from_numpy(b).cuda(), True, pool2x2=L.pool_after)
+        torch.cuda.synchronize()
+        xin = x.cpu().numpy()
+        if L.pool_after:
+            ref, den = _pool_ref(W, xin, b, L.keep, 1, True)
+        else:
+            ref, den = oracle(W, xin, b, L.keep)
+        err = OC.max_norm_err(y.double().cpu().numpy(), ref, den)
+        assert err <= 1e-4, f"{L.name}: {err:.3e}"
+        x = y
+    assert tuple(x.shape) == (2, 512, 7, 7)
+
+
 # --------------------------------------------------------------------------- channel split
 
 def _split_case():
