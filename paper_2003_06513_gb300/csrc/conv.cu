@@ -26,7 +26,10 @@
 #include <climits>
 #include <cstdint>
 #include <cstring>
+#include <map>
 #include <mutex>
+#include <tuple>
+#include <vector>
 
 #include "../../include/patconv.h"
 #include "layer.h"
@@ -93,6 +96,7 @@ struct TmParams {
     int WG, WS;                        // filter groups x spatial warps per CTA (WG * WS = 16)
     int BY, BX, NB;                    // spatial tile: BY x BX blocks (4x4 outputs) of NB images
     int tiles_x, tiles_y, tiles_n, n_fchunks;
+    int linear;                        // linear tiles: lanes take consecutive blocks across images
     int CK, n_chunks, maxk;            // channels per stage, stages per CTA (max), max kept per group-stage
     int KS, c_split;                   // input-channel splits; channels per split (multiple of CK)
     float* ws;                         // KS > 1: fp32 partial sums [KS][N][Cout][Ho][Wo]
@@ -275,7 +279,10 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     const int ks = t / p.tiles_n;                         // input-channel split of this CTA
     const int c_lo = ks * p.c_split, c_hi = min(p.C, c_lo + p.c_split);
     const int nck = (c_hi - c_lo + p.CK - 1) / p.CK;       // channel chunks of this CTA
-    const int n0 = tn * p.NB;
+    // linear tiles: tile tn holds blocks [tn * lanes, (tn + 1) * lanes) of the (image, block row,
+    // block column) sequence and stages the whole images from n0 on
+    const int lanes_t = 32 * p.WS, bpi = p.BY * p.BX;
+    const int n0 = p.linear ? (int)(((long long)tn * lanes_t) / bpi) : tn * p.NB;
     const int oy0 = ty * p.BY * RY, ox0 = tx * p.BX * RX;
     const int iy0 = oy0 * S - 1, ix0 = ox0 * S - 4;     // stage origin: 1 halo row, 16-B aligned col
     const int g0 = fchunk * p.WG;
@@ -322,11 +329,20 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     for (int f = 0; f < kF; ++f) tmem_zero16(tw + 16u * f);
 
     const int blk = ws * 32 + lane;
-    const int per_img = p.BY * p.BX;
-    const int img = blk / per_img;
-    const int rem = blk - img * per_img;
+    int img, rem;
+    bool active;
+    if (p.linear) {
+        const long long b = (long long)tn * lanes_t + blk;
+        const int ng = (int)(b / bpi);
+        img = ng - n0;
+        rem = (int)(b - (long long)ng * bpi);
+        active = ng < p.N && img < p.NB;
+    } else {
+        img = blk / bpi;
+        rem = blk - img * bpi;
+        active = img < p.NB;
+    }
     const int by = rem / p.BX, bx = rem - (rem / p.BX) * p.BX;
-    const bool active = img < p.NB;
     const int plane = p.IH * p.BWb;
     const int in_off = active ? img * p.CK * plane + by * RY * S * p.BWb + bx * RX * S + 3 : 3;
 
@@ -1006,41 +1022,8 @@ unsigned* status_word() {
 
 struct TileChoice {
     int BY = 1, BX = 1, NB = 1, IH = 0, BWb = 0;
+    int linear = 0;   // lanes take consecutive blocks of the (image, row, column) sequence
 };
-
-// Spatial tile of at most 32*WS blocks (4x4 outputs each) minimising CTA waves, then the lanes
-// left idle; stride-1 rows need 4*BX + 5 staged columns, stride-2 rows 8*BX + 4, rounded to a
-// 16-byte multiple and padded to 4 (mod 8) floats so that rows four apart fall in other banks.
-TileChoice choose_tile(int N, int Ho, int Wo, int S, int lanes, int n_fchunks, int C) {
-    const int nby = (Ho + 3) / 4, nbx = (Wo + 3) / 4;
-    const long long sms = sm_count();
-    TileChoice best;
-    long long best_waves = LLONG_MAX, best_cover = LLONG_MAX;
-    for (int bx = 1; bx <= std::min(nbx, lanes); ++bx) {
-        for (int by = 1; by <= std::min(nby, lanes / bx); ++by) {
-            // several images per tile only when each image contributes a whole image's blocks
-            // (lanes then step through one image before the next: no bank-aligned image stride)
-            const bool whole = by == nby && bx == nbx;
-            const int nb = whole ? std::max(1, std::min(std::min(N, 256), lanes / (bx * by))) : 1;
-            const int ih = S == 1 ? 4 * by + 2 : 8 * by + 1;
-            int bw = S == 1 ? 4 * bx + 8 : 8 * bx + 4;
-            if (bw % 8 == 0) bw += 4;
-            if (bw > 256 || ih > 256) continue;
-            const int ck_min = (C + kMaxChunks - 1) / kMaxChunks;
-            if ((long long)nb * ih * bw * 4 * ck_min > 48 * 1024) continue;   // enough channels per stage
-            const long long tiles = (long long)((N + nb - 1) / nb) * ((nby + by - 1) / by) * ((nbx + bx - 1) / bx);
-            const long long waves = (tiles * n_fchunks + sms - 1) / sms;
-            const long long cover = tiles * lanes;
-            if (waves < best_waves || (waves == best_waves && (cover < best_cover ||
-                                                               (cover == best_cover && bx > best.BX)))) {
-                best = TileChoice{by, bx, nb, ih, bw};
-                best_waves = waves;
-                best_cover = cover;
-            }
-        }
-    }
-    return best;
-}
 
 size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
@@ -1056,7 +1039,47 @@ struct Plan {
     size_t ws_bytes = 0;          // workspace the chosen split needs (0 without a split)
 };
 
-int make_plan(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out) {
+struct PlanCache : PlanCacheBase {
+    std::mutex mu;
+    std::map<std::tuple<int, int, int, size_t>, Plan> plans;
+};
+
+// Candidate spatial tiles of at most 32*WS blocks (4x4 outputs each).
+//   rectangles: BY x BX blocks of one image (several whole images when the rectangle is the
+//     whole image); stride-1 rows need 4*BX + 5 staged columns, stride-2 rows 8*BX + 4, rounded
+//     to a 16-byte multiple and padded to 4 (mod 8) floats so that rows four apart fall in other
+//     banks;
+//   linear: 32*WS consecutive blocks of the (image, block row, block column) sequence, staged as
+//     the whole images they touch; no lane idles even when an image's block count is no divisor
+//     of the lane count (28 x 28 outputs: 49 blocks).
+std::vector<TileChoice> tile_candidates(int N, int Ho, int Wo, int S, int lanes) {
+    const int nby = (Ho + 3) / 4, nbx = (Wo + 3) / 4;
+    auto bw_of = [&](int bx) {
+        int bw = S == 1 ? 4 * bx + 8 : 8 * bx + 4;
+        if (bw % 8 == 0) bw += 4;
+        return bw;
+    };
+    auto ih_of = [&](int by) { return S == 1 ? 4 * by + 2 : 8 * by + 1; };
+    std::vector<TileChoice> out;
+    for (int bx = 1; bx <= std::min(nbx, lanes); ++bx) {
+        for (int by = 1; by <= std::min(nby, lanes / bx); ++by) {
+            const bool whole = by == nby && bx == nbx;
+            const int nb = whole ? std::max(1, std::min(std::min(N, 256), lanes / (bx * by))) : 1;
+            const int ih = ih_of(by), bw = bw_of(bx);
+            if (bw > 256 || ih > 256) continue;
+            out.push_back(TileChoice{by, bx, nb, ih, bw, 0});
+        }
+    }
+    const long long bpi = (long long)nby * nbx;
+    if (bpi < lanes && lanes % bpi == 0) return out;    // the whole-image rectangle is this tile
+    const int nb = (int)std::min<long long>(N, (lanes - 1) / bpi + 2);
+    const int ih = ih_of(nby), bw = bw_of(nbx);
+    if (N > 1 && bpi < 4LL * lanes && ih <= 256 && bw <= 256 && nb <= 256)
+        out.push_back(TileChoice{nby, nbx, nb, ih, bw, 1});
+    return out;
+}
+
+int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out) {
     Plan pl;
     const int S = L->stride;
     const int Ho = (H - 1) / S + 1, Wo = (W - 1) / S + 1;
@@ -1066,11 +1089,42 @@ int make_plan(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out
     pl.WS = kCompute / wg;
     pl.n_fchunks = (L->G + wg - 1) / wg;
     const int C = L->cin_g;
-    pl.tile = choose_tile(N, Ho, Wo, S, 32 * pl.WS, pl.n_fchunks, C);
-    if (pl.tile.IH == 0) return PP_ERR_SHAPE;
-    pl.tiles_x = ((Wo + 3) / 4 + pl.tile.BX - 1) / pl.tile.BX;
-    pl.tiles_y = ((Ho + 3) / 4 + pl.tile.BY - 1) / pl.tile.BY;
-    pl.tiles_n = (N + pl.tile.NB - 1) / pl.tile.NB;
+    const int lanes = 32 * pl.WS;
+    const int nby = (Ho + 3) / 4, nbx = (Wo + 3) / 4;
+    const long long sms = sm_count();
+
+    // spatial tile: fewest CTA waves, then fewest lanes covered (idle lanes), then the widest
+    // rows; a tile must leave room for at least the channels per stage that kMaxChunks needs
+    const int ck_min = (C + kMaxChunks - 1) / kMaxChunks;
+    long long best_waves = LLONG_MAX, best_cover = LLONG_MAX;
+    bool found = false;
+    for (const TileChoice& t : tile_candidates(N, Ho, Wo, S, lanes)) {
+        if ((long long)t.NB * t.IH * t.BWb * 4 * ck_min > 48 * 1024) continue;
+        long long tiles;
+        int tx = 1, ty = 1, tn;
+        if (t.linear) {
+            tn = (int)(((long long)N * nby * nbx + lanes - 1) / lanes);
+            tiles = tn;
+        } else {
+            tx = (nbx + t.BX - 1) / t.BX;
+            ty = (nby + t.BY - 1) / t.BY;
+            tn = (N + t.NB - 1) / t.NB;
+            tiles = (long long)tn * ty * tx;
+        }
+        const long long waves = (tiles * pl.n_fchunks + sms - 1) / sms;
+        const long long cover = tiles * lanes;
+        if (waves < best_waves ||
+            (waves == best_waves && (cover < best_cover || (cover == best_cover && t.BX > pl.tile.BX)))) {
+            pl.tile = t;
+            pl.tiles_x = tx;
+            pl.tiles_y = ty;
+            pl.tiles_n = tn;
+            best_waves = waves;
+            best_cover = cover;
+            found = true;
+        }
+    }
+    if (!found) return PP_ERR_SHAPE;
     pl.ctas = (long long)pl.tiles_n * pl.tiles_y * pl.tiles_x * pl.n_fchunks;
 
     // channels per stage: the largest that fits three stages in shared memory
@@ -1108,7 +1162,6 @@ int make_plan(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out
     // into KS parts (whole chunks each) if the caller's workspace holds the partial sums.
     // Cost in channel-stage units: waves x (chunks per split + start-up) + a reduction term.
     const size_t out_elems = (size_t)N * L->cout * Ho * Wo;
-    const long long sms = sm_count();
     int best_ks = 1;
     double best_cost = 1e300;
     for (int ksp = 1; ksp <= std::min(8, nck_total); ++ksp) {
@@ -1128,6 +1181,33 @@ int make_plan(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out
     pl.c_split = per * ck;
     pl.n_chunks = std::min(per, nck_total);
     pl.ws_bytes = best_ks > 1 ? (size_t)best_ks * out_elems * 4 : 0;
+    *out = pl;
+    return PP_OK;
+}
+
+int make_plan(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out) {
+    auto* cache = static_cast<PlanCache*>(L->plans.get());
+    if (!cache) {
+        static std::mutex create_mu;
+        std::lock_guard<std::mutex> g(create_mu);
+        if (!L->plans) const_cast<pp_layer*>(L)->plans.reset(new PlanCache);
+        cache = static_cast<PlanCache*>(L->plans.get());
+    }
+    const auto key = std::make_tuple(N, H, W, ws_avail);
+    {
+        std::lock_guard<std::mutex> g(cache->mu);
+        auto it = cache->plans.find(key);
+        if (it != cache->plans.end()) {
+            *out = it->second;
+            return PP_OK;
+        }
+    }
+    Plan pl;
+    const int rc = make_plan_uncached(L, N, H, W, ws_avail, &pl);
+    if (rc != PP_OK) return rc;
+    std::lock_guard<std::mutex> g(cache->mu);
+    if (cache->plans.size() >= 256) cache->plans.clear();
+    cache->plans[key] = pl;
     *out = pl;
     return PP_OK;
 }
@@ -1226,6 +1306,7 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
     p.NB = pl.tile.NB;
     p.IH = pl.tile.IH;
     p.BWb = pl.tile.BWb;
+    p.linear = pl.tile.linear;
     p.tiles_x = pl.tiles_x;
     p.tiles_y = pl.tiles_y;
     p.tiles_n = pl.tiles_n;

@@ -4,6 +4,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <memory>
 #include <vector>
 
 namespace patconv {
@@ -21,6 +22,11 @@ constexpr uint16_t kDefaultMasks[kMaxPatterns] = {0x0B8, 0x0B2, 0x09A, 0x03A,
                                                   0x017, 0x059, 0x134, 0x1D0};
 
 inline size_t align256(size_t n) { return (n + 255) / 256 * 256; }
+
+// Launch plans the CUDA side caches per handle (defined in conv.cu; destroyed with the handle).
+struct PlanCacheBase {
+    virtual ~PlanCacheBase() = default;
+};
 
 }  // namespace patconv
 
@@ -42,4 +48,6 @@ struct pp_layer {
 
     void* dev = nullptr;               // caller-owned device copy of `image`
     size_t dev_bytes = 0;
+
+    std::unique_ptr<patconv::PlanCacheBase> plans;   // launch plans by call shape (conv.cu)
 };
