@@ -1080,54 +1080,17 @@ std::vector<TileChoice> tile_candidates(int N, int Ho, int Wo, int S, int lanes)
 }
 
 int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out) {
-    Plan pl;
     const int S = L->stride;
     const int Ho = (H - 1) / S + 1, Wo = (W - 1) / S + 1;
     int wg = 1;
     while (wg < L->G && wg < kCompute) wg *= 2;
-    pl.WG = wg;
-    pl.WS = kCompute / wg;
-    pl.n_fchunks = (L->G + wg - 1) / wg;
+    const int WS = kCompute / wg, lanes = 32 * WS;
+    const int n_fchunks = (L->G + wg - 1) / wg;
     const int C = L->cin_g;
-    const int lanes = 32 * pl.WS;
     const int nby = (Ho + 3) / 4, nbx = (Wo + 3) / 4;
     const long long sms = sm_count();
+    const size_t out_elems = (size_t)N * L->cout * Ho * Wo;
 
-    // spatial tile: fewest CTA waves, then fewest lanes covered (idle lanes), then the widest
-    // rows; a tile must leave room for at least the channels per stage that kMaxChunks needs
-    const int ck_min = (C + kMaxChunks - 1) / kMaxChunks;
-    long long best_waves = LLONG_MAX, best_cover = LLONG_MAX;
-    bool found = false;
-    for (const TileChoice& t : tile_candidates(N, Ho, Wo, S, lanes)) {
-        if ((long long)t.NB * t.IH * t.BWb * 4 * ck_min > 48 * 1024) continue;
-        long long tiles;
-        int tx = 1, ty = 1, tn;
-        if (t.linear) {
-            tn = (int)(((long long)N * nby * nbx + lanes - 1) / lanes);
-            tiles = tn;
-        } else {
-            tx = (nbx + t.BX - 1) / t.BX;
-            ty = (nby + t.BY - 1) / t.BY;
-            tn = (N + t.NB - 1) / t.NB;
-            tiles = (long long)tn * ty * tx;
-        }
-        const long long waves = (tiles * pl.n_fchunks + sms - 1) / sms;
-        const long long cover = tiles * lanes;
-        if (waves < best_waves ||
-            (waves == best_waves && (cover < best_cover || (cover == best_cover && t.BX > pl.tile.BX)))) {
-            pl.tile = t;
-            pl.tiles_x = tx;
-            pl.tiles_y = ty;
-            pl.tiles_n = tn;
-            best_waves = waves;
-            best_cover = cover;
-            found = true;
-        }
-    }
-    if (!found) return PP_ERR_SHAPE;
-    pl.ctas = (long long)pl.tiles_n * pl.tiles_y * pl.tiles_x * pl.n_fchunks;
-
-    // channels per stage: the largest that fits three stages in shared memory
     auto maxk_for = [&](int ck) {
         uint32_t m = 0;
         for (int g = 0; g < L->G; ++g)
@@ -1137,51 +1100,97 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
             }
         return (int)m;
     };
-    auto layout = [&](int ck, int maxk, size_t* stage_bytes, size_t* kb_bytes) {
-        const size_t in_b = align_up((size_t)pl.tile.NB * ck * pl.tile.IH * pl.tile.BWb * 4, 128);
-        const size_t desc_b = align_up((size_t)pl.WG * ck * 8, 16);
-        const size_t vals_b = (size_t)pl.WG * std::max(maxk, 1) * 16;
-        *stage_bytes = align_up(in_b + desc_b + vals_b, 128);
-        const int nch = (C + ck - 1) / ck;
-        *kb_bytes = (size_t)pl.WG * (nch + 1) * 4;
-        return align_up(64 + *kb_bytes, 128) + kStages * *stage_bytes;
+    // channels per stage (the largest that fits three stages in shared memory) and input-channel
+    // split of one tile; returns the estimated time in channel steps (infinite if it cannot run).
+    // The split is chosen in chunk units: waves x (chunks per split + start-up) + a reduction term.
+    auto finish = [&](const TileChoice& t, int tx, int ty, int tn, Plan* pl) -> double {
+        pl->WG = wg;
+        pl->WS = WS;
+        pl->n_fchunks = n_fchunks;
+        pl->tile = t;
+        pl->tiles_x = tx;
+        pl->tiles_y = ty;
+        pl->tiles_n = tn;
+        pl->ctas = (long long)tn * ty * tx * n_fchunks;
+        auto layout = [&](int ck, int maxk, size_t* stage_bytes, size_t* kb_bytes) {
+            const size_t in_b = align_up((size_t)t.NB * ck * t.IH * t.BWb * 4, 128);
+            const size_t desc_b = align_up((size_t)wg * ck * 8, 16);
+            const size_t vals_b = (size_t)wg * std::max(maxk, 1) * 16;
+            *stage_bytes = align_up(in_b + desc_b + vals_b, 128);
+            const int nch = (C + ck - 1) / ck;
+            *kb_bytes = (size_t)wg * (nch + 1) * 4;
+            return align_up(64 + *kb_bytes, 128) + kStages * *stage_bytes;
+        };
+        int ck = std::min(C, 64);
+        for (;; --ck) {
+            if (ck < 1 || (C + ck - 1) / ck > kMaxChunks) return 1e300;
+            pl->maxk = maxk_for(ck);
+            pl->smem = layout(ck, pl->maxk, &pl->stage_bytes, &pl->kb_bytes);
+            if (pl->smem <= 200 * 1024) break;
+        }
+        pl->CK = ck;
+        pl->maxk = std::max(pl->maxk, 1);
+        const int nck_total = (C + ck - 1) / ck;
+        int best_ks = 1;
+        double best_cost = 1e300;
+        for (int ksp = 1; ksp <= std::min(8, nck_total); ++ksp) {
+            const int per = (nck_total + ksp - 1) / ksp;
+            const int used = (nck_total + per - 1) / per;
+            if (used != ksp) continue;                       // every split must get chunks
+            if (ksp > 1 && ws_avail < (size_t)ksp * out_elems * 4) break;
+            const long long waves = (pl->ctas * ksp + sms - 1) / sms;
+            const double cost = (double)waves * (per + 2.0) + (ksp > 1 ? 0.5 * ksp : 0.0);
+            if (cost < best_cost - 1e-9) {
+                best_cost = cost;
+                best_ks = ksp;
+            }
+        }
+        pl->KS = best_ks;
+        const int per = (nck_total + best_ks - 1) / best_ks;
+        pl->c_split = per * ck;
+        pl->n_chunks = std::min(per, nck_total);
+        pl->ws_bytes = best_ks > 1 ? (size_t)best_ks * out_elems * 4 : 0;
+        const long long waves = (pl->ctas * best_ks + sms - 1) / sms;
+        return (double)waves * (std::min(pl->c_split, C) + 2.0 * per + 2.0 * ck);
     };
-    int ck = std::min(C, 64);
-    for (;; --ck) {
-        if (ck < 1) return PP_ERR_SHAPE;
-        if ((C + ck - 1) / ck > kMaxChunks) return PP_ERR_SHAPE;
-        pl.maxk = maxk_for(ck);
-        pl.smem = layout(ck, pl.maxk, &pl.stage_bytes, &pl.kb_bytes);
-        if (pl.smem <= 200 * 1024) break;
-    }
-    pl.CK = ck;
-    pl.maxk = std::max(pl.maxk, 1);
-    const int nck_total = (C + ck - 1) / ck;
 
-    // input-channel split: when one split gives too few CTAs for the SMs, cut the channel range
-    // into KS parts (whole chunks each) if the caller's workspace holds the partial sums.
-    // Cost in channel-stage units: waves x (chunks per split + start-up) + a reduction term.
-    const size_t out_elems = (size_t)N * L->cout * Ho * Wo;
-    int best_ks = 1;
-    double best_cost = 1e300;
-    for (int ksp = 1; ksp <= std::min(8, nck_total); ++ksp) {
-        const int per = (nck_total + ksp - 1) / ksp;
-        const int used = (nck_total + per - 1) / per;
-        if (used != ksp) continue;                       // every split must get chunks
-        if (ksp > 1 && ws_avail < (size_t)ksp * out_elems * 4) break;
-        const long long waves = (pl.ctas * ksp + sms - 1) / sms;
-        const double cost = (double)waves * (per + 2.0) + (ksp > 1 ? 0.5 * ksp : 0.0);
-        if (cost < best_cost - 1e-9) {
-            best_cost = cost;
-            best_ks = ksp;
+    // rectangles: fewest CTA waves, then fewest lanes covered (idle lanes), then the widest rows;
+    // a tile must leave room for at least the channels per stage that kMaxChunks needs
+    const int ck_min = (C + kMaxChunks - 1) / kMaxChunks;
+    long long best_waves = LLONG_MAX, best_cover = LLONG_MAX;
+    TileChoice rect, lin;
+    int rtx = 0, rty = 0, rtn = 0;
+    bool have_rect = false, have_lin = false;
+    for (const TileChoice& t : tile_candidates(N, Ho, Wo, S, lanes)) {
+        if ((long long)t.NB * t.IH * t.BWb * 4 * ck_min > 48 * 1024) continue;
+        if (t.linear) {
+            lin = t;
+            have_lin = true;
+            continue;
+        }
+        const int tx = (nbx + t.BX - 1) / t.BX, ty = (nby + t.BY - 1) / t.BY, tn = (N + t.NB - 1) / t.NB;
+        const long long tiles = (long long)tn * ty * tx;
+        const long long waves = (tiles * n_fchunks + sms - 1) / sms;
+        const long long cover = tiles * lanes;
+        if (waves < best_waves ||
+            (waves == best_waves && (cover < best_cover || (cover == best_cover && t.BX > rect.BX)))) {
+            rect = t;
+            rtx = tx;
+            rty = ty;
+            rtn = tn;
+            best_waves = waves;
+            best_cover = cover;
+            have_rect = true;
         }
     }
-    pl.KS = best_ks;
-    const int per = (nck_total + best_ks - 1) / best_ks;
-    pl.c_split = per * ck;
-    pl.n_chunks = std::min(per, nck_total);
-    pl.ws_bytes = best_ks > 1 ? (size_t)best_ks * out_elems * 4 : 0;
-    *out = pl;
+    // the linear tile stages whole images (fewer channels per stage) and its lanes hit more bank
+    // conflicts; it must beat the best rectangle by that margin in estimated channel steps
+    Plan pr, pli;
+    const double cr = have_rect ? finish(rect, rtx, rty, rtn, &pr) : 1e300;
+    const int ltn = (int)(((long long)N * nby * nbx + lanes - 1) / lanes);
+    const double cl = have_lin ? 1.2 * finish(lin, 1, 1, ltn, &pli) : 1e300;
+    if (cr >= 1e300 && cl >= 1e300) return PP_ERR_SHAPE;
+    *out = cl < cr ? pli : pr;
     return PP_OK;
 }
 
