@@ -77,6 +77,7 @@ constexpr int kStages = 3;                         // input-channel pipeline dep
 constexpr int kMaxChunks = 256;                    // input-channel stages per CTA
 constexpr long long kTimeoutCycles = 2000000000LL; // about one second of SM clock
 constexpr uint32_t kTmemCols = 512;                // 16 warps x 8 slots x 16 accumulators
+constexpr int kMaxUnitsPerCta = 64;                // units one persistent CTA holds in its table
 
 // Device status word: a wait that ran out of time records its code here and the kernel returns
 // early instead of hanging (read back by pp_device_status).
@@ -97,6 +98,7 @@ struct TmParams {
     int BY, BX, NB;                    // spatial tile: BY x BX blocks (4x4 outputs) of NB images
     int tiles_x, tiles_y, tiles_n, n_fchunks;
     int linear;                        // linear tiles: lanes take consecutive blocks across images
+    int n_units;                       // units: tiles x filter chunks x input-channel splits
     int CK, n_chunks, maxk;            // channels per stage, stages per CTA (max), max kept per group-stage
     int KS, c_split;                   // input-channel splits; channels per split (multiple of CK)
     float* ws;                         // KS > 1: fp32 partial sums [KS][N][Cout][Ho][Wo]
@@ -218,34 +220,66 @@ __device__ __forceinline__ void stage_input_share(const TmParams& p, float* s_in
     }
 }
 
-// This thread's share of filling pipeline stage k % kStages with input channel chunk k
+// One unit of work of a CTA: a spatial tile, a filter chunk (WG groups) and an input-channel
+// split.  Units are numbered with the filter chunk fastest, so CTAs working at the same time
+// share input tiles in L2.
+struct __align__(16) Unit {
+    int ks, tn, n0, oy0, ox0, iy0, ix0, g0, c_lo, c_hi, nck, pad;
+};
+
+template <int S>
+__device__ __forceinline__ Unit unit_of(const TmParams& p, int u) {
+    Unit U;
+    const int fchunk = u % p.n_fchunks;
+    int t = u / p.n_fchunks;
+    const int tx = t % p.tiles_x;
+    t /= p.tiles_x;
+    const int ty = t % p.tiles_y;
+    t /= p.tiles_y;
+    U.tn = t % p.tiles_n;
+    U.ks = t / p.tiles_n;
+    U.c_lo = U.ks * p.c_split;
+    U.c_hi = min(p.C, U.c_lo + p.c_split);
+    U.nck = (U.c_hi - U.c_lo + p.CK - 1) / p.CK;
+    // linear tiles: tile tn holds blocks [tn * lanes, (tn + 1) * lanes) of the (image, block row,
+    // block column) sequence and stages the whole images from n0 on
+    U.n0 = p.linear ? (int)(((long long)U.tn * 32 * p.WS) / (p.BY * p.BX)) : U.tn * p.NB;
+    U.oy0 = ty * p.BY * 4;
+    U.ox0 = tx * p.BX * 4;
+    U.iy0 = U.oy0 * S - 1;          // stage origin: 1 halo row, 16-byte aligned column
+    U.ix0 = U.ox0 * S - 4;
+    U.g0 = fchunk * p.WG;
+    return U;
+}
+
+// This thread's share of filling pipeline stage q % kStages with input channel chunk k of unit U
 // (non-blocking): warp 0 lane 0 issues the input tile's TMA, or every thread copies its share of
-// the tile; the warps of filter group wg copy that group's descriptors and kept weights.  The
-// stage's full barrier completes when all 512 threads have arrived and every byte has landed.
+// the tile; the warps of filter group wg copy that group's descriptors and its kept weights
+// vals[beg, end).  The stage's full barrier completes when all 512 threads have arrived and
+// every byte has landed.
 template <typename TIn>
 __device__ __forceinline__ void fill_share(const TmParams& p, const CUtensorMap* tmap, unsigned char* smem,
-                                           const uint32_t* s_kb, uint32_t full0, int k, int n0, int iy0,
-                                           int ix0, int g0, int c_lo, int c_hi, int warp, int lane) {
-    const int s = k % kStages;
-    const int nkb = p.n_chunks + 1;
+                                           uint32_t full0, int q, const Unit& U, int k, uint32_t beg,
+                                           uint32_t end, int warp, int lane) {
+    const int s = q % kStages;
     unsigned char* st = smem + p.stage_off + (size_t)s * p.stage_bytes;
     const uint32_t fb = full0 + 8 * s;
-    const int c0 = c_lo + k * p.CK, ckv = min(p.CK, c_hi - c0);
+    const int c0 = U.c_lo + k * p.CK, ckv = min(p.CK, U.c_hi - c0);
     if (warp == 0 && lane == 0) {
         mbar_arrive_expect_tx(fb, p.use_tma ? p.tma_bytes : 0u);
         if (p.use_tma) {
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            tma_load_4d(smem_u32(st), tmap, ix0, iy0, c0, n0, fb);
+            tma_load_4d(smem_u32(st), tmap, U.ix0, U.iy0, c0, U.n0, fb);
         }
     }
-    if (!p.use_tma) stage_input_share<TIn>(p, reinterpret_cast<float*>(st), c0, ckv, n0, iy0, ix0, warp * 32 + lane);
-    const int wg = warp / p.WS, ws = warp - wg * p.WS, g = g0 + wg;
+    if (!p.use_tma)
+        stage_input_share<TIn>(p, reinterpret_cast<float*>(st), c0, ckv, U.n0, U.iy0, U.ix0, warp * 32 + lane);
+    const int wg = warp / p.WS, ws = warp - wg * p.WS, g = U.g0 + wg;
     if (g < p.G) {
         uint64_t* sd = reinterpret_cast<uint64_t*>(st + p.desc_off) + wg * p.CK;
         for (int cl = ws * 32 + lane; cl < ckv; cl += p.WS * 32)
             cp_async8(sd + cl, p.desc + (size_t)g * p.C + c0 + cl);
         float4* sv = reinterpret_cast<float4*>(st + p.vals_off) + wg * p.maxk;
-        const uint32_t beg = s_kb[wg * nkb + k], end = s_kb[wg * nkb + k + 1];
         for (uint32_t i = beg + ws * 32 + lane; i < end; i += p.WS * 32) cp_async16(sv + (i - beg), p.vals + i);
     }
     __threadfence_block();   // orders the fp16 path's plain shared stores before the arrival
@@ -263,39 +297,19 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     uint64_t* bar = reinterpret_cast<uint64_t*>(smem);
     uint32_t* s_tmem = reinterpret_cast<uint32_t*>(smem + 16 * kStages);
     uint32_t* s_issued = s_tmem + 1;
-    uint32_t* s_kb = reinterpret_cast<uint32_t*>(smem + p.kb_off);
     const uint32_t full0 = smem_u32(bar), empty0 = full0 + 8 * kStages;
 
-    // CTA -> (spatial tile, filter chunk); the filter chunk varies fastest so CTAs that share an
-    // input tile run together and hit it in L2
-    const int cta = blockIdx.x;
-    const int fchunk = cta % p.n_fchunks;
-    int t = cta / p.n_fchunks;
-    const int tx = t % p.tiles_x;
-    t /= p.tiles_x;
-    const int ty = t % p.tiles_y;
-    t /= p.tiles_y;
-    const int tn = t % p.tiles_n;
-    const int ks = t / p.tiles_n;                         // input-channel split of this CTA
-    const int c_lo = ks * p.c_split, c_hi = min(p.C, c_lo + p.c_split);
-    const int nck = (c_hi - c_lo + p.CK - 1) / p.CK;       // channel chunks of this CTA
-    // linear tiles: tile tn holds blocks [tn * lanes, (tn + 1) * lanes) of the (image, block row,
-    // block column) sequence and stages the whole images from n0 on
-    const int lanes_t = 32 * p.WS, bpi = p.BY * p.BX;
-    const int n0 = p.linear ? (int)(((long long)tn * lanes_t) / bpi) : tn * p.NB;
-    const int oy0 = ty * p.BY * RY, ox0 = tx * p.BX * RX;
-    const int iy0 = oy0 * S - 1, ix0 = ox0 * S - 4;     // stage origin: 1 halo row, 16-B aligned col
-    const int g0 = fchunk * p.WG;
-    const int nkb = p.n_chunks + 1;
+    // this CTA's units: blockIdx.x, blockIdx.x + gridDim.x, ... (one per CTA unless the launch is
+    // persistent); their chunks form one stream q = 0 .. Q-1 through the three stages, so the
+    // next unit's first stages fill while the current one finishes
+    const int n_my = p.n_units > (int)blockIdx.x ? (p.n_units - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+    Unit* s_units = reinterpret_cast<Unit*>(smem + p.kb_off);   // at most kMaxUnitsPerCta
+    if ((int)threadIdx.x < n_my) s_units[threadIdx.x] = unit_of<S>(p, blockIdx.x + threadIdx.x * gridDim.x);
 
     if (!p.use_tma) {   // the fallback writes only in-image elements: zero all stages once
         float* z = reinterpret_cast<float*>(smem + p.stage_off);
         const int nf = (int)(kStages * p.stage_bytes / 4);
         for (int i = threadIdx.x; i < nf; i += kThreadsTM) z[i] = 0.0f;
-    }
-    for (int i = threadIdx.x; i < p.WG * nkb; i += kThreadsTM) {
-        const int wg = i / nkb, j = i - wg * nkb, g = g0 + wg;
-        s_kb[i] = g < p.G ? p.kofs[(size_t)g * p.C + min(c_lo + j * p.CK, c_hi)] : 0u;
     }
     if (warp == 0) {
         if (lane == 0) {
@@ -313,83 +327,98 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tbase = *s_tmem;
+    int Q = 0;
+    for (int i = 0; i < n_my; ++i) Q += s_units[i].nck;
 
+    const int wg = warp / p.WS, ws = warp - (warp / p.WS) * p.WS;
+    // fill cursor: unit fi (of this CTA), its chunk fk, and the warp's group's weight range for
+    // that chunk (loaded one fill ahead, so its latency hides behind a chunk of compute)
+    // (units are read from the table where needed: few registers live across the loop)
+    int fi = 0, fk = 0;
+    uint32_t fbeg = 0, fend = 0;
+    auto fetch_range = [&]() {
+        fbeg = fend = 0;
+        if (fi < n_my) {
+            const Unit FU = s_units[fi];
+            const int g = FU.g0 + wg;
+            if (g < p.G) {
+                const int c0 = FU.c_lo + fk * p.CK;
+                const size_t b = (size_t)g * p.C;
+                fbeg = p.kofs[b + c0];
+                fend = p.kofs[b + min(c0 + p.CK, FU.c_hi)];
+            }
+        }
+    };
+    auto advance_fill = [&]() {
+        if (++fk == s_units[fi].nck) {
+            fk = 0;
+            ++fi;
+        }
+        fetch_range();
+    };
+    auto fill = [&](int q) {
+        fill_share<TIn>(p, &tmap, smem, full0, q, s_units[fi], fk, fbeg, fend,
+                        warp, lane);
+        advance_fill();
+    };
+    fetch_range();
     {   // prologue: every thread's share of the first kStages chunks
-        const int first = min(kStages, nck);
-        for (int k = 0; k < first; ++k)
-            fill_share<TIn>(p, &tmap, smem, s_kb, full0, k, n0, iy0, ix0, g0, c_lo, c_hi, warp, lane);
+        const int first = min(kStages, Q);
+        for (int q = 0; q < first; ++q) fill(q);
         if (threadIdx.x == 0) *s_issued = first;
     }
 
-    const int wg = warp / p.WS, ws = warp - (warp / p.WS) * p.WS;
-    const int g = g0 + wg;
     // tensor memory: warp w owns lanes 32*(w%4).. and columns 128*(w/4) + 16*slot ..
     const uint32_t tw = tbase + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)(128 * (warp >> 2));
 #pragma unroll
     for (int f = 0; f < kF; ++f) tmem_zero16(tw + 16u * f);
 
     const int blk = ws * 32 + lane;
-    int img, rem;
-    bool active;
-    if (p.linear) {
-        const long long b = (long long)tn * lanes_t + blk;
-        const int ng = (int)(b / bpi);
-        img = ng - n0;
-        rem = (int)(b - (long long)ng * bpi);
-        active = ng < p.N && img < p.NB;
-    } else {
-        img = blk / bpi;
-        rem = blk - img * bpi;
-        active = img < p.NB;
-    }
-    const int by = rem / p.BX, bx = rem - (rem / p.BX) * p.BX;
+    const int lanes_t = 32 * p.WS, bpi = p.BY * p.BX;
     const int plane = p.IH * p.BWb;
-    const int in_off = active ? img * p.CK * plane + by * RY * S * p.BWb + bx * RX * S + 3 : 3;
-
-    for (int k = 0; k < nck; ++k) {
-        const int s = k % kStages;
-        if (!mbar_wait_warp(full0 + 8 * s, (k / kStages) & 1, p.status, kStatusFullTimeout)) break;
-        if (g < p.G) {
-            const unsigned char* st = smem + p.stage_off + (size_t)s * p.stage_bytes;
-            const uint32_t win_addr = smem_u32(reinterpret_cast<const float*>(st) + in_off);
-            const uint32_t desc_addr = smem_u32(reinterpret_cast<const uint64_t*>(st + p.desc_off) + wg * p.CK);
-            const uint32_t vals_addr = smem_u32(reinterpret_cast<const float4*>(st + p.vals_off) + wg * p.maxk);
-            const int ckv = min(p.CK, c_hi - c_lo - k * p.CK);
-            if constexpr (S == 1) {
-                PP_STAGE_KERNELS_S1(ckv, desc_addr, vals_addr, win_addr, 4 * p.BWb, 4 * plane, tw);
-            } else {
-                PP_STAGE_KERNELS_S2(ckv, desc_addr, vals_addr, win_addr, 4 * p.BWb, 4 * plane, tw);
-            }
+    // compute cursor: unit ci, its chunk ck, and this lane's block of the unit's tile
+    int ci = 0, ck = 0;
+    int img = 0, by = 0, bx = 0, in_off = 3;
+    bool active = false;
+    auto place_lane = [&]() {
+        const Unit CU = s_units[ci];
+        int rem;
+        if (p.linear) {
+            const long long b = (long long)CU.tn * lanes_t + blk;
+            const int ng = (int)(b / bpi);
+            img = ng - CU.n0;
+            rem = (int)(b - (long long)ng * bpi);
+            active = ng < p.N && img < p.NB;
+        } else {
+            img = blk / bpi;
+            rem = blk - img * bpi;
+            active = img < p.NB;
         }
-        // release the stage, then take this warp's share of filling chunk k + kStages - 1 into the
-        // stage chunk k - 1 used, once all 16 warps have released that one
-        __syncwarp();
-        if (lane == 0) mbar_arrive(empty0 + 8 * s);
-        const int j = k + kStages - 1;
-        if (k >= 1 && j < nck) {
-            if (!mbar_wait_warp(empty0 + 8 * (j % kStages), ((k - 1) / kStages) & 1, p.status, kStatusEmptyTimeout))
-                break;
-            fill_share<TIn>(p, &tmap, smem, s_kb, full0, j, n0, iy0, ix0, g0, c_lo, c_hi, warp, lane);
-            if (threadIdx.x == 0) *s_issued = j + 1;
-        }
-    }
+        by = rem / p.BX;
+        bx = rem - by * p.BX;
+        in_off = active ? img * p.CK * plane + by * RY * S * p.BWb + bx * RX * S + 3 : 3;
+    };
+    place_lane();
 
-    // epilogue: accumulators out of tensor memory, + bias, ReLU, store to the original channel
-    {
-        const int n = n0 + img;
-        const int oyb = oy0 + by * RY, oxb = ox0 + bx * RX;
-        using TOut = TIn;
-        TOut* y = static_cast<TOut*>(p.y);
+    using TOut = TIn;
+    TOut* y = static_cast<TOut*>(p.y);
+    // accumulators of unit U out of tensor memory (zeroed behind) + bias, ReLU, optional pool, to
+    // the original channel; with a split, raw partial sums to the workspace
+    auto epilogue = [&](const Unit& U) {
+        const int g = U.g0 + wg;
+        const int n = U.n0 + img;
+        const int oyb = U.oy0 + by * RY, oxb = U.ox0 + bx * RX;
 #pragma unroll 1
         for (int f = 0; f < kF; ++f) {
             float a[16];
             __syncwarp();
             tmem_ld16(tw + 16u * f, a);
+            tmem_zero16(tw + 16u * f);
             if (g >= p.G || !active || n >= p.N) continue;
             const uint32_t co = p.perm[g * kF + f];
             if (co == kPadSlot) continue;
             if (p.KS > 1) {   // raw partial sums of this split; bias, ReLU and rounding come later
-                float* wc = p.ws + (size_t)ks * p.ws_stride + ((size_t)n * p.Cout + co) * p.Ho * p.Wo;
+                float* wc = p.ws + (size_t)U.ks * p.ws_stride + ((size_t)n * p.Cout + co) * p.Ho * p.Wo;
 #pragma unroll
                 for (int r = 0; r < RY; ++r) {
                     const int oy = oyb + r;
@@ -468,7 +497,42 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
                 }
             }
         }
+    };
+
+    for (int q = 0; q < Q; ++q) {
+        const int s = q % kStages;
+        if (!mbar_wait_warp(full0 + 8 * s, (q / kStages) & 1, p.status, kStatusFullTimeout)) break;
+        const Unit CU = s_units[ci];
+        if (CU.g0 + wg < p.G) {
+            const unsigned char* st = smem + p.stage_off + (size_t)s * p.stage_bytes;
+            const uint32_t win_addr = smem_u32(reinterpret_cast<const float*>(st) + in_off);
+            const uint32_t desc_addr = smem_u32(reinterpret_cast<const uint64_t*>(st + p.desc_off) + wg * p.CK);
+            const uint32_t vals_addr = smem_u32(reinterpret_cast<const float4*>(st + p.vals_off) + wg * p.maxk);
+            const int ckv = min(p.CK, CU.c_hi - CU.c_lo - ck * p.CK);
+            if constexpr (S == 1) {
+                PP_STAGE_KERNELS_S1(ckv, desc_addr, vals_addr, win_addr, 4 * p.BWb, 4 * plane, tw);
+            } else {
+                PP_STAGE_KERNELS_S2(ckv, desc_addr, vals_addr, win_addr, 4 * p.BWb, 4 * plane, tw);
+            }
+        }
+        // release the stage, then take this warp's share of filling chunk q + kStages - 1 into the
+        // stage chunk q - 1 used, once all 16 warps have released that one
+        __syncwarp();
+        if (lane == 0) mbar_arrive(empty0 + 8 * s);
+        const int j = q + kStages - 1;
+        if (q >= 1 && j < Q) {
+            if (!mbar_wait_warp(empty0 + 8 * (j % kStages), ((q - 1) / kStages) & 1, p.status, kStatusEmptyTimeout))
+                break;
+            fill(j);
+            if (threadIdx.x == 0) *s_issued = j + 1;
+        }
+        if (++ck == CU.nck) {   // unit done: results out, accumulators zeroed, next unit's tile
+            epilogue(CU);
+            ck = 0;
+            if (++ci < n_my) place_lane();
+        }
     }
+
     asm volatile("cp.async.wait_all;" ::: "memory");   // this thread's copies (only after a timeout)
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
@@ -1117,8 +1181,7 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
             const size_t desc_b = align_up((size_t)wg * ck * 8, 16);
             const size_t vals_b = (size_t)wg * std::max(maxk, 1) * 16;
             *stage_bytes = align_up(in_b + desc_b + vals_b, 128);
-            const int nch = (C + ck - 1) / ck;
-            *kb_bytes = (size_t)wg * (nch + 1) * 4;
+            *kb_bytes = (size_t)kMaxUnitsPerCta * sizeof(int) * 12;   // the CTA's unit table
             return align_up(64 + *kb_bytes, 128) + kStages * *stage_bytes;
         };
         int ck = std::min(C, 64);
@@ -1354,8 +1417,15 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
     }
     auto kern = pconv_tm<S, T>;
     if (!allow_max_smem<S, T>(pl.smem)) return PP_ERR_CUDA;
-    const long long ctas = pl.ctas * pl.KS;
-    if (ctas > INT_MAX) return PP_ERR_SHAPE;
+    const long long units = pl.ctas * pl.KS;
+    if (units > INT_MAX) return PP_ERR_SHAPE;
+    p.n_units = (int)units;
+    // TMA path: one persistent CTA per SM walks its units as one chunk stream (the halo is zero
+    // filled by the TMA unit, so stages carry over between tiles); the copy fallback relies on
+    // stages zeroed once, so there every unit gets its own CTA
+    const long long ctas = p.use_tma ? std::max<long long>(std::min<long long>(units, sm_count()),
+                                                           (units + kMaxUnitsPerCta - 1) / kMaxUnitsPerCta)
+                                     : units;
     kern<<<(unsigned)ctas, kThreadsTM, pl.smem, st>>>(p, tmap);
     if (cudaGetLastError() != cudaSuccess) return PP_ERR_CUDA;
     if (pl.KS > 1) {
