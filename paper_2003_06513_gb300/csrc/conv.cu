@@ -1209,12 +1209,40 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
             }
         }
         pl->KS = best_ks;
-        const int per = (nck_total + best_ks - 1) / best_ks;
+        int per = (nck_total + best_ks - 1) / best_ks;
         pl->c_split = per * ck;
         pl->n_chunks = std::min(per, nck_total);
         pl->ws_bytes = best_ks > 1 ? (size_t)best_ks * out_elems * 4 : 0;
-        const long long waves = (pl->ctas * best_ks + sms - 1) / sms;
-        return (double)waves * (std::min(pl->c_split, C) + 2.0 * per + 2.0 * ck);
+        long long waves = (pl->ctas * best_ks + sms - 1) / sms;
+        double steps = (double)waves * (std::min(pl->c_split, C) + 2.0 * per + 2.0 * ck);
+        // tiny launches (the SMs stay idle even with 8 splits): fewer channels per stage and up to
+        // 64 splits within one wave, chosen by estimated channel steps
+        if (pl->ctas * std::min(8, nck_total) < sms) {
+            for (int ck2 = ck;; ck2 = std::max(1, ck2 / 2)) {
+                const int nck2 = (C + ck2 - 1) / ck2;
+                if (nck2 > kMaxChunks) break;
+                for (int ksp = 2; ksp <= std::min(64, nck2); ++ksp) {
+                    const int per2 = (nck2 + ksp - 1) / ksp;
+                    if ((nck2 + per2 - 1) / per2 != ksp) continue;
+                    if (ws_avail < (size_t)ksp * out_elems * 4 || pl->ctas * ksp > sms) break;   // one wave
+                    const long long w2 = (pl->ctas * ksp + sms - 1) / sms;
+                    const double st2 = (double)w2 * (std::min(per2 * ck2, C) + 2.0 * per2 + 2.0 * ck2) + 4.0;
+                    if (st2 < steps - 1e-9) {
+                        steps = st2;
+                        pl->CK = ck2;
+                        pl->KS = ksp;
+                        per = per2;
+                        pl->c_split = per2 * ck2;
+                        pl->n_chunks = std::min(per2, nck2);
+                        pl->ws_bytes = (size_t)ksp * out_elems * 4;
+                        pl->maxk = std::max(maxk_for(ck2), 1);
+                    }
+                }
+                if (ck2 == 1) break;
+            }
+            pl->smem = layout(pl->CK, pl->maxk, &pl->stage_bytes, &pl->kb_bytes);
+        }
+        return steps;
     };
 
     // rectangles: fewest CTA waves, then fewest lanes covered (idle lanes), then the widest rows;
