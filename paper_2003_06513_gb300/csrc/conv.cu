@@ -379,6 +379,7 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     // compute cursor: unit ci, its chunk ck, and this lane's block of the unit's tile
     int ci = 0, ck = 0;
     int img = 0, by = 0, bx = 0, in_off = 3;
+    uint32_t edge = 1;
     bool active = false;
     auto place_lane = [&]() {
         const Unit CU = s_units[ci];
@@ -397,6 +398,9 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
         by = rem / p.BX;
         bx = rem - by * p.BX;
         in_off = active ? img * p.CK * plane + by * RY * S * p.BWb + bx * RX * S + 3 : 3;
+        // lanes whose left neighbour lane does not hold the block to their left (stride 2 takes
+        // window column 0 from that neighbour)
+        edge = (bx == 0 || lane == 0) ? 1u : 0u;
     };
     place_lane();
 
@@ -510,9 +514,9 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
             const uint32_t vals_addr = smem_u32(reinterpret_cast<const float4*>(st + p.vals_off) + wg * p.maxk);
             const int ckv = min(p.CK, CU.c_hi - CU.c_lo - ck * p.CK);
             if constexpr (S == 1) {
-                PP_STAGE_KERNELS_S1(ckv, desc_addr, vals_addr, win_addr, 4 * p.BWb, 4 * plane, tw);
+                PP_STAGE_KERNELS_S1(ckv, desc_addr, vals_addr, win_addr, 4 * p.BWb, 4 * plane, tw, edge);
             } else {
-                PP_STAGE_KERNELS_S2(ckv, desc_addr, vals_addr, win_addr, 4 * p.BWb, 4 * plane, tw);
+                PP_STAGE_KERNELS_S2(ckv, desc_addr, vals_addr, win_addr, 4 * p.BWb, 4 * plane, tw, edge);
             }
         }
         // release the stage, then take this warp's share of filling chunk q + kStages - 1 into the

@@ -41,14 +41,15 @@ def macro(S):
     # operands: %0 channels, %1 descriptor address, %2 weights address, %3 window address of
     # channel 0, %4 row pitch in bytes, %5 channel plane in bytes, %6 tensor-memory base
     L = ["{",
-         ".reg .pred P;",
+         ".reg .pred P, EL;",
          f".reg .b32 cl, cnt, code, ta, pat, va, da, t1, {rows};",
          ".reg .b64 d, dd;",
          f".reg .f32 x<{WY * WX}>, a<{R}>, w<4>;",
          "mov.b32 cl, %0;",
          "mov.b32 da, %1;",
          "mov.b32 va, %2;",
-         "mov.b32 rb0, %3;"]
+         "mov.b32 rb0, %3;",
+         "setp.ne.u32 EL, %7, 0;"]
     for r in range(1, WY):
         L.append(f"add.u32 rb{r}, rb{r - 1}, %4;")
     L += ["CL:",
@@ -60,9 +61,18 @@ def macro(S):
           "and.b32 cnt, cnt, 15;",
           "setp.eq.u32 P, cnt, 0;",
           "@P bra.uni CN;"]
-    # window: column 0 alone, then aligned groups of four
+    # window: column 0 alone, then aligned groups of four.  Stride 2: lanes sit 32 bytes apart, so
+    # a scalar load of column 0 meets an 8-way bank conflict; it is the left neighbour lane's
+    # column 8 instead (a warp shuffle), and only lanes at the start of a tile row or of the warp
+    # (%7 nonzero) load it from shared memory
     for r in range(WY):
         base = r * WX
+        if S == 2:
+            L.append(f"ld.shared.v4.f32 {{x{base + 1}, x{base + 2}, x{base + 3}, x{base + 4}}}, [rb{r}+4];")
+            L.append(f"ld.shared.v4.f32 {{x{base + 5}, x{base + 6}, x{base + 7}, x{base + 8}}}, [rb{r}+20];")
+            L.append(f"shfl.sync.up.b32 x{base}, x{base + 8}, 1, 0, -1;")
+            L.append(f"@EL ld.shared.f32 x{base}, [rb{r}];")
+            continue
         L.append(f"ld.shared.f32 x{base}, [rb{r}];")
         c = 1
         while c + 4 <= WX:
@@ -117,9 +127,9 @@ def macro(S):
           "}"]
     body = "\\n\\t".join(L)
     return (f"// stride {S}: 4x4 outputs per lane, {WY}x{WX} input window\n"
-            f"#define PP_STAGE_KERNELS_S{S}(nch, desc_addr, vals_addr, win_addr, pitch_b, plane_b, tbase) \\\n"
+            f"#define PP_STAGE_KERNELS_S{S}(nch, desc_addr, vals_addr, win_addr, pitch_b, plane_b, tbase, edge) \\\n"
             f'    asm volatile("{body}" :: "r"(nch), "r"(desc_addr), "r"(vals_addr), "r"(win_addr), '
-            f'"r"(pitch_b), "r"(plane_b), "r"(tbase) : "memory")\n')
+            f'"r"(pitch_b), "r"(plane_b), "r"(tbase), "r"(edge) : "memory")\n')
 
 
 def main():
