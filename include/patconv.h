@@ -91,6 +91,20 @@ typedef enum {
  * if masks is NULL with capacity > 0). */
 int pp_default_patterns(uint16_t* masks, int capacity);
 
+/* Pattern-library design heuristic (§4.2): the central weight is always kept, and each kernel
+ * proposes the pattern made of the centre and its three largest non-central weights (largest
+ * magnitude; equal magnitudes take the lower raster tap first); the m most frequent proposals
+ * over all kernels given form the library, ordered by frequency (descending), equal counts by
+ * mask value (ascending) -- the order matters, because projection ties go to the lower index.
+ *   W       HOST fp32 [n_kernels][9]: every 3x3 kernel of the network (or layer), raster taps;
+ *   m       library size, 1..8 (§4.2 finds 6-8 best);
+ *   masks   HOST out, room for m masks; *n_masks gets the number written (fewer than m when
+ *           fewer distinct proposals exist).
+ * A library other than pp_default_patterns packs and runs through pp_pack / pp_conv like the
+ * default one; dense layers then take the generic kernel (taps from a table, slower).
+ * Errors: PP_ERR_NULL, PP_ERR_SHAPE (n_kernels == 0, m outside 1..8), PP_ERR_NONFINITE. */
+int pp_design_patterns(const float* W, size_t n_kernels, int m, uint16_t* masks, int* n_masks);
+
 /* Pattern projection (§4.3 Eq. 6), connectivity pruning (§4.4) and packing (§3.4) of one layer.
  *   W        host fp32 [Cout][Cin/groups][3][3], read only, caller-owned;
  *   groups   1 (dense) or Cout == Cin (depthwise);

@@ -91,3 +91,30 @@ def grid(mask: int) -> str:
     for r in range(3):
         rows.append("".join("x" if (mask >> (3 * r + c)) & 1 else "." for c in range(3)))
     return "\n".join(rows)
+
+
+def design_library(kernels, m: int) -> List[int]:
+    """Pattern library by the heuristic of §4.2 (plain loops over the kernels).
+
+    The central weight is never pruned; each kernel proposes the pattern formed by the centre and
+    the locations of its three largest weights (largest magnitude, among the eight non-central
+    taps -- readings of this library: magnitude, and equal magnitudes take the lower raster tap
+    first).  The m most commonly proposed patterns over all kernels form the library, ordered by
+    count descending, equal counts by mask value ascending.  ``kernels``: rows of 9 raster taps.
+    """
+    counts = {}
+    for row in kernels:
+        w = [float(v) for v in row]
+        chosen = [CENTRE]
+        for _ in range(3):
+            best = None
+            for t in range(9):
+                if t in chosen:
+                    continue
+                if best is None or abs(w[t]) > abs(w[best]):
+                    best = t
+            chosen.append(best)
+        mk = mask_of(chosen)
+        counts[mk] = counts.get(mk, 0) + 1
+    ranked = sorted(counts, key=lambda mk: (-counts[mk], mk))
+    return ranked[:m]

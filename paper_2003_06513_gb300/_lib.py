@@ -26,6 +26,8 @@ SIGNATURES = {
                          _c_void_p, _c_void_p]),
     "pp_conv_ws": (_c_int, [_c_void_p, _c_void_p, _c_int, _c_int, _c_int, _c_int, _c_void_p, _c_int,
                             _c_void_p, _c_void_p, _c_size_t, _c_void_p]),
+    "pp_design_patterns": (_c_int, [ctypes.POINTER(ctypes.c_float), _c_size_t, _c_int,
+                                    ctypes.POINTER(ctypes.c_uint16), ctypes.POINTER(_c_int)]),
     "pp_conv_pool_ws": (_c_int, [_c_void_p, _c_void_p, _c_int, _c_int, _c_int, _c_int, _c_void_p, _c_int,
                                  _c_void_p, _c_void_p, _c_size_t, _c_void_p]),
     "pp_conv_workspace_size": (_c_int, [_c_void_p, _c_int, _c_int, _c_int, ctypes.POINTER(_c_size_t)]),

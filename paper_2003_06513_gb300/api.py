@@ -165,6 +165,18 @@ class Layer:
                 pass
 
 
+def design_patterns(weights: Sequence, m: int = 8) -> list:
+    """Pattern library of at most m masks from the kernels of ``weights`` (arrays [..., 3, 3]) by
+    the §4.2 heuristic (pp_design_patterns): centre + three largest-magnitude taps per kernel,
+    the m most frequent of those."""
+    W = np.ascontiguousarray(np.concatenate([np.asarray(w, np.float32).reshape(-1, 9) for w in weights]))
+    masks = (ctypes.c_uint16 * m)()
+    n = ctypes.c_int()
+    _lib.check("pp_design_patterns", _lib.load().pp_design_patterns(
+        W.ctypes.data_as(ctypes.POINTER(ctypes.c_float)), W.shape[0], m, masks, ctypes.byref(n)))
+    return [int(masks[i]) for i in range(n.value)]
+
+
 def pp_pack(W, pattern_set: Optional[Sequence[int]] = None, keep_ratio: float = 1.0,
             groups: int = 1, stride: int = 1) -> Layer:
     """Pattern projection + connectivity pruning + packing of host weights [Cout, Cin_g, 3, 3]."""

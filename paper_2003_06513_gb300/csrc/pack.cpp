@@ -207,6 +207,38 @@ int pp_default_patterns(uint16_t* masks, int capacity) {
     return kMaxPatterns;
 }
 
+int pp_design_patterns(const float* W, size_t n_kernels, int m, uint16_t* masks, int* n_masks) {
+    if (!W || !masks || !n_masks) return PP_ERR_NULL;
+    if (n_kernels == 0 || m < 1 || m > kMaxPatterns) return PP_ERR_SHAPE;
+    // candidate pattern of every kernel: the centre and the three non-central taps of largest
+    // magnitude (equal magnitudes: the lower tap first); a mask is a 9-bit integer < 512
+    std::vector<uint64_t> count(512, 0);
+    for (size_t k = 0; k < n_kernels; ++k) {
+        const float* w = W + 9 * k;
+        for (int t = 0; t < 9; ++t)
+            if (!std::isfinite(w[t])) return PP_ERR_NONFINITE;
+        uint32_t mask = 1u << 4;
+        for (int pick = 0; pick < 3; ++pick) {
+            int best = -1;
+            for (int t = 0; t < 9; ++t) {
+                if (mask >> t & 1u) continue;
+                if (best < 0 || std::fabs(w[t]) > std::fabs(w[best])) best = t;
+            }
+            mask |= 1u << best;
+        }
+        ++count[mask];
+    }
+    // the m most frequent candidates, by count descending, then by mask value ascending
+    std::vector<int> order;
+    for (int mk = 0; mk < 512; ++mk)
+        if (count[mk]) order.push_back(mk);
+    std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return count[a] > count[b]; });
+    const int n = std::min<int>(m, (int)order.size());
+    for (int i = 0; i < n; ++i) masks[i] = (uint16_t)order[i];
+    *n_masks = n;
+    return PP_OK;
+}
+
 int pp_pack(const float* W, int Cout, int Cin, int groups, int stride, const uint16_t* masks,
             int n_patterns, double keep, pp_handle* out) {
     if (!W || !masks || !out) return PP_ERR_NULL;

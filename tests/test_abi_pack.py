@@ -188,3 +188,26 @@ def test_conv_pool_rejections_without_gpu(lib):
     Wt = rng.standard_normal((8, 4, 3, 3)).astype(np.float32)
     dense = api.pp_pack(Wt, None, 0.5)
     assert lib.pp_conv_pool_ws(dense._h, None, 0, 1, 8, 8, None, 1, None, None, 0, None) == -8   # not bound
+
+
+def test_design_patterns_matches_oracle(lib):
+    """pp_design_patterns equals the oracle's heuristic on random kernels and on VGG-16's."""
+    rng = np.random.default_rng(8)
+    cases = [rng.standard_normal((500, 9)).astype(np.float32),
+             rng.integers(-2, 3, size=(400, 9)).astype(np.float32)]          # many magnitude ties
+    cases.append(np.concatenate([WL.weights(L).reshape(-1, 9) for L in WL.vgg16()[:4]]))
+    for K in cases:
+        for m in (1, 6, 8):
+            assert api.design_patterns([K], m) == OP.design_library(K, m)
+
+
+def test_design_patterns_validation(lib):
+    K = np.zeros((2, 9), np.float32)
+    masks = (ctypes.c_uint16 * 8)()
+    n = ctypes.c_int()
+    ptr = K.ctypes.data_as(ctypes.POINTER(ctypes.c_float))
+    assert lib.pp_design_patterns(ptr, 2, 0, masks, ctypes.byref(n)) == -2
+    assert lib.pp_design_patterns(ptr, 2, 9, masks, ctypes.byref(n)) == -2
+    assert lib.pp_design_patterns(ptr, 0, 8, masks, ctypes.byref(n)) == -2
+    K[1, 3] = np.nan
+    assert lib.pp_design_patterns(ptr, 2, 8, masks, ctypes.byref(n)) == -5

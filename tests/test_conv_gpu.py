@@ -180,6 +180,19 @@ def test_depthwise_unaligned_input(dtype):
     assert OC.max_norm_err(y.double().cpu().numpy(), ref, den) <= TOL[dtype]
 
 
+@pytest.mark.parametrize("m", [6, 8])
+def test_designed_library_end_to_end(m):
+    """A library designed from the layer's own kernels (§4.2 heuristic) packs and runs through
+    the same entry points; checked against the oracle projected with that library."""
+    L = WL.vgg16()[2]                                           # 64 -> 128
+    W, b = WL.weights(L), WL.bias(L)
+    masks = api.design_patterns([W], m)
+    assert masks == OP.design_library(W.reshape(-1, 9), m) and len(masks) == m
+    x = WL.layer_input(L, 1)[:, :, :20, :18].copy()
+    check(W, x, b, L.keep, 1, masks=masks)
+    check(W, x, b, L.keep, 2, masks=masks)
+
+
 def test_deterministic_and_zero_batch():
     L = WL.single_layer()
     x = WL.layer_input(L, 2)

@@ -235,3 +235,38 @@ def test_rejects_non_finite():
     W[1, 0, 2, 2] = np.inf
     with pytest.raises(ValueError):
         PR.project(W, P.default8(), 1.0)
+
+
+# --------------------------------------------------------------------------- library design (§4.2)
+
+def _design_fixture():
+    rows = [[float(v) for v in line.split()[1:]] for line in golden_lines("pattern_design_hand.txt")
+            if line.startswith("k ")]
+    return np.array(rows, dtype=np.float32), golden_kv("pattern_design_hand.txt")
+
+
+def test_design_library_hand_fixture():
+    K, g = _design_fixture()
+    assert P.design_library(K, 2) == [int(v) for v in g["lib_m2"]]
+    assert P.design_library(K, 8) == [int(v) for v in g["lib_m8"]]
+
+
+def test_design_library_recovers_planted_patterns():
+    """Kernels built with three dominant non-central taps propose exactly those taps + centre;
+    the library lists the planted masks by how often they were planted."""
+    rng = np.random.default_rng(4)
+    planted = {}
+    rows = []
+    for i in range(300):
+        taps3 = sorted(rng.choice([0, 1, 2, 3, 5, 6, 7, 8], size=3, replace=False).tolist())
+        w = rng.uniform(-0.1, 0.1, size=9)
+        w[4] = rng.uniform(-20, 20)                    # the centre may be the largest or not
+        for t in taps3:
+            w[t] = rng.choice([-1, 1]) * rng.uniform(1.0, 2.0)
+        mk = P.mask_of(taps3 + [4])
+        planted[mk] = planted.get(mk, 0) + 1
+        rows.append(w)
+    lib = P.design_library(np.array(rows, np.float32), 8)
+    expected = sorted(planted, key=lambda mk: (-planted[mk], mk))[:8]
+    assert lib == expected
+    assert all(bin(mk).count("1") == 4 and (mk >> 4) & 1 for mk in lib)
