@@ -178,9 +178,12 @@ int pp_conv_workspace_size(pp_handle h, int N, int H, int W, size_t* bytes);
 
 /* Launch plan of pp_conv_ws for a call shape and workspace size, for tests and tuning:
  * info[0] = path (1 dense fast kernel, 2 depthwise kernel, 3 generic kernel); for path 1:
- * info[1] channel splits KS, [2] workspace bytes used, [3] CTAs, [4..6] tile BY, BX, NB (4x4
- * output blocks, images), [7] channels per stage, [8] filter groups and [9] spatial warps per
- * CTA, [10] shared-memory bytes, [11] stages per CTA.  Writes min(n_info, 12) values.  Host-only. */
+ * info[1] channel splits KS, [2] workspace bytes used, [3] work units (spatial tiles x filter
+ * chunks x splits), [4..6] tile BY, BX, NB (4x4 output blocks, images), [7] channels per stage,
+ * [8] filter groups and [9] spatial warps per CTA, [10] shared-memory bytes, [11] channel chunks
+ * per unit, [12] CTAs launched when the input goes through TMA (fp32 with rows a multiple of 16
+ * bytes: persistent CTAs, at most one per SM unless the units overflow a CTA's unit table; the
+ * copy fallback launches one CTA per unit).  Writes min(n_info, 13) values.  Host-only. */
 int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info);
 
 /* pp_conv_ws for callers that cannot allocate device memory (the paper has no counterpart to

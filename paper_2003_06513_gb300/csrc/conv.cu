@@ -1772,7 +1772,7 @@ int pp_conv_pool_ws(pp_handle h, const void* x, int dtype, int N, int H, int W, 
 int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info) {
     if (!h || !info) return PP_ERR_NULL;
     if (N < 1 || H < 1 || W < 1 || n_info < 1) return PP_ERR_SHAPE;
-    int64_t v[12] = {0};
+    int64_t v[13] = {0};
     if (!h->fast || h->depthwise) {
         v[0] = h->depthwise ? 2 : 3;   // depthwise kernel / generic kernel: no plan, no workspace
     } else {
@@ -1783,6 +1783,10 @@ int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64
         v[1] = pl.KS;
         v[2] = (int64_t)pl.ws_bytes;
         v[3] = pl.ctas * pl.KS;
+        // CTAs of the TMA path (fp32 input, rows a multiple of 16 bytes): persistent, one per SM
+        // unless the units overflow a CTA's table; the copy fallback launches one per unit
+        v[12] = std::max<long long>(std::min<long long>(v[3], sm_count()),
+                                    (v[3] + kMaxUnitsPerCta - 1) / kMaxUnitsPerCta);
         v[4] = pl.tile.BY;
         v[5] = pl.tile.BX;
         v[6] = pl.tile.NB;
@@ -1792,7 +1796,7 @@ int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64
         v[10] = (int64_t)pl.smem;
         v[11] = pl.n_chunks;
     }
-    for (int i = 0; i < n_info && i < 12; ++i) info[i] = v[i];
+    for (int i = 0; i < n_info && i < 13; ++i) info[i] = v[i];
     return PP_OK;
 }
 
