@@ -12,9 +12,16 @@ one lane's 4x4 output block.  Per input channel:
       ld.shared.v4   its four kept weights (consecutive in the compact storage, §3.4)
       tcgen05.ld     the 16 accumulators of its filter slot from tensor memory
       compare tree   three uniform branches select the body of its pattern
-      body           64 fma.rn.f32 whose tap operands are compile-time window registers (the
-                     four kept positions of the pattern, §3.2): nothing is decoded per element
+      body           64 fused multiply-adds whose tap operands are compile-time window registers
+                     (the four kept positions of the pattern, §3.2): nothing is decoded per element
       tcgen05.st     the accumulators back
+
+Stride 1 runs the taps of the centre column (1, 4, 7) as fma.rn.f32x2 on pairs of outputs: their
+window pairs, columns (1, 2) and (3, 4) of each row, are the halves of the row's aligned 16-byte
+load, so they cost no register moves, and each packed instruction does two of the per-lane
+fma.rn.f32 operations (same rounding) in one issue slot.  The other taps read pairs that straddle
+that alignment and stay scalar.  Every pattern holds 1 to 3 centre-column taps, so about a quarter
+of the body's instructions go away.
 
 Every branch is warp-uniform (bra.uni), so no convergence code surrounds the loop.  Taps are
 applied in ascending raster order for every output.  The library masks are the eight defaults
@@ -40,11 +47,15 @@ def macro(S):
     rows = ", ".join(f"rb{r}" for r in range(WY))
     # operands: %0 channels, %1 descriptor address, %2 weights address, %3 window address of
     # channel 0, %4 row pitch in bytes, %5 channel plane in bytes, %6 tensor-memory base
+    packed = S == 1
     L = ["{",
          ".reg .pred P, EL;",
          f".reg .b32 cl, cnt, code, ta, pat, va, da, t1, {rows};",
          ".reg .b64 d, dd;",
-         f".reg .f32 x<{WY * WX}>, a<{R}>, w<4>;",
+         f".reg .f32 x<{WY * WX}>, a<{R}>, w<4>;"]
+    if packed:   # window pairs (row r, columns 1-2 / 3-4), accumulator pairs, duplicated weights
+        L.append(f".reg .b64 xq<{2 * WY}>, ap<{R // 2}>, wq<4>;")
+    L += [
          "mov.b32 cl, %0;",
          "mov.b32 da, %1;",
          "mov.b32 va, %2;",
@@ -82,6 +93,9 @@ def macro(S):
         while c < WX:
             L.append(f"ld.shared.f32 x{base + c}, [rb{r}+{4 * c}];")
             c += 1
+        if packed:
+            L.append(f"mov.b64 xq{2 * r}, {{x{base + 1}, x{base + 2}}};")
+            L.append(f"mov.b64 xq{2 * r + 1}, {{x{base + 3}, x{base + 4}}};")
     L += ["shr.b64 dd, d, 4;",
           "PL:",
           "ld.shared.v4.f32 {w0, w1, w2, w3}, [va];",
@@ -104,12 +118,28 @@ def macro(S):
     for p, m in enumerate(MASKS):
         L.append(f"B{p}:")
         tp = taps(m)
+        if packed:
+            L += [f"mov.b64 ap{i}, {{a{2 * i}, a{2 * i + 1}}};" for i in range(R // 2)]
+            L += [f"mov.b64 wq{k}, {{w{k}, w{k}}};" for k in range(4) if tp[k] % 3 == 1]
         for k in range(4):                   # tap-outer: 16 independent FMAs per tap
             t = tp[k]
+            dy, dx = t // 3, t % 3
+            if packed and dx == 1:           # outputs (r, 0-1) and (r, 2-3): window pairs of row r + dy
+                for r in range(RY):
+                    for h in range(2):
+                        L.append(f"fma.rn.f32x2 ap{2 * r + h}, wq{k}, xq{2 * (r + dy) + h}, ap{2 * r + h};")
+                continue
             for r in range(RY):
                 for c in range(RX):
-                    wr = (r * S + t // 3) * WX + (c * S + t % 3)
-                    L.append(f"fma.rn.f32 a{r * RX + c}, w{k}, x{wr}, a{r * RX + c};")
+                    wr = (r * S + dy) * WX + (c * S + dx)
+                    o = r * RX + c
+                    if packed and c % 2 == 0:
+                        L.append(f"mov.b64 {{a{o}, a{o + 1}}}, ap{o // 2};")
+                    L.append(f"fma.rn.f32 a{o}, w{k}, x{wr}, a{o};")
+                    if packed and c % 2 == 1:
+                        L.append(f"mov.b64 ap{o // 2}, {{a{o - 1}, a{o}}};")
+        if packed:
+            L += [f"mov.b64 {{a{2 * i}, a{2 * i + 1}}}, ap{i};" for i in range(R // 2)]
         if p != len(MASKS) - 1:
             L.append("bra.uni BS;")
     L += ["BS:",
