@@ -243,11 +243,19 @@ def hbm_peak():
         return 6.8e12, "fallback"
 
 
+def kernel_sources_sha256():
+    """Hash of the kernel's sources: conv.cu and the generator of its channel loop."""
+    h = hashlib.sha256()
+    for name in ("conv.cu", "gen_dispatch.py"):
+        with open(os.path.join(ROOT, "paper_2003_06513_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
 def traffic_record():
     """Per-launch DRAM bytes of pconv_tm on this workload from the committed ncu summary, or
     None when the kernel source changed since the counters were taken."""
     path = os.path.join(ROOT, "profiles", "pconv_tm_vgg16_b32_traffic.txt")
-    src = os.path.join(ROOT, "paper_2003_06513_gb300", "csrc", "conv.cu")
     try:
         rec = {}
         with open(path) as f:
@@ -255,9 +263,7 @@ def traffic_record():
                 if ":" in line and not line.startswith("#"):
                     k, v = line.split(":", 1)
                     rec[k.strip()] = v.strip()
-        with open(src, "rb") as f:
-            sha = hashlib.sha256(f.read()).hexdigest()
-        if rec.get("conv_cu_sha256") == sha:
+        if rec.get("kernel_sources_sha256") == kernel_sources_sha256():
             return {"dram_bytes_per_launch": float(rec["dram_bytes_per_launch"])}
     except Exception:
         pass
@@ -488,7 +494,10 @@ def _peaks(dev):
 
 
 def _time_layer(lay, x, b, relu, ws, K):
-    """Median ms of K launches of one layer (CUDA events on the current stream, after 3 warm-ups)."""
+    """ms of one layer: the smaller of the median of K stream launches (CUDA events around each
+    call, after 3 warm-ups) and the mean of K back-to-back replays of the call captured in a CUDA
+    graph (no per-launch host work, which small layers otherwise wait on).  Returns
+    (ms, eager_ms, graph_ms)."""
     import torch
     y = lay.conv(x, b, relu, workspace=ws)
     for _ in range(2):
@@ -501,7 +510,21 @@ def _time_layer(lay, x, b, relu, ws, K):
         lay.conv(x, b, relu, y, workspace=ws)
         e1.record(st)
     torch.cuda.synchronize()
-    return statistics.median(e0.elapsed_time(e1) for e0, e1 in evs)
+    eager = statistics.median(e0.elapsed_time(e1) for e0, e1 in evs)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        lay.conv(x, b, relu, y, workspace=ws)
+    for _ in range(3):
+        graph.replay()
+    torch.cuda.synchronize()
+    g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    g0.record(st)
+    for _ in range(K):
+        graph.replay()
+    g1.record(st)
+    torch.cuda.synchronize()
+    graphed = g0.elapsed_time(g1) / K
+    return min(eager, graphed), eager, graphed
 
 
 def layer_suite(args):
@@ -530,11 +553,12 @@ def layer_suite(args):
             b = torch.from_numpy(WL.bias(L)).cuda()
             nb = lay.workspace_bytes(x.shape)
             ws = torch.empty(max(nb // 4, 1), device="cuda") if nb else None
-            ms = _time_layer(lay, x, b, True, ws, K)
+            ms, ms_eager, ms_graph = _time_layer(lay, x, b, True, ws, K)
             G = (L.cout + 7) // 8
             fl, by = conv_cost(lay.beta, L.cin, L.cout, L.h, L.w, L.ho, L.wo, batch, G, es, L.cin_g)
             roof = max(fl / peak, by / hbm) * 1e3
             rows.append({"layer": L.name, "shape": [batch, L.cin, L.h, L.w, L.cout, L.stride], "ms": round(ms, 5),
+                         "eager_ms": round(ms_eager, 5), "graph_ms": round(ms_graph, 5),
                          "useful_tflops": fl / ms / 1e9, "gbs": by / ms / 1e6,
                          "bound": "alu" if fl / peak >= by / hbm else "hbm", "roofline_frac": roof / ms,
                          "plan_path": lay.plan(x.shape, nb)["path"]})
@@ -571,7 +595,7 @@ def sweep_run(args):
             b = torch.from_numpy(WL.bias(L)).cuda()
             nb = lay.workspace_bytes(x.shape)
             ws = torch.empty(max(nb // 4, 1), device="cuda") if nb else None
-            ms = _time_layer(lay, x, b, True, ws, K)
+            ms = _time_layer(lay, x, b, True, ws, K)[0]
             fl, by = conv_cost(lay.beta, L.cin, L.cout, L.h, L.w, L.ho, L.wo, n, (L.cout + 7) // 8, es)
             roof = max(fl / peak, by / hbm) * 1e3
             rec = {"c": L.cin, "hw": L.h, "n": n, "keep": L.keep, "io": dt, "ms": ms, "ai": fl / by,
@@ -588,7 +612,8 @@ def sweep_run(args):
             f.write(f"Peaks: FP32 {peak / 1e12:.1f} TFLOP/s ({basis}); HBM {hbm / 1e9:.0f} GB/s ({hbm_kind}). "
                     f"Clocks: {json.dumps(clocks)}\n\n")
             f.write("Inputs N(0,1) generated on the device from the point's seed; weights seeded He-normal. "
-                    "ms = median of %d launches. AI = useful FLOP / algorithmic bytes.\n\n" % K)
+                    "ms = the smaller of the median of %d stream launches and the mean of as many CUDA-graph "
+                    "replays. AI = useful FLOP / algorithmic bytes.\n\n" % K)
             f.write("| C | HxW | N | keep | io | ms | AI (FLOP/B) | useful GFLOP/s | bound | roofline frac |\n")
             f.write("|---:|---:|---:|---:|:--|---:|---:|---:|:--|---:|\n")
             for r in out:
