@@ -95,6 +95,27 @@ def test_shapes_fp32(N, Cin, Cout, H, W, keep, stride):
     check(Wt, x, b, keep, stride)
 
 
+@pytest.mark.parametrize("ws", [False, True])
+@pytest.mark.parametrize("N,Cin,Cout,H,W,keep,stride", [
+    (1, 8, 8, 3, 1000, 0.5, 1),      # rows wider than any tile: several tiles along x
+    (1, 8, 8, 3, 1001, 0.5, 2),
+    (1, 16, 8, 5, 2100, 0.5, 1),
+    (2, 4, 8, 300, 3, 1.0, 1),       # tall and narrow
+    (1, 2048, 16, 2, 2, 0.2, 1),     # many input channels on a tiny image: 32+ stages per unit
+    (1, 4096, 8, 1, 1, 0.1, 1)])     # a 1 x 1 image: every tap but the centre reads padding
+def test_extreme_shapes(N, Cin, Cout, H, W, keep, stride, ws):
+    rng = np.random.default_rng(Cin + W)
+    Wt = (rng.standard_normal((Cout, Cin, 3, 3)) * np.sqrt(2 / (9 * Cin))).astype(np.float32)
+    x = rnd((N, Cin, H, W), Cin + H)
+    b = (rng.standard_normal(Cout) * 0.1).astype(np.float32)
+    y, layer = run_gpu(Wt, x, b, keep, stride, guard=64, ws=ws)
+    if ws:
+        assert layer.plan(x.shape, layer.workspace_bytes(x.shape))["splits"] >= 1
+    ref, den = oracle(Wt, x, b, keep, stride)
+    err = OC.max_norm_err(y, ref, den)
+    assert err <= TOL[torch.float32], f"normalised error {err:.3e}"
+
+
 @pytest.mark.parametrize("stride", [1, 2])
 def test_fp16_io(stride):
     rng = np.random.default_rng(5)
