@@ -149,6 +149,50 @@ def blas_threads():
     return len(os.sched_getaffinity(0))
 
 
+def set_blas_threads(n):
+    """Set OpenBLAS's thread count (numpy's BLAS, found as in blas_threads); False if not found."""
+    try:
+        with open("/proc/self/maps") as f:
+            libs = {l.split()[-1] for l in f if "openblas" in l.lower() and l.split()[-1].startswith("/")}
+        for path in libs:
+            lib = ctypes.CDLL(path)
+            for fn in ("openblas_set_num_threads", "openblas_set_num_threads64_",
+                       "scipy_openblas_set_num_threads", "scipy_openblas_set_num_threads64_"):
+                if hasattr(lib, fn):
+                    getattr(lib, fn)(int(n))
+                    return True
+    except Exception:
+        pass
+    return False
+
+
+def oracle_single_layer(budget_s=10.0):
+    """The float64 oracle on the 64->64 32x32 N=1 layer, timed on all BLAS threads and on one:
+    [{"threads": t, "ms": median ms}, ...] (projection outside the timed region)."""
+    import numpy as np
+    from oracle import conv as OC
+    from oracle import patterns as OP
+    from oracle import project as OPR
+    from paper_2003_06513_gb300 import workloads as WL
+    L = WL.single_layer()
+    Wh = OPR.project(WL.weights(L), OP.default8(), L.keep)["W_hat"]
+    b = WL.bias(L).astype(np.float64)
+    x = WL.layer_input(L, 1).astype(np.float64)
+    full = blas_threads()
+    rows = []
+    for t in (full, 1):
+        if t == 1 and not set_blas_threads(1):
+            break
+        times, t0 = [], time.perf_counter()
+        while len(times) < 30 and (time.perf_counter() - t0 < budget_s or len(times) < 3):
+            s0 = time.perf_counter()
+            OC.conv_ref(x, Wh, b, 1, True)
+            times.append(time.perf_counter() - s0)
+        rows.append({"threads": blas_threads(), "ms": 1e3 * statistics.median(times), "runs": len(times)})
+    set_blas_threads(full)
+    return rows
+
+
 def oracle_setup(max_images=8):
     """Projected weights of the 13 layers (outside any timed region) and the sample images."""
     from oracle import patterns as OP
@@ -525,14 +569,14 @@ def _peaks(dev):
     return peak, hbm, kind, f"{props.multi_processor_count} SMs x 128 FP32 lanes x 2 x {mhz:.0f} MHz"
 
 
-def _time_layer(lay, x, b, relu, ws, K):
+def _time_layer(lay, x, b, relu, ws, K, warmup=3):
     """ms of one layer: the smaller of the median of K stream launches (CUDA events around each
-    call, after 3 warm-ups) and the mean of K back-to-back replays of the call captured in a CUDA
-    graph (no per-launch host work, which small layers otherwise wait on).  Returns
-    (ms, eager_ms, graph_ms)."""
+    call, after `warmup` warm-up calls) and the mean of K back-to-back replays of the call
+    captured in a CUDA graph (after `warmup` replays; no per-launch host work, which small layers
+    otherwise wait on).  Returns (ms, eager_ms, graph_ms)."""
     import torch
     y = lay.conv(x, b, relu, workspace=ws)
-    for _ in range(2):
+    for _ in range(warmup - 1):
         lay.conv(x, b, relu, y, workspace=ws)
     torch.cuda.synchronize()
     st = torch.cuda.current_stream()
@@ -546,7 +590,7 @@ def _time_layer(lay, x, b, relu, ws, K):
     graph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(graph):
         lay.conv(x, b, relu, y, workspace=ws)
-    for _ in range(3):
+    for _ in range(warmup):
         graph.replay()
     torch.cuda.synchronize()
     g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -575,7 +619,7 @@ def layer_suite(args):
         layers, batch, dt = WL.mobilenet_v2_dw(), 128, "f16"
     tdt, ndt, es = (torch.float16, np.float16, 2) if dt == "f16" else (torch.float32, np.float32, 4)
     peak, hbm, hbm_kind, basis = _peaks(0)
-    K = max(args.steps, 5)
+    K = max(args.steps, 30)
     rows, tot_ms, tot_roof, tot_flops = [], 0.0, 0.0, 0.0
     with ClockSampler(0) as clk:
         for L in layers:
@@ -585,7 +629,7 @@ def layer_suite(args):
             b = torch.from_numpy(WL.bias(L)).cuda()
             nb = lay.workspace_bytes(x.shape)
             ws = torch.empty(max(nb // 4, 1), device="cuda") if nb else None
-            ms, ms_eager, ms_graph = _time_layer(lay, x, b, True, ws, K)
+            ms, ms_eager, ms_graph = _time_layer(lay, x, b, True, ws, K, warmup=10)
             G = (L.cout + 7) // 8
             fl, by = conv_cost(lay.beta, L.cin, L.cout, L.h, L.w, L.ho, L.wo, batch, G, es, L.cin_g)
             roof = max(fl / peak, by / hbm) * 1e3
@@ -606,6 +650,12 @@ def layer_suite(args):
                          "hbm_gbs": hbm / 1e9, "hbm_kind": hbm_kind,
                          "note": "time-weighted: sum of per-layer roofline times / sum of measured times"},
             "per_layer": rows, "clocks": clk.summary()}
+    if which == "single" and not args.no_cpu_baseline:
+        orc = oracle_single_layer()
+        line["cpu_baseline"] = {"value": tot_flops / (orc[0]["ms"] * 1e-3) / 1e9, "unit": "GFLOP/s",
+                                "cores": orc[0]["threads"], "kind": "oracle",
+                                "sample": "the whole layer, median of up to 30 runs (numpy float64)",
+                                "rows": orc}
     print(json.dumps(line), flush=True)
 
 
