@@ -315,6 +315,23 @@ def traffic_record():
     return None
 
 
+def max_over_ranks(dist, values, device):
+    """Each of ``values`` (times measured on this rank) replaced by its maximum over the ranks of
+    the process group (the slowest rank sets the job's time); unchanged without a group."""
+    import torch
+    if dist is None:
+        return [float(v) for v in values]
+    t = torch.tensor([float(v) for v in values], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t.tolist()]
+
+
+def job_images_per_s(world, ms_per_step):
+    """Whole-job throughput: every rank pushes its own batch of BATCH images per step (weak
+    scaling), and the step takes the slowest rank's time."""
+    return world * BATCH / (ms_per_step * 1e-3)
+
+
 def our_arm(args, rank, world, local_rank):
     import numpy as np
     import torch
@@ -468,10 +485,7 @@ def our_arm(args, rank, world, local_rank):
     barrier()
     e2e_ms = e0.elapsed_time(e1) / Ke
 
-    t = torch.tensor([elapsed_ms, e2e_ms, graph_ms], device=dev, dtype=torch.float64)
-    if dist is not None:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    elapsed_ms, e2e_ms, graph_ms = float(t[0]), float(t[1]), float(t[2])
+    elapsed_ms, e2e_ms, graph_ms = max_over_ranks(dist, [elapsed_ms, e2e_ms, graph_ms], dev)
 
     if rank == 0:
         props = torch.cuda.get_device_properties(dev)
@@ -486,7 +500,7 @@ def our_arm(args, rank, world, local_rank):
         roof_ms = sum(max(f / peak, b / hbm) for f, b in zip(flops, bytes_)) * 1e3
         eager_ms = elapsed_ms / K
         ms_step = min(eager_ms, graph_ms)      # the faster of stream launches and graph replay
-        img_s = world * BATCH / (ms_step * 1e-3)
+        img_s = job_images_per_s(world, ms_step)
         trec = traffic_record()
         line = {
             "metric": METRIC, "value": img_s, "unit": "img/s", "n_gpus": world, "steps": K,
