@@ -103,7 +103,8 @@ struct TmParams {
     int KS, c_split;                   // input-channel splits; channels per split (multiple of CK)
     float* ws;                         // KS > 1: fp32 partial sums [KS][N][Cout][Ho][Wo]
     size_t ws_stride;                  // elements per split
-    int IH, BWb;                       // staged rows / row width (floats) per (image, channel)
+    int IH, BWb;                       // staged rows / row width (elements) per (image, channel)
+    int ixa;                           // stage origin column: a multiple of ixa (16 bytes of input)
     int use_tma, vec_store;
     int pool, vec_pool;                // fused 2x2/2 max-pool of the output; pair stores of it
     unsigned tma_bytes;                // bytes one TMA box delivers
@@ -173,10 +174,10 @@ __device__ __forceinline__ void tmem_zero16(uint32_t ta) {
 }
 
 // Fallback input staging when no TMA descriptor applies (row pitch not a multiple of 16 bytes,
-// or fp16 input widened to fp32 on the way): thread tid copies elements tid, tid + 512, ... of the
+// the stage holds the input's own type): thread tid copies elements tid, tid + 512, ... of the
 // in-image part of the tile; everything else in the stage keeps the zero written at kernel start.
 template <typename TIn>
-__device__ __forceinline__ void stage_input_share(const TmParams& p, float* s_in, int c0, int ckv, int n0,
+__device__ __forceinline__ void stage_input_share(const TmParams& p, TIn* s_in, int c0, int ckv, int n0,
                                                   int iy0, int ix0, int tid) {
     const TIn* x = static_cast<const TIn*>(p.x);
     const int ry0 = max(0, iy0), ry1 = min(p.H, iy0 + p.IH);
@@ -184,9 +185,11 @@ __device__ __forceinline__ void stage_input_share(const TmParams& p, float* s_in
     const int nr = ry1 - ry0, nc = rx1 - rx0;
     if (nr <= 0 || nc <= 0) return;
     const int nimg = min(p.NB, p.N - n0);
-    // fp32 rows whose global start and length are even go as 8-byte pairs; the staged column of
-    // image column ix is ix - ix0 with ix0 a multiple of 4, so the shared side is 8-byte aligned too
-    const bool pairs = sizeof(TIn) == 4 && (p.W % 2 == 0) && (rx0 % 2 == 0) && (nc % 2 == 0);
+    // rows whose global start and length are even go as pairs (8 bytes of fp32, 4 bytes of fp16,
+    // copied asynchronously); the staged column of image column ix is ix - ix0 with ix0 a
+    // multiple of 16 bytes, so the shared side is aligned too
+    const bool pairs = (p.W % 2 == 0) && (rx0 % 2 == 0) && (nc % 2 == 0) &&
+                       reinterpret_cast<uintptr_t>(x) % (2 * sizeof(TIn)) == 0;
     const int units = pairs ? nc / 2 : nc;                  // copy units per row
     // element e = ((img * ckv + cl) * nr + r) * units + u as digits (img, cl, r, u); adding the
     // thread count digit by digit needs at most one carry per digit
@@ -203,12 +206,13 @@ __device__ __forceinline__ void stage_input_share(const TmParams& p, float* s_in
     while (img < nimg) {
         const int iy = ry0 + r, ix = rx0 + (pairs ? 2 * u : u);
         const TIn* src = x + ((size_t)(n0 + img) * p.C + c0 + cl) * HW + (size_t)iy * p.W + ix;
-        float* dst = s_in + ((img * p.CK + cl) * p.IH + (iy - iy0)) * p.BWb + (ix - ix0);
+        TIn* dst = s_in + ((img * p.CK + cl) * p.IH + (iy - iy0)) * p.BWb + (ix - ix0);
         if constexpr (sizeof(TIn) == 4) {
             if (pairs) cp_async8(dst, src);
             else cp_async4(dst, src, true);
         } else {
-            *dst = to_f32<TIn>(*src);
+            if (pairs) cp_async4(dst, src, true);
+            else *dst = *src;
         }
         u += su;
         if (u >= units) { u -= units; ++r; }
@@ -247,7 +251,9 @@ __device__ __forceinline__ Unit unit_of(const TmParams& p, int u) {
     U.oy0 = ty * p.BY * 4;
     U.ox0 = tx * p.BX * 4;
     U.iy0 = U.oy0 * S - 1;          // stage origin: 1 halo row, 16-byte aligned column
-    U.ix0 = U.ox0 * S - 4;
+    // stage origin: the 16-byte boundary at or left of the tile's first input column ox0 * S - 1
+    const int m = (U.ox0 * S) % p.ixa;
+    U.ix0 = U.ox0 * S - (m == 0 ? p.ixa : m);
     U.g0 = fchunk * p.WG;
     return U;
 }
@@ -273,7 +279,7 @@ __device__ __forceinline__ void fill_share(const TmParams& p, const CUtensorMap*
         }
     }
     if (!p.use_tma)
-        stage_input_share<TIn>(p, reinterpret_cast<float*>(st), c0, ckv, U.n0, U.iy0, U.ix0, warp * 32 + lane);
+        stage_input_share<TIn>(p, reinterpret_cast<TIn*>(st), c0, ckv, U.n0, U.iy0, U.ix0, warp * 32 + lane);
     const int wg = warp / p.WS, ws = warp - wg * p.WS, g = U.g0 + wg;
     if (g < p.G) {
         uint64_t* sd = reinterpret_cast<uint64_t*>(st + p.desc_off) + wg * p.CK;
@@ -397,7 +403,10 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
         }
         by = rem / p.BX;
         bx = rem - by * p.BX;
-        in_off = active ? img * p.CK * plane + by * RY * S * p.BWb + bx * RX * S + 3 : 3;
+        // window column 0 (input column ox0 * S - 1 of the lane's block) sits at d in the stage
+        // row: 3 for fp32 stages, 3 or 7 for fp16 ones (their origin is 16 bytes = 8 columns)
+        const int d = CU.ox0 * S - 1 - CU.ix0;
+        in_off = active ? img * p.CK * plane + by * RY * S * p.BWb + bx * RX * S + d : d;
         // lanes whose left neighbour lane does not hold the block to their left (stride 2 takes
         // window column 0 from that neighbour)
         edge = (bx == 0 || lane == 0) ? 1u : 0u;
@@ -509,14 +518,19 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
         const Unit CU = s_units[ci];
         if (CU.g0 + wg < p.G) {
             const unsigned char* st = smem + p.stage_off + (size_t)s * p.stage_bytes;
-            const uint32_t win_addr = smem_u32(reinterpret_cast<const float*>(st) + in_off);
+            const uint32_t win_addr = smem_u32(reinterpret_cast<const TIn*>(st) + in_off);
             const uint32_t desc_addr = smem_u32(reinterpret_cast<const uint64_t*>(st + p.desc_off) + wg * p.CK);
             const uint32_t vals_addr = smem_u32(reinterpret_cast<const float4*>(st + p.vals_off) + wg * p.maxk);
             const int ckv = min(p.CK, CU.c_hi - CU.c_lo - ck * p.CK);
-            if constexpr (S == 1) {
-                PP_STAGE_KERNELS_S1(ckv, desc_addr, vals_addr, win_addr, 4 * p.BWb, 4 * plane, tw, edge);
+            constexpr int es = (int)sizeof(TIn);
+            if constexpr (S == 1 && es == 4) {
+                PP_STAGE_KERNELS_S1(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw, edge);
+            } else if constexpr (S == 1) {
+                PP_STAGE_KERNELS_S1_H(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw, edge);
+            } else if constexpr (es == 4) {
+                PP_STAGE_KERNELS_S2(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw, edge);
             } else {
-                PP_STAGE_KERNELS_S2(ckv, desc_addr, vals_addr, win_addr, 4 * p.BWb, 4 * plane, tw, edge);
+                PP_STAGE_KERNELS_S2_H(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw, edge);
             }
         }
         // release the stage, then take this warp's share of filling chunk q + kStages - 1 into the
@@ -1409,7 +1423,11 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
     p.BX = pl.tile.BX;
     p.NB = pl.tile.NB;
     p.IH = pl.tile.IH;
-    p.BWb = pl.tile.BWb;
+    const size_t es = sizeof(T);
+    // fp16 stages hold fp16 (widened as the window is loaded): half the bytes of the plan's fp32
+    // stage, with 8 more columns so that the origin can sit on an 8-column (16-byte) boundary
+    p.BWb = es == 4 ? pl.tile.BWb : (int)align_up((size_t)pl.tile.BWb + 8, 8);
+    p.ixa = (int)(16 / es);
     p.linear = pl.tile.linear;
     p.tiles_x = pl.tiles_x;
     p.tiles_y = pl.tiles_y;
@@ -1422,13 +1440,14 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
     p.ws = static_cast<float*>(ws);
     p.ws_stride = (size_t)N * L->cout * Ho * Wo;
     const int C = L->cin_g;
-    const size_t es = sizeof(T);
-    p.use_tma = es == 4 && (W * es) % 16 == 0 && reinterpret_cast<uintptr_t>(x) % 16 == 0 && encode_tiled() != nullptr;
+    p.use_tma = (W * es) % 16 == 0 && reinterpret_cast<uintptr_t>(x) % 16 == 0 && encode_tiled() != nullptr;
     p.kb_off = 64;
     p.stage_off = (unsigned)align_up(64 + pl.kb_bytes, 128);
-    p.stage_bytes = (unsigned)pl.stage_bytes;
-    p.desc_off = (unsigned)align_up((size_t)p.NB * p.CK * p.IH * p.BWb * 4, 128);
+    p.desc_off = (unsigned)align_up((size_t)p.NB * p.CK * p.IH * p.BWb * es, 128);
     p.vals_off = p.desc_off + (unsigned)align_up((size_t)p.WG * p.CK * 8, 16);
+    p.stage_bytes = (unsigned)align_up((size_t)p.vals_off + (size_t)p.WG * p.maxk * 16, 128);
+    const size_t smem = p.stage_off + (size_t)kStages * p.stage_bytes;   // the plan's for fp32
+    if (smem > pl.smem) return PP_ERR_SHAPE;
     p.vec_store = (Wo % 4 == 0) && (reinterpret_cast<uintptr_t>(y) % (4 * es)) == 0;
     p.pool = pool;
     p.vec_pool = ((Wo >> 1) % 2 == 0) && (reinterpret_cast<uintptr_t>(y) % (2 * es)) == 0;
@@ -1440,15 +1459,16 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
         const cuuint64_t strides[3] = {(cuuint64_t)W * es, (cuuint64_t)H * W * es, (cuuint64_t)C * H * W * es};
         const cuuint32_t box[4] = {(cuuint32_t)p.BWb, (cuuint32_t)p.IH, (cuuint32_t)p.CK, (cuuint32_t)p.NB};
         const cuuint32_t estr[4] = {1, 1, 1, 1};
-        const CUresult r = encode_tiled()(&tmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<void*>(x), dims,
+        const CUresult r = encode_tiled()(&tmap, es == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16,
+                                          4, const_cast<void*>(x), dims,
                                           strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
                                           CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
                                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         if (r != CUDA_SUCCESS) p.use_tma = 0;
-        p.tma_bytes = (unsigned)((size_t)p.BWb * p.IH * p.CK * p.NB * 4);
+        p.tma_bytes = (unsigned)((size_t)p.BWb * p.IH * p.CK * p.NB * es);
     }
     auto kern = pconv_tm<S, T>;
-    if (!allow_max_smem<S, T>(pl.smem)) return PP_ERR_CUDA;
+    if (!allow_max_smem<S, T>(smem)) return PP_ERR_CUDA;
     const long long units = pl.ctas * pl.KS;
     if (units > INT_MAX) return PP_ERR_SHAPE;
     p.n_units = (int)units;
@@ -1458,7 +1478,7 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
     const long long ctas = p.use_tma ? std::max<long long>(std::min<long long>(units, sm_count()),
                                                            (units + kMaxUnitsPerCta - 1) / kMaxUnitsPerCta)
                                      : units;
-    kern<<<(unsigned)ctas, kThreadsTM, pl.smem, st>>>(p, tmap);
+    kern<<<(unsigned)ctas, kThreadsTM, smem, st>>>(p, tmap);
     if (cudaGetLastError() != cudaSuccess) return PP_ERR_CUDA;
     if (pl.KS > 1) {
         const size_t total = p.ws_stride;

@@ -39,7 +39,7 @@ def taps(mask):
     return [t for t in range(9) if (mask >> t) & 1]
 
 
-def macro(S):
+def macro(S, half=False):
     RY = RX = 4
     WY, WX = (RY - 1) * S + 3, (RX - 1) * S + 3
     R = RY * RX
@@ -55,6 +55,9 @@ def macro(S):
          f".reg .f32 x<{WY * WX}>, a<{R}>, w<4>;"]
     if packed:   # window pairs (row r, columns 1-2 / 3-4), accumulator pairs, duplicated weights
         L.append(f".reg .b64 xq<{2 * WY}>, ap<{R // 2}>, wq<4>;")
+    if half:     # fp16 stage: 16-bit elements widened to fp32 as the window is loaded
+        L.append(".reg .b16 h<10>;")
+        L.append(".reg .b32 pA, pB, pC, pD;")
     L += [
          "mov.b32 cl, %0;",
          "mov.b32 da, %1;",
@@ -76,13 +79,35 @@ def macro(S):
     # a scalar load of column 0 meets an 8-way bank conflict; it is the left neighbour lane's
     # column 8 instead (a warp shuffle), and only lanes at the start of a tile row or of the warp
     # (%7 nonzero) load it from shared memory
+    def cvt_pair(p, a):                   # two packed halves to x{a}, x{a+1}
+        return [f"mov.b32 {{h0, h1}}, {p};", f"cvt.f32.f16 x{a}, h0;", f"cvt.f32.f16 x{a + 1}, h1;"]
     for r in range(WY):
         base = r * WX
+        if S == 2 and half:                  # columns 1-8 as two 8-byte loads of four halves
+            L.append(f"ld.shared.v2.b32 {{pA, pB}}, [rb{r}+2];")
+            L.append(f"ld.shared.v2.b32 {{pC, pD}}, [rb{r}+10];")
+            for i, pr in enumerate(("pA", "pB", "pC", "pD")):
+                L += cvt_pair(pr, base + 1 + 2 * i)
+            L.append(f"shfl.sync.up.b32 x{base}, x{base + 8}, 1, 0, -1;")
+            L.append(f"@EL ld.shared.b16 h2, [rb{r}];")
+            L.append(f"@EL cvt.f32.f16 x{base}, h2;")
+            continue
         if S == 2:
             L.append(f"ld.shared.v4.f32 {{x{base + 1}, x{base + 2}, x{base + 3}, x{base + 4}}}, [rb{r}+4];")
             L.append(f"ld.shared.v4.f32 {{x{base + 5}, x{base + 6}, x{base + 7}, x{base + 8}}}, [rb{r}+20];")
             L.append(f"shfl.sync.up.b32 x{base}, x{base + 8}, 1, 0, -1;")
             L.append(f"@EL ld.shared.f32 x{base}, [rb{r}];")
+            continue
+        if half:                             # column 0, columns 1-4 (one 8-byte load), column 5
+            L.append(f"ld.shared.b16 h2, [rb{r}];")
+            L.append(f"ld.shared.v2.b32 {{pA, pB}}, [rb{r}+2];")
+            L.append(f"ld.shared.b16 h3, [rb{r}+10];")
+            L.append(f"cvt.f32.f16 x{base}, h2;")
+            L += cvt_pair("pA", base + 1) + cvt_pair("pB", base + 3)
+            L.append(f"cvt.f32.f16 x{base + 5}, h3;")
+            if packed:
+                L.append(f"mov.b64 xq{2 * r}, {{x{base + 1}, x{base + 2}}};")
+                L.append(f"mov.b64 xq{2 * r + 1}, {{x{base + 3}, x{base + 4}}};")
             continue
         L.append(f"ld.shared.f32 x{base}, [rb{r}];")
         c = 1
@@ -156,8 +181,9 @@ def macro(S):
           "CD:",
           "}"]
     body = "\\n\\t".join(L)
-    return (f"// stride {S}: 4x4 outputs per lane, {WY}x{WX} input window\n"
-            f"#define PP_STAGE_KERNELS_S{S}(nch, desc_addr, vals_addr, win_addr, pitch_b, plane_b, tbase, edge) \\\n"
+    name = f"PP_STAGE_KERNELS_S{S}" + ("_H" if half else "")
+    return (f"// stride {S}{', fp16 stage' if half else ''}: 4x4 outputs per lane, {WY}x{WX} input window\n"
+            f"#define {name}(nch, desc_addr, vals_addr, win_addr, pitch_b, plane_b, tbase, edge) \\\n"
             f'    asm volatile("{body}" :: "r"(nch), "r"(desc_addr), "r"(vals_addr), "r"(win_addr), '
             f'"r"(pitch_b), "r"(plane_b), "r"(tbase), "r"(edge) : "memory")\n')
 
@@ -165,7 +191,8 @@ def macro(S):
 def main():
     text = ["// generated by gen_dispatch.py -- do not edit", "#pragma once", ""]
     for S in STRIDES:
-        text.append(macro(S))
+        for half in (False, True):
+            text.append(macro(S, half))
     with open(sys.argv[1], "w") as f:
         f.write("\n".join(text))
 

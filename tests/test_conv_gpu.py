@@ -116,6 +116,25 @@ def test_extreme_shapes(N, Cin, Cout, H, W, keep, stride, ws):
     assert err <= TOL[torch.float32], f"normalised error {err:.3e}"
 
 
+@pytest.mark.parametrize("dtype", [torch.float32, torch.float16])
+@pytest.mark.parametrize("stride", [1, 2])
+def test_input_one_element_off_alignment(dtype, stride):
+    """x one element past a 16-byte boundary (even rows): the copy fallback must not pair
+    elements across a misaligned address."""
+    rng = np.random.default_rng(41)
+    Wt = (rng.standard_normal((16, 12, 3, 3)) * np.sqrt(2 / 108)).astype(np.float32)
+    x = rnd((2, 12, 10, 16), 43, dtype=_np_dt(dtype))
+    b = (rng.standard_normal(16) * 0.1).astype(np.float32)
+    layer = api.pp_pack(Wt, None, 0.5, 1, stride).bind("cuda")
+    flat = torch.empty(x.size + 1, dtype=dtype, device="cuda")
+    xt = flat[1:].view(x.shape)
+    xt.copy_(torch.from_numpy(x))
+    y = layer.conv(xt, torch.from_numpy(b).cuda(), True)
+    ref, den = oracle(Wt, x, b, 0.5, stride)
+    err = OC.max_norm_err(y.double().cpu().numpy(), ref, den)
+    assert err <= TOL[dtype], f"normalised error {err:.3e}"
+
+
 @pytest.mark.parametrize("stride", [1, 2])
 def test_fp16_io(stride):
     rng = np.random.default_rng(5)
