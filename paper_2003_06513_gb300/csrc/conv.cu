@@ -782,8 +782,9 @@ __global__ void __launch_bounds__(kDwThreads) pconv_depthwise(const __grid_const
 // contiguous run of memory: npl consecutive channels of one image as whole planes, or one
 // channel's band of output rows (npl == 1).  A persistent CTA copies its next tile into shared
 // memory with 16-byte cp.async (at the run's own alignment phase) while it computes the current
-// one, keeping HBM busy whatever the row width; the slot of every channel comes from an inverse
-// of the filter permutation built once per CTA.
+// one, keeping HBM busy whatever the row width.  Each CTA first decodes the kept weights, bias
+// and tap mask of every channel into a shared table (6 words a channel).  Planes whose output rows
+// are 7, 14 or 28 wide are computed one whole output row per item (RW below).
 struct DwStagedParams {
     const void* x;
     void* y;
@@ -798,26 +799,43 @@ struct DwStagedParams {
     int n_tiles;
     long long total_in;           // elements of x
     int buf_elems;                // elements per staging buffer
-    unsigned off_w, off_buf;      // shared-memory layout: inverse permutation | taps | 2 buffers
+    unsigned off_w, off_buf;      // shared-memory layout: taps of every channel | 2 buffers
     uint16_t masks[kMaxPatterns];
 };
 
-template <int S, typename T, bool VIN, bool VOUT>
+// RW > 0: every plane of a tile is whole and its output rows are RW wide (input rows W = RW for
+// stride 1, 2 * RW for stride 2); an item is then one whole output row, read from the staged
+// rows with the padding columns as zeros and no bounds test per element, in pairs where the rows
+// start on an even element.
+template <typename T>
+__device__ __forceinline__ void dw_row_load(const T* row, float* r, int W, bool pairs) {
+    if (pairs) {
+        for (int k = 0; k < W; k += 2) {
+            if constexpr (sizeof(T) == 2) {
+                const float2 f = __half22float2(*reinterpret_cast<const __half2*>(row + k));
+                r[k] = f.x;
+                r[k + 1] = f.y;
+            } else {
+                const float2 f = *reinterpret_cast<const float2*>(row + k);
+                r[k] = f.x;
+                r[k + 1] = f.y;
+            }
+        }
+    } else {
+        for (int k = 0; k < W; ++k) r[k] = to_f32<T>(row[k]);
+    }
+}
+
+template <int S, typename T, bool VIN, bool VOUT, int RW>
 __global__ void __launch_bounds__(kDwThreads) pconv_depthwise_staged(const __grid_constant__ DwStagedParams p) {
     constexpr int VE = 16 / (int)sizeof(T);      // elements per 16-byte copy
     constexpr int NIN = (kDwVW - 1) * S + 3;
     extern __shared__ __align__(16) unsigned char dsm[];
-    int* s_inv = reinterpret_cast<int*>(dsm);
-    float* s_w = reinterpret_cast<float*>(dsm + p.off_w);
+    float* s_w = reinterpret_cast<float*>(dsm + p.off_w);   // [C][6]: four kept weights, bias, mask
     T* bufs = reinterpret_cast<T*>(dsm + p.off_buf);
     const T* x = static_cast<const T*>(p.x);
     T* y = static_cast<T*>(p.y);
     const int tid = threadIdx.x;
-
-    for (int s = tid; s < p.NS; s += kDwThreads) {
-        const uint32_t co = p.perm[s];
-        if (co != kPadSlot) s_inv[co] = s;
-    }
 
     struct Tile {
         int n, c0, np, oy0, nro, iy_lo, nri;
@@ -856,10 +874,12 @@ __global__ void __launch_bounds__(kDwThreads) pconv_depthwise_staged(const __gri
             }
         }
     };
-    // thread t < np: taps and bias of the tile's channel c0 + t
-    auto decode = [&](const Tile& u) {
-        if (tid < u.np) {
-            const int s = s_inv[u.c0 + tid];
+    // kept weights, bias and tap mask of every channel, once per CTA: the thread of slot s decodes
+    // its kernel (a pruned one has no entry: mask 0, the output is the bias)
+    auto decode_all = [&]() {
+        for (int s = tid; s < p.NS; s += kDwThreads) {
+            const uint32_t co = p.perm[s];
+            if (co == kPadSlot) continue;
             const int g = s >> 3, f = s & 7;
             const uint64_t d = p.desc[g];
             const int cnt = (int)(d & 15u);
@@ -870,17 +890,74 @@ __global__ void __launch_bounds__(kDwThreads) pconv_depthwise_staged(const __gri
                 if ((code >> 3) == f) { pat = code & 7; k0 += j; }
             }
             const float4 v = pat >= 0 ? p.vals[k0] : make_float4(0.f, 0.f, 0.f, 0.f);
-            const unsigned m = pat >= 0 ? p.masks[pat] : 0u;
-            int k = 0;
+            float* w = s_w + co * 6;
+            w[0] = v.x;
+            w[1] = v.y;
+            w[2] = v.z;
+            w[3] = v.w;
+            w[4] = p.bias ? p.bias[co] : 0.0f;
+            w[5] = __uint_as_float(pat >= 0 ? p.masks[pat] : 0u);
+        }
+    };
+    // nine taps of channel c (zeros at the pruned ones), its bias and mask
+    auto taps_of = [&](int c, float (&w9)[9], float& bias, unsigned& m) {
+        const float* w = s_w + c * 6;
+        m = __float_as_uint(w[5]);
+        bias = w[4];
+        int k = 0;
 #pragma unroll
-            for (int t = 0; t < 9; ++t) {
-                const bool on = (m >> t) & 1u;
-                const float vk = k == 0 ? v.x : k == 1 ? v.y : k == 2 ? v.z : v.w;
-                s_w[tid * 11 + t] = on ? vk : 0.0f;
-                k += on ? 1 : 0;
+        for (int t = 0; t < 9; ++t) {
+            const bool on = (m >> t) & 1u;
+            const float vk = w[k < 3 ? k : 3];
+            w9[t] = on ? vk : 0.0f;
+            k += on ? 1 : 0;
+        }
+    };
+    auto compute_rows = [&](const Tile& u, int b) {   // RW > 0: one whole output row per item
+        constexpr int RWO = RW > 0 ? RW : 2;             // (the RW = 0 instance never calls this)
+        constexpr int RIN = (RWO - 1) * S + 3;           // input columns -1 .. (RW - 1) * S + 1
+        constexpr int WI = S * RWO;                      // staged row width
+        const T* buf = bufs + (size_t)b * p.buf_elems;
+        const int off0 = (int)(u.g0 - (u.g0 / VE) * VE);
+        const bool pairs = WI % 2 == 0 && off0 % 2 == 0;
+        const bool opairs = RWO % 2 == 0 && reinterpret_cast<uintptr_t>(y) % (2 * sizeof(T)) == 0;
+        const int items = u.np * u.nro;
+        for (int it = tid; it < items; it += kDwThreads) {
+            const int pl = it / u.nro, oyl = it - pl * u.nro;
+            float w9[9], bv;
+            unsigned mk;
+            taps_of(u.c0 + pl, w9, bv, mk);
+            const int oy = u.oy0 + oyl;
+            float acc[RWO];
+#pragma unroll
+            for (int j = 0; j < RWO; ++j) acc[j] = bv;
+#pragma unroll
+            for (int dy = 0; dy < 3; ++dy) {
+                const int iy = oy * S - 1 + dy;
+                if (iy < 0 || iy >= p.H) continue;
+                float r[RIN + 1];
+                r[0] = 0.0f;
+                r[RIN] = 0.0f;
+                r[RIN - 1] = 0.0f;                       // stride 1: column W
+                dw_row_load<T>(buf + off0 + (pl * u.nri + iy - u.iy_lo) * WI, r + 1, WI, pairs);
+#pragma unroll
+                for (int dx = 0; dx < 3; ++dx)
+#pragma unroll
+                    for (int j = 0; j < RWO; ++j) acc[j] = fmaf(w9[3 * dy + dx], r[j * S + dx], acc[j]);
             }
-            s_w[tid * 11 + 9] = p.bias ? p.bias[u.c0 + tid] : 0.0f;
-            s_w[tid * 11 + 10] = __uint_as_float(m);
+            T* out = y + (((size_t)u.n * p.C + u.c0 + pl) * p.Ho + oy) * RWO;
+            if (opairs) {
+#pragma unroll
+                for (int j = 0; j < RWO; j += 2) {
+                    const float a0 = p.relu ? fmaxf(acc[j], 0.0f) : acc[j];
+                    const float a1 = p.relu ? fmaxf(acc[j + 1], 0.0f) : acc[j + 1];
+                    if constexpr (sizeof(T) == 2) *reinterpret_cast<__half2*>(out + j) = __floats2half2_rn(a0, a1);
+                    else *reinterpret_cast<float2*>(out + j) = make_float2(a0, a1);
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < RWO; ++j) out[j] = from_f32<T>(p.relu ? fmaxf(acc[j], 0.0f) : acc[j]);
+            }
         }
     };
     auto compute = [&](const Tile& u, int b) {
@@ -901,10 +978,7 @@ __global__ void __launch_bounds__(kDwThreads) pconv_depthwise_staged(const __gri
         for (int i = tid; i < items; i += kDwThreads) {
             if (pl != cur) {
                 cur = pl;
-#pragma unroll
-                for (int t = 0; t < 9; ++t) w9[t] = s_w[pl * 11 + t];
-                bv = s_w[pl * 11 + 9];
-                m = __float_as_uint(s_w[pl * 11 + 10]);
+                taps_of(u.c0 + pl, w9, bv, m);
             }
             const int oy = u.oy0 + oyl;
             const int c0 = kDwVW * gx, ic = c0 * S - 1;
@@ -971,17 +1045,17 @@ __global__ void __launch_bounds__(kDwThreads) pconv_depthwise_staged(const __gri
     int t = blockIdx.x;
     if (t < p.n_tiles) load(tile_of(t), 0);
     asm volatile("cp.async.commit_group;" ::: "memory");
-    __syncthreads();                                   // s_inv complete
+    decode_all();                                      // overlaps the first tile's copy
     for (int k = 0; t < p.n_tiles; ++k, t += gridDim.x) {
         const Tile u = tile_of(t);
         const int tn = t + (int)gridDim.x;
         if (tn < p.n_tiles) load(tile_of(tn), (k + 1) & 1);
         asm volatile("cp.async.commit_group;" ::: "memory");
-        decode(u);
         asm volatile("cp.async.wait_group 1;" ::: "memory");
-        __syncthreads();                               // tile t staged, its taps decoded
-        compute(u, k & 1);
-        __syncthreads();                               // buffer k & 1 and the taps free again
+        __syncthreads();                               // tile t staged (and, at k = 0, the taps)
+        if constexpr (RW > 0) compute_rows(u, k & 1);
+        else compute(u, k & 1);
+        __syncthreads();                               // buffer k & 1 free again
     }
     asm volatile("cp.async.wait_all;" ::: "memory");
 }
@@ -1503,7 +1577,7 @@ int launch_depthwise_s(const DwParams& p, unsigned ctas, bool vin, bool vout, cu
     return cudaGetLastError() == cudaSuccess ? PP_OK : PP_ERR_CUDA;
 }
 
-template <int S, typename T, bool VIN, bool VOUT>
+template <int S, typename T, bool VIN, bool VOUT, int RW>
 bool dw_staged_smem(size_t need) {
     static std::atomic<int> done[64];
     int dev = 0;
@@ -1512,27 +1586,33 @@ bool dw_staged_smem(size_t need) {
     int optin = 0;
     if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess) return false;
     if ((size_t)optin < need) return false;
-    if (cudaFuncSetAttribute(pconv_depthwise_staged<S, T, VIN, VOUT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if (cudaFuncSetAttribute(pconv_depthwise_staged<S, T, VIN, VOUT, RW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              optin) != cudaSuccess)
         return false;
     done[dev].store(1, std::memory_order_release);
     return true;
 }
 
-template <int S, typename T, bool VIN, bool VOUT>
+template <int S, typename T, bool VIN, bool VOUT, int RW = 0>
 int launch_dw_staged(const DwStagedParams& p, size_t smem, cudaStream_t st) {
-    if (!dw_staged_smem<S, T, VIN, VOUT>(smem)) return PP_ERR_CUDA;
+    if (!dw_staged_smem<S, T, VIN, VOUT, RW>(smem)) return PP_ERR_CUDA;
     int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, pconv_depthwise_staged<S, T, VIN, VOUT>, kDwThreads,
-                                                      smem) != cudaSuccess || per_sm < 1)
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, pconv_depthwise_staged<S, T, VIN, VOUT, RW>,
+                                                      kDwThreads, smem) != cudaSuccess || per_sm < 1)
         return PP_ERR_CUDA;
     const long long ctas = std::min<long long>(p.n_tiles, (long long)sm_count() * per_sm);
-    pconv_depthwise_staged<S, T, VIN, VOUT><<<(unsigned)ctas, kDwThreads, smem, st>>>(p);
+    pconv_depthwise_staged<S, T, VIN, VOUT, RW><<<(unsigned)ctas, kDwThreads, smem, st>>>(p);
     return cudaGetLastError() == cudaSuccess ? PP_OK : PP_ERR_CUDA;
 }
 
 template <int S, typename T>
 int launch_dw_staged_s(const DwStagedParams& p, size_t smem, bool vin, bool vout, cudaStream_t st) {
+    // whole planes whose output rows are 7, 14 or 28 wide: the row-item kernel
+    if (p.n_bands == 1 && p.W == S * p.Wo) {
+        if (p.Wo == 28) return launch_dw_staged<S, T, false, false, 28>(p, smem, st);
+        if (p.Wo == 14) return launch_dw_staged<S, T, false, false, 14>(p, smem, st);
+        if (p.Wo == 7) return launch_dw_staged<S, T, false, false, 7>(p, smem, st);
+    }
     if (vin && vout) return launch_dw_staged<S, T, true, true>(p, smem, st);
     if (vin) return launch_dw_staged<S, T, true, false>(p, smem, st);
     if (vout) return launch_dw_staged<S, T, false, true>(p, smem, st);
@@ -1542,7 +1622,8 @@ int launch_dw_staged_s(const DwStagedParams& p, size_t smem, bool vin, bool vout
 constexpr size_t kDwStageBytes = 16384;   // one staging buffer of the staged depthwise kernel
 
 // Tile shape and shared-memory layout of the staged depthwise kernel; false when it does not
-// apply (x not 16-byte aligned, a plane row wider than a buffer, too many channels to invert).
+// apply (x not 16-byte aligned, a plane row wider than a buffer, more channels than the per-CTA
+// tap table holds).
 template <typename T>
 bool dw_staged_plan(const pp_layer* L, const void* x, int N, int H, int W, int Ho, DwStagedParams* p,
                     size_t* smem) {
@@ -1550,7 +1631,7 @@ bool dw_staged_plan(const pp_layer* L, const void* x, int N, int H, int W, int H
     const long long es = sizeof(T), VE = 16 / es;
     const long long budget = kDwStageBytes / es;
     // rows that are 16-byte aligned already load as vectors straight from global memory
-    if (reinterpret_cast<uintptr_t>(x) % 16 != 0 || ((size_t)W * es) % 16 == 0 || L->cout > 8192) return false;
+    if (reinterpret_cast<uintptr_t>(x) % 16 != 0 || ((size_t)W * es) % 16 == 0 || L->cout > 3072) return false;
     const long long plane = (long long)H * W;
     if (plane <= budget) {
         p->npl = (int)std::min<long long>({(long long)L->cout, budget / plane, (long long)kDwMaxPlanes});
@@ -1571,8 +1652,8 @@ bool dw_staged_plan(const pp_layer* L, const void* x, int N, int H, int W, int H
     const long long max_len = (long long)p->npl * max_rows * W;
     p->buf_elems = (int)((max_len + 2 * VE + VE - 1) / VE * VE);
     p->total_in = (long long)N * L->cout * H * W;
-    p->off_w = (unsigned)align_up((size_t)L->cout * 4, 16);
-    p->off_buf = (unsigned)align_up(p->off_w + (size_t)kDwMaxPlanes * 11 * 4, 16);
+    p->off_w = 0;
+    p->off_buf = (unsigned)align_up((size_t)L->cout * 6 * 4, 16);
     *smem = p->off_buf + 2 * (size_t)p->buf_elems * es;
     return true;
 }
