@@ -1308,12 +1308,13 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
         long long waves = (pl->ctas * best_ks + sms - 1) / sms;
         double steps = (double)waves * (std::min(pl->c_split, C) + 2.0 * per + 2.0 * ck);
         // tiny launches (the SMs stay idle even with 8 splits): fewer channels per stage and up to
-        // 64 splits within one wave, chosen by estimated channel steps
+        // 32 splits within one wave (more cost more in partial sums than they save: measured on the
+        // 64->64 32x32 N=1 layer and the sweep's N=1 points), chosen by estimated channel steps
         if (pl->ctas * std::min(8, nck_total) < sms) {
             for (int ck2 = ck;; ck2 = std::max(1, ck2 / 2)) {
                 const int nck2 = (C + ck2 - 1) / ck2;
                 if (nck2 > kMaxChunks) break;
-                for (int ksp = 2; ksp <= std::min(64, nck2); ++ksp) {
+                for (int ksp = 2; ksp <= std::min(32, nck2); ++ksp) {
                     const int per2 = (nck2 + ksp - 1) / ksp;
                     if ((nck2 + per2 - 1) / per2 != ksp) continue;
                     if (ws_avail < (size_t)ksp * out_elems * 4 || pl->ctas * ksp > sms) break;   // one wave
