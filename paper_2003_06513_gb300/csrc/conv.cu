@@ -703,24 +703,77 @@ __global__ void __launch_bounds__(kDwThreads) pconv_depthwise(const __grid_const
     st -= s_pl * p.ipp;
     const int s_oy = st / p.NGX, s_gx = st - (st / p.NGX) * p.NGX;
 
+    // a thread's items stay on one plane for several steps: its taps and base pointers are
+    // reloaded only when the plane changes
+    int cur = -1, co = -1;
+    const T* xp = x;
+    T* yp = y;
+    float w9[9], b = 0.0f;
+    unsigned m = 0;
     for (int i = tid; i < count; i += kDwThreads) {
-        const int co = s_co[pl];
-        if (co >= 0) {
+        if (pl != cur) {
+            cur = pl;
+            co = s_co[pl];
             const int n = (int)((pl0 + pl) / p.NS);
-            const T* xp = x + ((size_t)n * p.C + co) * p.H * p.W;
-            T* yp = y + ((size_t)n * p.C + co) * p.Ho * p.Wo;
-            float w9[9];
+            xp = x + ((size_t)n * p.C + (co >= 0 ? co : 0)) * p.H * p.W;
+            yp = y + ((size_t)n * p.C + (co >= 0 ? co : 0)) * p.Ho * p.Wo;
 #pragma unroll
             for (int t = 0; t < 9; ++t) w9[t] = s_w[pl][t];
-            const float b = s_w[pl][9];
-            const unsigned m = __float_as_uint(s_w[pl][10]);
+            b = s_w[pl][9];
+            m = __float_as_uint(s_w[pl][10]);
+        }
+        if (co >= 0) {
             const int c0 = kDwVW * gx;            // first output column of this thread
             const int ic = c0 * S - 1;            // first input column it reads
             float acc[kDwVW];
 #pragma unroll
             for (int j = 0; j < kDwVW; ++j) acc[j] = b;
+            bool done = false;
+            if constexpr (VIN && sizeof(T) == 2) {
+                if (ic + 1 + kDwVW * S <= p.W) {
+                    // fp16 rows inside the image: the three rows' 16-byte groups and halo columns are
+                    // all requested before any is used (raw, 6 or 10 registers a row), then widened
+                    constexpr int NV = kDwVW * S / 8;      // 16-byte groups per row
+                    uint4 raw[3][NV];
+                    __half hl[3], hr[3];
 #pragma unroll
-            for (int dy = 0; dy < 3; ++dy) {
+                    for (int dy = 0; dy < 3; ++dy) {
+                        const int iy = min(max(oy * S - 1 + dy, 0), p.H - 1);
+                        const __half* row = reinterpret_cast<const __half*>(xp) + (size_t)iy * p.W;
+#pragma unroll
+                        for (int v = 0; v < NV; ++v) raw[dy][v] = *reinterpret_cast<const uint4*>(row + ic + 1 + 8 * v);
+                        hl[dy] = ic >= 0 ? row[ic] : __float2half(0.0f);
+                        hr[dy] = (S == 1 && ic + NIN - 1 < p.W) ? row[ic + NIN - 1] : __float2half(0.0f);
+                    }
+#pragma unroll
+                    for (int dy = 0; dy < 3; ++dy) {
+                        const int iy = oy * S - 1 + dy;
+                        if (iy < 0 || iy >= p.H) continue;
+                        float r[NIN];
+                        r[0] = __half2float(hl[dy]);
+#pragma unroll
+                        for (int v = 0; v < NV; ++v) {
+                            const __half2* h = reinterpret_cast<const __half2*>(&raw[dy][v]);
+#pragma unroll
+                            for (int k = 0; k < 4; ++k) {
+                                const float2 f = __half22float2(h[k]);
+                                r[1 + 8 * v + 2 * k] = f.x;
+                                r[2 + 8 * v + 2 * k] = f.y;
+                            }
+                        }
+                        if (S == 1) r[NIN - 1] = __half2float(hr[dy]);
+#pragma unroll
+                        for (int dx = 0; dx < 3; ++dx) {
+                            if (!((m >> (3 * dy + dx)) & 1u)) continue;   // pruned tap
+#pragma unroll
+                            for (int j = 0; j < kDwVW; ++j) acc[j] = fmaf(w9[3 * dy + dx], r[j * S + dx], acc[j]);
+                        }
+                    }
+                    done = true;
+                }
+            }
+#pragma unroll
+            for (int dy = 0; dy < 3 && !done; ++dy) {
                 const int iy = oy * S - 1 + dy;
                 if (iy < 0 || iy >= p.H) continue;
                 const T* row = xp + (size_t)iy * p.W;
