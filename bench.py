@@ -47,7 +47,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0, help="oracle sample budget")
     ap.add_argument("--profile-layer", type=int, default=None,
-                    help="run only VGG-16 layer IDX (0-based) --steps times at --batch (for ncu)")
+                    help="run only layer IDX (0-based) of VGG-16, or of --workload resnet50 / "
+                         "mobilenet, --steps times at --batch (for ncu)")
     ap.add_argument("--batch", type=int, default=BATCH, help="batch of --profile-layer")
     ap.add_argument("--workload", choices=["vgg16", "single", "resnet50", "mobilenet"], default="vgg16",
                     help="vgg16: the headline step; the others time each layer of that config alone "
@@ -718,13 +719,18 @@ def sweep_run(args):
 
 
 def profile_layer(args):
-    """One VGG-16 layer alone at a chosen batch, for profiler captures on small cases."""
+    """One layer alone at a chosen batch, for profiler captures on small cases: VGG-16 layer
+    IDX, or with --workload resnet50 / mobilenet that suite's layer IDX (MobileNet in fp16)."""
+    import numpy as np
     import torch
     from paper_2003_06513_gb300 import api
     from paper_2003_06513_gb300 import workloads as WL
-    L = WL.vgg16()[args.profile_layer]
-    lay = api.pp_pack(WL.weights(L), None, L.keep).bind("cuda")
-    x = torch.from_numpy(WL.layer_input(L, args.batch)).cuda()
+    layers = {"resnet50": WL.resnet50_3x3, "mobilenet": WL.mobilenet_v2_dw}.get(args.workload, WL.vgg16)()
+    L = layers[args.profile_layer]
+    lay = api.pp_pack(WL.weights(L), None, L.keep, groups=L.cout if L.depthwise else 1,
+                      stride=L.stride).bind("cuda")
+    ndt = np.float16 if args.workload == "mobilenet" else np.float32
+    x = torch.from_numpy(WL.layer_input(L, args.batch, relu=not L.depthwise, dtype=ndt)).cuda()
     b = torch.from_numpy(WL.bias(L)).cuda()
     ws_n = lay.workspace_bytes(x.shape)
     ws = torch.empty(max(ws_n // 4, 1), device="cuda") if ws_n else None
