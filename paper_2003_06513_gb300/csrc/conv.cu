@@ -879,7 +879,7 @@ __device__ __forceinline__ void dw_row_load(const T* row, float* r, int W, bool 
     }
 }
 
-template <int S, typename T, bool VIN, bool VOUT, int RW>
+template <int S, typename T, bool VIN, bool VOUT, int RW, int NH>
 __global__ void __launch_bounds__(kDwThreads) pconv_depthwise_staged(const __grid_constant__ DwStagedParams p) {
     constexpr int VE = 16 / (int)sizeof(T);      // elements per 16-byte copy
     constexpr int NIN = (kDwVW - 1) * S + 3;
@@ -966,17 +966,20 @@ __global__ void __launch_bounds__(kDwThreads) pconv_depthwise_staged(const __gri
             k += on ? 1 : 0;
         }
     };
-    auto compute_rows = [&](const Tile& u, int b) {   // RW > 0: one whole output row per item
+    auto compute_rows = [&](const Tile& u, int b) {   // RW > 0: an output row (or half of it) per item
         constexpr int RWO = RW > 0 ? RW : 2;             // (the RW = 0 instance never calls this)
-        constexpr int RIN = (RWO - 1) * S + 3;           // input columns -1 .. (RW - 1) * S + 1
-        constexpr int WI = S * RWO;                      // staged row width
+        constexpr int RIN = (RWO - 1) * S + 3;           // input columns -1 .. (RW - 1) * S + 1 of a piece
+        constexpr int nh = NH;                           // pieces per output row (2 for 28-wide rows)
+        constexpr int WI = RWO * S * NH;                 // staged row width (== p.W)
         const T* buf = bufs + (size_t)b * p.buf_elems;
         const int off0 = (int)(u.g0 - (u.g0 / VE) * VE);
-        const bool pairs = WI % 2 == 0 && off0 % 2 == 0;
+        const bool pairs = WI % 2 == 0 && off0 % 2 == 0 && (RWO * S) % 2 == 0;
         const bool opairs = RWO % 2 == 0 && reinterpret_cast<uintptr_t>(y) % (2 * sizeof(T)) == 0;
-        const int items = u.np * u.nro;
+        const int items = u.np * u.nro * nh;
         for (int it = tid; it < items; it += kDwThreads) {
-            const int pl = it / u.nro, oyl = it - pl * u.nro;
+            const int q = it / nh, h = it - q * nh;
+            const int pl = q / u.nro, oyl = q - pl * u.nro;
+            const int cb = h * RWO * S;                  // first input column of the piece
             float w9[9], bv;
             unsigned mk;
             taps_of(u.c0 + pl, w9, bv, mk);
@@ -988,17 +991,18 @@ __global__ void __launch_bounds__(kDwThreads) pconv_depthwise_staged(const __gri
             for (int dy = 0; dy < 3; ++dy) {
                 const int iy = oy * S - 1 + dy;
                 if (iy < 0 || iy >= p.H) continue;
+                const T* row = buf + off0 + (size_t)(pl * u.nri + iy - u.iy_lo) * WI;
                 float r[RIN + 1];
-                r[0] = 0.0f;
+                r[0] = cb > 0 ? to_f32<T>(row[cb - 1]) : 0.0f;
                 r[RIN] = 0.0f;
-                r[RIN - 1] = 0.0f;                       // stride 1: column W
-                dw_row_load<T>(buf + off0 + (pl * u.nri + iy - u.iy_lo) * WI, r + 1, WI, pairs);
+                if constexpr (S == 1) r[RIN - 1] = cb + RWO < WI ? to_f32<T>(row[cb + RWO]) : 0.0f;
+                dw_row_load<T>(row + cb, r + 1, RWO * S, pairs);
 #pragma unroll
                 for (int dx = 0; dx < 3; ++dx)
 #pragma unroll
                     for (int j = 0; j < RWO; ++j) acc[j] = fmaf(w9[3 * dy + dx], r[j * S + dx], acc[j]);
             }
-            T* out = y + (((size_t)u.n * p.C + u.c0 + pl) * p.Ho + oy) * RWO;
+            T* out = y + (((size_t)u.n * p.C + u.c0 + pl) * p.Ho + oy) * (RWO * NH) + h * RWO;
             if (opairs) {
 #pragma unroll
                 for (int j = 0; j < RWO; j += 2) {
@@ -1631,7 +1635,7 @@ int launch_depthwise_s(const DwParams& p, unsigned ctas, bool vin, bool vout, cu
     return cudaGetLastError() == cudaSuccess ? PP_OK : PP_ERR_CUDA;
 }
 
-template <int S, typename T, bool VIN, bool VOUT, int RW>
+template <int S, typename T, bool VIN, bool VOUT, int RW, int NH>
 bool dw_staged_smem(size_t need) {
     static std::atomic<int> done[64];
     int dev = 0;
@@ -1640,31 +1644,32 @@ bool dw_staged_smem(size_t need) {
     int optin = 0;
     if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess) return false;
     if ((size_t)optin < need) return false;
-    if (cudaFuncSetAttribute(pconv_depthwise_staged<S, T, VIN, VOUT, RW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if (cudaFuncSetAttribute(pconv_depthwise_staged<S, T, VIN, VOUT, RW, NH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              optin) != cudaSuccess)
         return false;
     done[dev].store(1, std::memory_order_release);
     return true;
 }
 
-template <int S, typename T, bool VIN, bool VOUT, int RW = 0>
+template <int S, typename T, bool VIN, bool VOUT, int RW = 0, int NH = 1>
 int launch_dw_staged(const DwStagedParams& p, size_t smem, cudaStream_t st) {
-    if (!dw_staged_smem<S, T, VIN, VOUT, RW>(smem)) return PP_ERR_CUDA;
+    if (!dw_staged_smem<S, T, VIN, VOUT, RW, NH>(smem)) return PP_ERR_CUDA;
     int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, pconv_depthwise_staged<S, T, VIN, VOUT, RW>,
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, pconv_depthwise_staged<S, T, VIN, VOUT, RW, NH>,
                                                       kDwThreads, smem) != cudaSuccess || per_sm < 1)
         return PP_ERR_CUDA;
     const long long ctas = std::min<long long>(p.n_tiles, (long long)sm_count() * per_sm);
-    pconv_depthwise_staged<S, T, VIN, VOUT, RW><<<(unsigned)ctas, kDwThreads, smem, st>>>(p);
+    pconv_depthwise_staged<S, T, VIN, VOUT, RW, NH><<<(unsigned)ctas, kDwThreads, smem, st>>>(p);
     return cudaGetLastError() == cudaSuccess ? PP_OK : PP_ERR_CUDA;
 }
 
 template <int S, typename T>
 int launch_dw_staged_s(const DwStagedParams& p, size_t smem, bool vin, bool vout, cudaStream_t st) {
-    // whole planes whose output rows are 7, 14 or 28 wide: the row-item kernel
+    // whole planes whose output rows are 7, 14 or 28 wide: the row-item kernel (28-wide rows in two
+    // 14-wide pieces, which keeps its registers low enough for four CTAs per SM)
     if (p.n_bands == 1 && p.W == S * p.Wo) {
-        if (p.Wo == 28) return launch_dw_staged<S, T, false, false, 28>(p, smem, st);
-        if (p.Wo == 14) return launch_dw_staged<S, T, false, false, 14>(p, smem, st);
+        if (p.Wo == 28) return launch_dw_staged<S, T, false, false, 14, 2>(p, smem, st);
+        if (p.Wo == 14) return launch_dw_staged<S, T, false, false, 14, 1>(p, smem, st);
         if (p.Wo == 7) return launch_dw_staged<S, T, false, false, 7>(p, smem, st);
     }
     if (vin && vout) return launch_dw_staged<S, T, true, true>(p, smem, st);
