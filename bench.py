@@ -436,6 +436,7 @@ def our_arm(args, rank, world, local_rank):
     dense = None
     if not args.no_dense_context:
         dense = dense_context(packed, biases, layers, x0, K, barrier)
+    b1_ms, b1_eager = batch1_context(packed, biases, layers, K, barrier, dev)
 
     # e2e: every step's input batch from pinned host memory and its final feature map back,
     # inside the timed region.  The copies run on a second stream, double-buffered, so that the
@@ -527,6 +528,9 @@ def our_arm(args, rank, world, local_rank):
             "gpu_launches": K * launches_per_step,
             "clocks": clocks,
         }
+        line["batch1"] = {"value": world * 1.0 / (b1_ms * 1e-3), "unit": "img/s", "ms_per_step": b1_ms,
+                          "eager_ms_per_step": b1_eager,
+                          "what": "the same 13 layers at batch 1 (latency; graph replay where faster)"}
         if dense is not None:
             line["cudnn_dense_context"] = {"value": world * BATCH / (dense * 1e-3), "unit": "img/s",
                                            "ms_per_step": dense,
@@ -540,6 +544,54 @@ def our_arm(args, rank, world, local_rank):
     if dist is not None:
         dist.barrier()
         dist.destroy_process_group()
+
+
+def batch1_context(packed, biases, layers, K, barrier, dev):
+    """ms per step of the same 13 layers at batch 1 (latency): the smaller of stream launches and
+    CUDA-graph replay, with the batch-1 plan's own workspace."""
+    import numpy as np
+    import torch
+    from paper_2003_06513_gb300 import api
+    from paper_2003_06513_gb300 import workloads as WL
+    x = torch.from_numpy(WL.vgg16_image(1)).to(dev)
+    shapes, in_shapes, h = [], [], 224
+    for L in layers:
+        in_shapes.append((1, L.cin, h, h))
+        h = h // 2 if L.pool_after else h
+        shapes.append((1, L.cout, h, h))
+    ws = api.workspace_for(packed, in_shapes, dev)
+    outs = [torch.empty(sh, dtype=torch.float32, device=dev) for sh in shapes]
+
+    def step():
+        cur = x
+        for L, lay, b, y in zip(layers, packed, biases, outs):
+            lay.conv(cur, b, True, y, torch.cuda.current_stream(dev), ws, pool2x2=L.pool_after)
+            cur = y
+
+    for _ in range(3):
+        step()
+    barrier()
+    st = torch.cuda.current_stream(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    Kb = max(10, K)
+    e0.record(st)
+    for _ in range(Kb):
+        step()
+    e1.record(st)
+    barrier()
+    eager = e0.elapsed_time(e1) / Kb
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        step()
+    for _ in range(3):
+        graph.replay()
+    barrier()
+    e0.record(st)
+    for _ in range(Kb):
+        graph.replay()
+    e1.record(st)
+    barrier()
+    return min(eager, e0.elapsed_time(e1) / Kb), eager
 
 
 def dense_context(packed, biases, layers, x0, K, barrier):
