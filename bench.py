@@ -528,6 +528,12 @@ def our_arm(args, rank, world, local_rank):
             "gpu_launches": K * launches_per_step,
             "clocks": clocks,
         }
+        line["paper_context"] = {
+            "note": "the paper's own numbers, for context only: relative speedups of its generated "
+                    "mobile code on ResNet-18 (6x compressed), no datacentre-GPU or absolute numbers (§5.3)",
+            "device": "Samsung Galaxy S10 (Snapdragon 855: Kryo 485 CPU, Adreno 640 GPU)",
+            "speedup_mobile_cpu": {"vs_tflite": 4.2, "vs_tvm": 2.3, "vs_mnn": 2.0},
+            "speedup_mobile_gpu": {"vs_tflite": 3.3, "vs_tvm": 2.5, "vs_mnn": 1.4}}
         line["batch1"] = {"value": world * 1.0 / (b1_ms * 1e-3), "unit": "img/s", "ms_per_step": b1_ms,
                           "eager_ms_per_step": b1_eager,
                           "what": "the same 13 layers at batch 1 (latency; graph replay where faster)"}
