@@ -1,13 +1,16 @@
 #!/usr/bin/env python3
 """Generate pattern_dispatch.h: the channel loop of the pattern-sparse kernel as inline PTX.
 
-One macro per stride processes one pipeline stage (CK input channels) for one filter group and
-one lane's 4x4 output block.  Per input channel:
+One macro per stride and stage type (fp32 stages; fp16 stages, whose window elements are widened
+to fp32 as they are loaded) processes one pipeline stage (CK input channels) for one filter
+group and one lane's 4x4 output block.  Per input channel:
 
     ld.shared        the group's 64-bit descriptor (count in bits 0-3, then 6-bit
                      (slot << 3 | pattern) codes of the kept kernels, slots ascending)
-    ld.shared        the lane's input window, (4-1)*S+3 rows of (4-1)*S+3 floats; row r starts at
-                     a register advanced by one channel plane per channel, columns are immediates
+    ld.shared        the lane's input window, (4-1)*S+3 rows of (4-1)*S+3 elements; row r starts
+                     at a register advanced by one channel plane per channel, columns are
+                     immediates; stride 2 takes column 0 from the left neighbour lane (a warp
+                     shuffle) where that lane holds the block to the left
     per kept kernel:
       ld.shared.v4   its four kept weights (consecutive in the compact storage, §3.4)
       tcgen05.ld     the 16 accumulators of its filter slot from tensor memory
@@ -24,7 +27,7 @@ that alignment and stay scalar.  Every pattern holds 1 to 3 centre-column taps, 
 of the body's instructions go away.
 
 Every branch is warp-uniform (bra.uni), so no convergence code surrounds the loop.  Taps are
-applied in ascending raster order for every output.  The library masks are the eight defaults
+applied in ascending raster order for every output.  The macros' operands are listed in macro().  The library masks are the eight defaults
 (centre + 3 of the 4 edge neighbours; centre + one edge + its 2 flanking corners).
 
 Usage: gen_dispatch.py OUT.h
@@ -46,7 +49,8 @@ def macro(S, half=False):
     acc = ", ".join(f"a{i}" for i in range(R))
     rows = ", ".join(f"rb{r}" for r in range(WY))
     # operands: %0 channels, %1 descriptor address, %2 weights address, %3 window address of
-    # channel 0, %4 row pitch in bytes, %5 channel plane in bytes, %6 tensor-memory base
+    # channel 0, %4 row pitch in bytes, %5 channel plane in bytes, %6 tensor-memory base, %7
+    # nonzero where the left neighbour lane does not hold the block to the left (stride 2)
     packed = S == 1
     L = ["{",
          ".reg .pred P, EL;",
