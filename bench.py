@@ -290,11 +290,16 @@ def hbm_peak():
 
 
 def kernel_sources_sha256():
-    """Hash of the kernel's sources: conv.cu and the generator of its channel loop."""
+    """Hash of the kernel's sources: conv.cu and the channel loop its generator emits."""
+    import importlib.util
+    csrc = os.path.join(ROOT, "paper_2003_06513_gb300", "csrc")
+    spec = importlib.util.spec_from_file_location("gen_dispatch", os.path.join(csrc, "gen_dispatch.py"))
+    gen = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(gen)
     h = hashlib.sha256()
-    for name in ("conv.cu", "gen_dispatch.py"):
-        with open(os.path.join(ROOT, "paper_2003_06513_gb300", "csrc", name), "rb") as f:
-            h.update(f.read())
+    with open(os.path.join(csrc, "conv.cu"), "rb") as f:
+        h.update(f.read())
+    h.update(gen.generate().encode())
     return h.hexdigest()
 
 

@@ -192,13 +192,18 @@ def macro(S, half=False):
             f'"r"(pitch_b), "r"(plane_b), "r"(tbase), "r"(edge) : "memory")\n')
 
 
-def main():
+def generate() -> str:
+    """The text of pattern_dispatch.h."""
     text = ["// generated by gen_dispatch.py -- do not edit", "#pragma once", ""]
     for S in STRIDES:
         for half in (False, True):
             text.append(macro(S, half))
+    return "\n".join(text)
+
+
+def main():
     with open(sys.argv[1], "w") as f:
-        f.write("\n".join(text))
+        f.write(generate())
 
 
 if __name__ == "__main__":
