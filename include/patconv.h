@@ -19,7 +19,12 @@
  *     caller; streams are passed as `void*` holding a cudaStream_t (NULL = legacy default);
  *   - taps are numbered in raster order t = 3*(dy+1) + (dx+1), dy, dx in {-1,0,1}; a pattern is
  *     a 9-bit mask with bit t set for each kept tap;
- *   - tensors are contiguous NCHW; weights are host fp32 [Cout][Cin/groups][3][3].
+ *   - tensors are contiguous NCHW; weights are host fp32 [Cout][Cin/groups][3][3];
+ *   - kernels are launched with programmatic dependent launch on a stream that is not being
+ *     captured into a CUDA graph: a convolution may start its set-up while the kernel before it
+ *     on the stream finishes, and reads or writes no activation before that kernel has completed,
+ *     so stream order holds as for a plain launch.  The environment variable PATCONV_PDL=0
+ *     (read once) makes every launch a plain one.
  *
  * Thread safety: a handle is immutable after pp_pack/pp_bind_device, so pp_conv on one handle
  * may be called from several host threads and streams at once.

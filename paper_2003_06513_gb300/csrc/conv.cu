@@ -24,6 +24,7 @@
 #include <algorithm>
 #include <atomic>
 #include <climits>
+#include <cstdlib>
 #include <cstdint>
 #include <cstring>
 #include <map>
@@ -40,6 +41,15 @@ using namespace patconv;
 namespace {
 
 // ------------------------------------------------------------------------------ helpers
+
+// Programmatic dependent launch.  Every kernel of the library lets the next kernel of its stream
+// start (launch_dependents: at once, or for the pattern-sparse kernel at its last epilogue) and
+// waits for the previous one (wait: that grid has completed and its memory is visible) before it
+// reads or writes activations, so one layer's launch and set-up (tensor-memory allocation,
+// barriers, tables) overlap the previous layer's tail.  Both are no-ops for a launch without the
+// programmatic-serialisation attribute.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
 __device__ __forceinline__ void cp_async4(void* smem, const void* gmem, bool valid) {
     const unsigned s = (unsigned)__cvta_generic_to_shared(smem);
@@ -335,6 +345,7 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     const uint32_t tbase = *s_tmem;
     int Q = 0;
     for (int i = 0; i < n_my; ++i) Q += s_units[i].nck;
+    pdl_wait();   // the previous kernel's output (this input) is complete from here on
 
     const int wg = warp / p.WS, ws = warp - (warp / p.WS) * p.WS;
     // fill cursor: unit fi (of this CTA), its chunk fk, and the warp's group's weight range for
@@ -545,6 +556,7 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
             if (threadIdx.x == 0) *s_issued = j + 1;
         }
         if (++ck == CU.nck) {   // unit done: results out, accumulators zeroed, next unit's tile
+            if (q == Q - 1) pdl_trigger();   // the next kernel may start its set-up from here on
             epilogue(CU);
             ck = 0;
             if (++ci < n_my) place_lane();
@@ -631,6 +643,8 @@ __device__ __forceinline__ void ld_vec(const __half* src, float* dst) {
 
 template <int S, typename T, bool VIN, bool VOUT>
 __global__ void __launch_bounds__(kDwThreads) pconv_depthwise(const __grid_constant__ DwParams p) {
+    pdl_trigger();
+    pdl_wait();
     constexpr int NIN = (kDwVW - 1) * S + 3;     // input columns one thread reads per row
     const T* x = static_cast<const T*>(p.x);
     T* y = static_cast<T*>(p.y);
@@ -881,6 +895,8 @@ __device__ __forceinline__ void dw_row_load(const T* row, float* r, int W, bool 
 
 template <int S, typename T, bool VIN, bool VOUT, int RW, int NH>
 __global__ void __launch_bounds__(kDwThreads) pconv_depthwise_staged(const __grid_constant__ DwStagedParams p) {
+    pdl_trigger();
+    pdl_wait();
     constexpr int VE = 16 / (int)sizeof(T);      // elements per 16-byte copy
     constexpr int NIN = (kDwVW - 1) * S + 3;
     extern __shared__ __align__(16) unsigned char dsm[];
@@ -1208,6 +1224,39 @@ int sm_count() {
     return n;
 }
 
+// Kernel launch with programmatic stream serialisation (pdl_wait / pdl_trigger) on a stream that
+// is not being captured, unless the environment sets PATCONV_PDL=0; returns the launch's error,
+// which it also clears.  In a CUDA graph the kernel nodes already follow each other without host
+// work, and programmatic edges there measured slower (VGG-16 at batch 1: 0.477 against 0.464 ms
+// per image), so a captured launch is a plain one.
+bool pdl_enabled() {
+    static const bool on = [] {
+        const char* e = std::getenv("PATCONV_PDL");
+        return !(e && e[0] == '0');
+    }();
+    return on;
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch(void (*kern)(KArgs...), unsigned grid, unsigned block, size_t smem, cudaStream_t st,
+                   const Args&... args) {
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(block);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    const bool captured = cudaStreamIsCapturing(st, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone;
+    cfg.numAttrs = pdl_enabled() && !captured ? 1 : 0;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, args...);
+    const cudaError_t l = cudaGetLastError();
+    return e != cudaSuccess ? e : l;
+}
+
 using EncodeTiledFn = PFN_cuTensorMapEncodeTiled_v12000;
 
 EncodeTiledFn encode_tiled() {
@@ -1466,6 +1515,8 @@ int make_plan(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out
 template <typename T>
 __global__ void splitk_reduce(const float* __restrict__ ws, T* __restrict__ y, const float* __restrict__ bias,
                               int KS, size_t stride, int Cout, int HoWo, int relu) {
+    pdl_trigger();
+    pdl_wait();
     const size_t total = stride;
     for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total; i += (size_t)gridDim.x * blockDim.x) {
         float a = ws[i];
@@ -1481,6 +1532,8 @@ __global__ void splitk_reduce(const float* __restrict__ ws, T* __restrict__ y, c
 template <typename T>
 __global__ void splitk_reduce_pool(const float* __restrict__ ws, T* __restrict__ y, const float* __restrict__ bias,
                                    int KS, size_t stride, int Cout, int Ho, int Wo, int relu) {
+    pdl_trigger();
+    pdl_wait();
     const int Hp = Ho >> 1, Wp = Wo >> 1;
     const size_t total = stride / ((size_t)Ho * Wo) * Hp * Wp;
     for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total; i += (size_t)gridDim.x * blockDim.x) {
@@ -1610,29 +1663,28 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
     const long long ctas = p.use_tma ? std::max<long long>(std::min<long long>(units, sm_count()),
                                                            (units + kMaxUnitsPerCta - 1) / kMaxUnitsPerCta)
                                      : units;
-    kern<<<(unsigned)ctas, kThreadsTM, smem, st>>>(p, tmap);
-    if (cudaGetLastError() != cudaSuccess) return PP_ERR_CUDA;
+    if (launch(kern, (unsigned)ctas, kThreadsTM, smem, st, p, tmap) != cudaSuccess) return PP_ERR_CUDA;
     if (pl.KS > 1) {
         const size_t total = p.ws_stride;
-        const int blocks = (int)std::max<size_t>(1, std::min<size_t>((total + 255) / 256, (size_t)sm_count() * 16));
-        if (pool)
-            splitk_reduce_pool<T><<<blocks, 256, 0, st>>>(p.ws, static_cast<T*>(y), bias, pl.KS, total, L->cout, Ho, Wo,
-                                                          relu);
-        else
-            splitk_reduce<T><<<blocks, 256, 0, st>>>(p.ws, static_cast<T*>(y), bias, pl.KS, total, L->cout, Ho * Wo,
-                                                     relu);
-        if (cudaGetLastError() != cudaSuccess) return PP_ERR_CUDA;
+        const unsigned blocks = (unsigned)std::max<size_t>(1, std::min<size_t>((total + 255) / 256, (size_t)sm_count() * 16));
+        const float* wsf = p.ws;
+        T* yt = static_cast<T*>(y);
+        const int ks = pl.KS, cout = L->cout, hw = Ho * Wo;
+        const cudaError_t e = pool ? launch(splitk_reduce_pool<T>, blocks, 256, 0, st, wsf, yt, bias, ks, total, cout, Ho, Wo, relu)
+                                   : launch(splitk_reduce<T>, blocks, 256, 0, st, wsf, yt, bias, ks, total, cout, hw, relu);
+        if (e != cudaSuccess) return PP_ERR_CUDA;
     }
     return PP_OK;
 }
 
 template <int S, typename T>
 int launch_depthwise_s(const DwParams& p, unsigned ctas, bool vin, bool vout, cudaStream_t st) {
-    if (vin && vout) pconv_depthwise<S, T, true, true><<<ctas, kDwThreads, 0, st>>>(p);
-    else if (vin) pconv_depthwise<S, T, true, false><<<ctas, kDwThreads, 0, st>>>(p);
-    else if (vout) pconv_depthwise<S, T, false, true><<<ctas, kDwThreads, 0, st>>>(p);
-    else pconv_depthwise<S, T, false, false><<<ctas, kDwThreads, 0, st>>>(p);
-    return cudaGetLastError() == cudaSuccess ? PP_OK : PP_ERR_CUDA;
+    cudaError_t e;
+    if (vin && vout) e = launch(pconv_depthwise<S, T, true, true>, ctas, kDwThreads, 0, st, p);
+    else if (vin) e = launch(pconv_depthwise<S, T, true, false>, ctas, kDwThreads, 0, st, p);
+    else if (vout) e = launch(pconv_depthwise<S, T, false, true>, ctas, kDwThreads, 0, st, p);
+    else e = launch(pconv_depthwise<S, T, false, false>, ctas, kDwThreads, 0, st, p);
+    return e == cudaSuccess ? PP_OK : PP_ERR_CUDA;
 }
 
 template <int S, typename T, bool VIN, bool VOUT, int RW, int NH>
@@ -1659,8 +1711,8 @@ int launch_dw_staged(const DwStagedParams& p, size_t smem, cudaStream_t st) {
                                                       kDwThreads, smem) != cudaSuccess || per_sm < 1)
         return PP_ERR_CUDA;
     const long long ctas = std::min<long long>(p.n_tiles, (long long)sm_count() * per_sm);
-    pconv_depthwise_staged<S, T, VIN, VOUT, RW, NH><<<(unsigned)ctas, kDwThreads, smem, st>>>(p);
-    return cudaGetLastError() == cudaSuccess ? PP_OK : PP_ERR_CUDA;
+    return launch(pconv_depthwise_staged<S, T, VIN, VOUT, RW, NH>, (unsigned)ctas, kDwThreads, smem, st, p) == cudaSuccess
+               ? PP_OK : PP_ERR_CUDA;
 }
 
 template <int S, typename T>

@@ -382,6 +382,54 @@ def test_vgg16_chained_network_fused_pool():
     assert tuple(x.shape) == (2, 512, 7, 7)
 
 
+@pytest.mark.parametrize("dtype", [torch.float32, torch.float16])
+def test_back_to_back_layers_match_layers_run_one_at_a_time(dtype):
+    """Layers launched one after another on one stream with no synchronisation (each kernel may
+    start its set-up while the previous one finishes) read exactly what the previous layer wrote:
+    ping-pong buffers (so a layer overwrites what the layer before it read), one workspace shared
+    by the split layers, a fused pool, a stride-2 layer and a depthwise layer; the chain, run three
+    times over, must equal the same layers run one at a time with a synchronisation after each."""
+    dev = torch.device("cuda")
+    N = 2
+    specs = [  # (Cin, Cout, H, stride, keep, depthwise, pool, input-channel split)
+        (8, 32, 28, 1, 0.5, False, False, False),
+        (32, 64, 28, 1, 0.3, False, True, True),
+        (64, 64, 14, 1, 0.3, False, False, False),
+        (64, 64, 14, 1, 0.3, False, False, True),
+        (64, 128, 14, 2, 0.4, False, False, True),
+        (128, 128, 7, 1, 1.0, True, False, False),
+        (128, 128, 7, 1, 0.3, False, False, True),
+    ]
+    layers, biases, in_shapes, out_shapes = [], [], [], []
+    for i, (ci, co, h, st, keep, dw, pool, _) in enumerate(specs):
+        L = WL.ConvLayer(f"b2b{i}", ci, co, h, h, st, dw, keep, w_seed=900 + i, b_seed=950 + i)
+        layers.append(api.pp_pack(WL.weights(L), None, keep, co if dw else 1, st).bind(dev))
+        biases.append(torch.from_numpy(WL.bias(L)).to(dev))
+        in_shapes.append((N, ci, h, h))
+        o = layers[-1].out_shape(in_shapes[-1])
+        out_shapes.append((o[0], o[1], o[2] // 2, o[3] // 2) if pool else o)
+    x0 = torch.from_numpy(rnd(in_shapes[0], 990, dtype=_np_dt(dtype))).to(dev)
+    ws = api.workspace_for(layers, in_shapes, dev)
+    splits = [lay.plan(s, ws.numel() * 4 if sp[7] else 0)["splits"] for lay, s, sp in zip(layers, in_shapes, specs)]
+    assert splits == [1, 32, 1, 32, 32, 0, 32], splits     # 0: the depthwise kernel
+
+    ref = x0
+    for lay, b, sp in zip(layers, biases, specs):
+        ref = lay.conv(ref.clone(), b, True, workspace=ws if sp[7] else None, pool2x2=sp[6])
+        torch.cuda.synchronize()
+
+    big = max(int(np.prod(s)) for s in out_shapes)
+    bufs = [torch.full((big,), float("nan"), dtype=dtype, device=dev) for _ in range(2)]
+    for _ in range(3):
+        cur = x0
+        for i, (lay, b, sp) in enumerate(zip(layers, biases, specs)):
+            y = bufs[i % 2].narrow(0, 0, int(np.prod(out_shapes[i]))).view(out_shapes[i])
+            lay.conv(cur, b, True, y, workspace=ws if sp[7] else None, pool2x2=sp[6])
+            cur = y
+    torch.cuda.synchronize()
+    assert torch.equal(cur, ref)
+
+
 # --------------------------------------------------------------------------- channel split
 
 def _split_case():
