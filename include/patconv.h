@@ -188,7 +188,9 @@ int pp_conv_workspace_size(pp_handle h, int N, int H, int W, size_t* bytes);
  * [8] filter groups and [9] spatial warps per CTA, [10] shared-memory bytes, [11] channel chunks
  * per unit, [12] CTAs launched when the input goes through TMA (fp32 with rows a multiple of 16
  * bytes: persistent CTAs, at most one per SM unless the units overflow a CTA's unit table; the
- * copy fallback launches one CTA per unit).  Writes min(n_info, 13) values.  Host-only. */
+ * copy fallback launches one CTA per unit), [13] 1 where a stride-1 fp32 launch deals each warp's
+ * blocks to its lanes by shared-memory bank group (fewer conflicting window loads; rows of 7 or
+ * 14 blocks), else 0.  Writes min(n_info, 14) values.  Host-only. */
 int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info);
 
 /* pp_conv_ws for callers that cannot allocate device memory (the paper has no counterpart to

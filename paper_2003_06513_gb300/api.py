@@ -102,14 +102,14 @@ class Layer:
 
     PLAN_KEYS = ("path", "splits", "workspace_bytes", "units", "tile_by", "tile_bx", "tile_nb",
                  "channels_per_stage", "filter_groups", "spatial_warps", "smem_bytes",
-                 "chunks_per_unit", "ctas")
+                 "chunks_per_unit", "ctas", "lane_sort")
 
     def plan(self, x_shape, workspace_bytes: int = 0) -> dict:
         """Launch plan pp_conv_ws would use for input shape [N, C, H, W] (pp_conv_plan)."""
         N, _, H, W = x_shape
-        info = (ctypes.c_int64 * 13)()
+        info = (ctypes.c_int64 * 14)()
         _lib.check("pp_conv_plan", _lib.load().pp_conv_plan(self._h, N, H, W, int(workspace_bytes),
-                                                            info, 13))
+                                                            info, 14))
         return dict(zip(self.PLAN_KEYS, (int(v) for v in info)))
 
     def workspace_bytes(self, x_shape) -> int:

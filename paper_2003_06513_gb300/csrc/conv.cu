@@ -302,7 +302,8 @@ __device__ __forceinline__ void fill_share(const TmParams& p, const CUtensorMap*
     cp_async_arrive(fb);
 }
 
-template <int S, typename TIn>
+// SORT (stride 1, fp32 only): each warp's blocks are dealt to its lanes by bank group.
+template <int S, typename TIn, bool SORT = false>
 __global__ void __launch_bounds__(kThreadsTM, 1)
     pconv_tm(const TmParams p, const __grid_constant__ CUtensorMap tmap) {
     constexpr int RY = 4, RX = 4;
@@ -400,24 +401,44 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     bool active = false;
     auto place_lane = [&]() {
         const Unit CU = s_units[ci];
-        int rem;
-        if (p.linear) {
-            const long long b = (long long)CU.tn * lanes_t + blk;
-            const int ng = (int)(b / bpi);
-            img = ng - CU.n0;
-            rem = (int)(b - (long long)ng * bpi);
-            active = ng < p.N && img < p.NB;
-        } else {
-            img = blk / bpi;
-            rem = blk - img * bpi;
-            active = img < p.NB;
+        // block t (0 .. 32 * WS - 1) of the unit's tile: image, block row and column, and where
+        // the lane's window column 0 (input column ox0 * S - 1 of the block) sits in the stage:
+        // d = 3 into the row for fp32 stages, 3 or 7 for fp16 ones (their origin is 16 bytes)
+        auto locate = [&](int t) {
+            int rem;
+            if (p.linear) {
+                const long long b = (long long)CU.tn * lanes_t + t;
+                const int ng = (int)(b / bpi);
+                img = ng - CU.n0;
+                rem = (int)(b - (long long)ng * bpi);
+                active = ng < p.N && img < p.NB;
+            } else {
+                img = t / bpi;
+                rem = t - img * bpi;
+                active = img < p.NB;
+            }
+            by = rem / p.BX;
+            bx = rem - by * p.BX;
+            const int d = CU.ox0 * S - 1 - CU.ix0;
+            in_off = active ? img * p.CK * plane + by * RY * S * p.BWb + bx * RX * S + d : d;
+        };
+        locate(blk);
+        if constexpr (SORT) {
+            static_assert(S == 1 && sizeof(TIn) == 4, "bank groups are those of fp32 stride-1 windows");
+            // The warp's 32 blocks are dealt to its lanes so that each 8-lane phase of the
+            // 16-byte window loads (window columns 1-4, at in_off + 1) meets distinct bank
+            // groups where the blocks allow it: blocks are ordered by (rank among the blocks of
+            // their bank group, bank group) and lane i takes the i-th.  Rows of 7 or 14 blocks
+            // otherwise put two blocks of a phase on one bank group.  Idle lanes go last.  The
+            // planner picks this instance where it lowers the wavefronts (window_wavefronts).
+            const int grp = active ? ((in_off + 1) >> 2) & 7 : 8;
+            const unsigned same = __match_any_sync(0xffffffffu, grp);
+            const int key = active ? 16 * __popc(same & ((1u << lane) - 1u)) + grp : 1024 + lane;   // distinct
+            int pos = 0, src = 0;
+            for (int i = 0; i < 32; ++i) pos += __shfl_sync(0xffffffffu, key, i) < key ? 1 : 0;
+            for (int i = 0; i < 32; ++i) src = __shfl_sync(0xffffffffu, pos, i) == lane ? i : src;
+            locate(ws * 32 + src);
         }
-        by = rem / p.BX;
-        bx = rem - by * p.BX;
-        // window column 0 (input column ox0 * S - 1 of the lane's block) sits at d in the stage
-        // row: 3 for fp32 stages, 3 or 7 for fp16 ones (their origin is 16 bytes = 8 columns)
-        const int d = CU.ox0 * S - 1 - CU.ix0;
-        in_off = active ? img * p.CK * plane + by * RY * S * p.BWb + bx * RX * S + d : d;
         // lanes whose left neighbour lane does not hold the block to their left (stride 2 takes
         // window column 0 from that neighbour)
         edge = (bx == 0 || lane == 0) ? 1u : 0u;
@@ -1298,6 +1319,7 @@ struct Plan {
     int CK = 0, n_chunks = 0, maxk = 0, KS = 1, c_split = 0;
     size_t stage_bytes = 0, kb_bytes = 0, smem = 0;
     long long ctas = 0;           // CTAs of one split
+    int lane_sort = 0;            // stride 1: pconv_tm deals blocks to lanes by bank group
     size_t ws_bytes = 0;          // workspace the chosen split needs (0 without a split)
 };
 
@@ -1339,6 +1361,57 @@ std::vector<TileChoice> tile_candidates(int N, int Ho, int Wo, int S, int lanes)
     if (N > 1 && bpi < 4LL * lanes && ih <= 256 && bw <= 256 && nb <= 256)
         out.push_back(TileChoice{nby, nbx, nb, ih, bw, 1});
     return out;
+}
+
+// Shared-memory wavefronts of warp 0's 16-byte window loads (window columns 1-4 of every lane,
+// fp32 stride-1 stage) in tile t: four phases of 8 lanes, each costing the largest number of its
+// lanes whose loads fall on one bank group (16 bytes = 4 banks; 8 groups).  Lanes take the tile's
+// blocks in raster order, or dealt by bank group as pconv_tm does with lane_sort.
+int window_wavefronts(const Plan& pl, int N, long long t, bool sorted) {
+    const TileChoice& tc = pl.tile;
+    const int lanes_t = 32 * pl.WS, bpi = tc.BY * tc.BX, plane = tc.IH * tc.BWb;
+    int grp[32], key[32], order[32];
+    for (int l = 0; l < 32; ++l) {
+        int img, rem;
+        bool active;
+        if (tc.linear) {
+            const long long b = t * lanes_t + l;
+            const long long ng = b / bpi, n0 = t * lanes_t / bpi;
+            img = (int)(ng - n0);
+            rem = (int)(b - ng * bpi);
+            active = ng < N && img < tc.NB;
+        } else {
+            img = l / bpi;
+            rem = l - img * bpi;
+            active = img < tc.NB;
+        }
+        const int by = rem / tc.BX, bx = rem - by * tc.BX;
+        const long long off = (long long)img * pl.CK * plane + (long long)by * 4 * tc.BWb + bx * 4;
+        grp[l] = active ? (int)((off / 4) & 7) : 8;
+    }
+    for (int l = 0; l < 32; ++l) {
+        int rank = 0;
+        for (int i = 0; i < l; ++i) rank += grp[i] == grp[l];
+        key[l] = grp[l] < 8 ? 16 * rank + grp[l] : 1024 + l;
+    }
+    for (int l = 0; l < 32; ++l) {
+        int pos = l;
+        if (sorted) {
+            pos = 0;
+            for (int i = 0; i < 32; ++i) pos += key[i] < key[l];
+        }
+        order[pos] = l;
+    }
+    int w = 0;
+    for (int ph = 0; ph < 4; ++ph) {
+        int cnt[9] = {0, 0, 0, 0, 0, 0, 0, 0, 0}, m = 0;
+        for (int k = 0; k < 8; ++k) {
+            const int g = grp[order[8 * ph + k]];
+            if (g < 8) m = std::max(m, ++cnt[g]);
+        }
+        w += m;
+    }
+    return w;
 }
 
 int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out) {
@@ -1388,6 +1461,24 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
             pl->maxk = maxk_for(ck);
             pl->smem = layout(ck, pl->maxk, &pl->stage_bytes, &pl->kb_bytes);
             if (pl->smem <= 200 * 1024) break;
+        }
+        // several images in a stage: an image stride of a multiple of 32 floats puts every image's
+        // windows on the same bank groups (7x7 maps: 8 images of 2x2 blocks, 4 bank groups in
+        // all); one channel less per stage where that lowers the modelled window wavefronts
+        auto wavefronts_for = [&](int c) {
+            Plan q = *pl;
+            q.CK = c;
+            const long long nt = t.linear ? std::min<long long>(tn, 64) : 1;
+            long long w = 0;
+            for (long long i = 0; i < nt; ++i)
+                w += std::min(window_wavefronts(q, N, i, false), window_wavefronts(q, N, i, true));
+            return w;
+        };
+        if (S == 1 && t.NB > 1 && ck > 1 && ((size_t)ck * t.IH * t.BWb) % 32 == 0 &&
+            (C + ck - 2) / (ck - 1) <= kMaxChunks && wavefronts_for(ck - 1) < wavefronts_for(ck)) {
+            --ck;
+            pl->maxk = maxk_for(ck);
+            pl->smem = layout(ck, pl->maxk, &pl->stage_bytes, &pl->kb_bytes);
         }
         pl->CK = ck;
         pl->maxk = std::max(pl->maxk, 1);
@@ -1481,6 +1572,15 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
     const double cl = have_lin ? 1.2 * finish(lin, 1, 1, ltn, &pli) : 1e300;
     if (cr >= 1e300 && cl >= 1e300) return PP_ERR_SHAPE;
     *out = cl < cr ? pli : pr;
+    if (S == 1) {   // the bank-group order where it lowers the window loads' wavefronts
+        const long long nt = out->tile.linear ? std::min<long long>(out->tiles_n, 64) : 1;
+        long long raster = 0, sorted = 0;
+        for (long long t = 0; t < nt; ++t) {
+            raster += window_wavefronts(*out, N, t, false);
+            sorted += window_wavefronts(*out, N, t, true);
+        }
+        out->lane_sort = sorted < raster ? 1 : 0;
+    }
     return PP_OK;
 }
 
@@ -1559,7 +1659,7 @@ __global__ void splitk_reduce_pool(const float* __restrict__ ws, T* __restrict__
 // Raise the kernel's dynamic shared-memory limit to the device's opt-in maximum once per device
 // (a launch needs at most that), so that later calls, including ones under stream capture, make
 // no attribute call.
-template <int S, typename T>
+template <int S, typename T, bool SORT>
 bool allow_max_smem(size_t need) {
     static std::atomic<int> done[64];
     int dev = 0;
@@ -1568,7 +1668,7 @@ bool allow_max_smem(size_t need) {
     int optin = 0;
     if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess) return false;
     if ((size_t)optin < need) return false;
-    if (cudaFuncSetAttribute(pconv_tm<S, T>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin) != cudaSuccess)
+    if (cudaFuncSetAttribute(pconv_tm<S, T, SORT>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin) != cudaSuccess)
         return false;
     done[dev].store(1, std::memory_order_release);
     return true;
@@ -1652,8 +1752,19 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
         if (r != CUDA_SUCCESS) p.use_tma = 0;
         p.tma_bytes = (unsigned)((size_t)p.BWb * p.IH * p.CK * p.NB * es);
     }
-    auto kern = pconv_tm<S, T>;
-    if (!allow_max_smem<S, T>(smem)) return PP_ERR_CUDA;
+    auto kern = pconv_tm<S, T, false>;
+    bool smem_ok;
+    if constexpr (S == 1 && sizeof(T) == 4) {
+        if (pl.lane_sort) {
+            kern = pconv_tm<1, float, true>;
+            smem_ok = allow_max_smem<1, float, true>(smem);
+        } else {
+            smem_ok = allow_max_smem<S, T, false>(smem);
+        }
+    } else {
+        smem_ok = allow_max_smem<S, T, false>(smem);
+    }
+    if (!smem_ok) return PP_ERR_CUDA;
     const long long units = pl.ctas * pl.KS;
     if (units > INT_MAX) return PP_ERR_SHAPE;
     p.n_units = (int)units;
@@ -1984,7 +2095,7 @@ int pp_conv_pool_ws(pp_handle h, const void* x, int dtype, int N, int H, int W, 
 int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info) {
     if (!h || !info) return PP_ERR_NULL;
     if (N < 1 || H < 1 || W < 1 || n_info < 1) return PP_ERR_SHAPE;
-    int64_t v[13] = {0};
+    int64_t v[14] = {0};
     if (!h->fast || h->depthwise) {
         v[0] = h->depthwise ? 2 : 3;   // depthwise kernel / generic kernel: no plan, no workspace
     } else {
@@ -2007,8 +2118,9 @@ int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64
         v[9] = pl.WS;
         v[10] = (int64_t)pl.smem;
         v[11] = pl.n_chunks;
+        v[13] = pl.lane_sort;
     }
-    for (int i = 0; i < n_info && i < 13; ++i) info[i] = v[i];
+    for (int i = 0; i < n_info && i < 14; ++i) info[i] = v[i];
     return PP_OK;
 }
 

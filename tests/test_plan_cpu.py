@@ -35,7 +35,102 @@ def _check(layer, shape, ws):
     # units: tiles x filter chunks x splits; persistent CTAs never exceed the units
     assert pl["units"] % pl["splits"] == 0
     assert pl["ctas"] <= pl["units"]
+    assert pl["lane_sort"] in (0, 1) and (layer.stride == 1 or pl["lane_sort"] == 0)
     return pl
+
+
+def _stage_geometry(pl, stride):
+    """Staged rows per (image, channel) and their width in floats, as the planner lays them out."""
+    by, bx = pl["tile_by"], pl["tile_bx"]
+    ih = 4 * by + 2 if stride == 1 else 8 * by + 1
+    bw = 4 * bx + 8 if stride == 1 else 8 * bx + 4
+    return ih, bw + 4 if bw % 8 == 0 else bw
+
+
+def _window_wavefronts(pl, shape, stride, t, dealt):
+    """Wavefronts of warp 0's 16-byte window loads in tile t: 4 phases of 8 lanes, each costing
+    the most lanes on one of the 8 bank groups; lanes in raster order or dealt by
+    (rank within bank group, bank group) with idle lanes last."""
+    n = shape[0]
+    ho, wo = (shape[2] - 1) // stride + 1, (shape[3] - 1) // stride + 1
+    nby, nbx = (ho + 3) // 4, (wo + 3) // 4
+    by_t, bx_t, nb = pl["tile_by"], pl["tile_bx"], pl["tile_nb"]
+    lanes = 32 * pl["spatial_warps"]
+    linear = by_t == nby and bx_t == nbx and nb > 1 and nby * nbx * nb != lanes and lanes % (nby * nbx) != 0
+    ih, bw = _stage_geometry(pl, stride)
+    grp = []
+    for lane in range(32):
+        if linear:
+            b = t * lanes + lane
+            img, rem = b // (by_t * bx_t) - (t * lanes) // (by_t * bx_t), b % (by_t * bx_t)
+            active = b // (by_t * bx_t) < n and img < nb
+        else:
+            img, rem = divmod(lane, by_t * bx_t)
+            active = img < nb
+        off = img * pl["channels_per_stage"] * ih * bw + (rem // bx_t) * 4 * bw + (rem % bx_t) * 4
+        grp.append((off // 4) % 8 if active else None)
+    order = list(range(32))
+    if dealt:
+        seen, keys = {}, []
+        for lane, g in enumerate(grp):
+            if g is None:
+                keys.append((1 << 20) + lane)
+            else:
+                keys.append(16 * seen.get(g, 0) + g)
+                seen[g] = seen.get(g, 0) + 1
+        order = sorted(range(32), key=lambda lane: keys[lane])
+    w = 0
+    for ph in range(4):
+        gs = [grp[lane] for lane in order[8 * ph:8 * ph + 8] if grp[lane] is not None]
+        w += max([gs.count(g) for g in set(gs)] or [0])
+    return w
+
+
+@pytest.mark.parametrize("which", ["vgg16", "resnet50"])
+def test_lane_order_by_bank_group(which):
+    """The planner deals blocks to lanes by bank group exactly where that lowers the modelled
+    wavefronts of the window loads (stride 1): on VGG-16 the 56x56 and 28x28 layers (rows of 14
+    and 7 blocks), not the 224, 112 or 14 ones."""
+    layers = WL.vgg16() if which == "vgg16" else WL.resnet50_3x3()
+    n = 32 if which == "vgg16" else 64
+    got = {}
+    for L in layers:
+        layer = api.pp_pack(WL.weights(L), None, L.keep, 1, L.stride)
+        shape = (n, L.cin, L.h, L.w)
+        pl = layer.plan(shape, layer.workspace_bytes(shape))
+        got[L.name] = pl["lane_sort"]
+        if L.stride != 1:
+            assert pl["lane_sort"] == 0
+            continue
+        tiles = 1
+        ho, wo = L.ho, L.wo
+        nby, nbx = (ho + 3) // 4, (wo + 3) // 4
+        if pl["tile_by"] == nby and pl["tile_bx"] == nbx and pl["tile_nb"] > 1:
+            tiles = min(64, (n * nby * nbx + 31) // 32)
+        raster = sum(_window_wavefronts(pl, shape, 1, t, False) for t in range(tiles))
+        dealt = sum(_window_wavefronts(pl, shape, 1, t, True) for t in range(tiles))
+        assert pl["lane_sort"] == (1 if dealt < raster else 0), (L.name, raster, dealt)
+    if which == "vgg16":
+        assert [got[f"vgg{i}"] for i in range(1, 14)] == [0, 0, 0, 0, 1, 1, 1, 1, 1, 1, 0, 0, 0]
+
+
+def test_multi_image_stages_are_not_bank_aligned():
+    """Where an 8-lane phase of the window loads holds blocks of several images (fewer than 8
+    blocks per image, stride 1), the image stride in the stage is no multiple of 32 floats, which
+    would put every image's windows on the same banks (ResNet-50's 7x7 layers: 2x2 blocks)."""
+    seen = 0
+    for which, n in (("vgg16", 32), ("resnet50", 64)):
+        layers = WL.vgg16() if which == "vgg16" else WL.resnet50_3x3()
+        for L in layers:
+            layer = api.pp_pack(WL.weights(L), None, L.keep, 1, L.stride)
+            shape = (n, L.cin, L.h, L.w)
+            pl = layer.plan(shape, layer.workspace_bytes(shape))
+            if (L.stride == 1 and pl["tile_nb"] > 1 and pl["tile_by"] * pl["tile_bx"] < 8
+                    and pl["channels_per_stage"] > 1):
+                ih, bw = _stage_geometry(pl, L.stride)
+                assert (pl["channels_per_stage"] * ih * bw) % 32 != 0, L.name
+                seen += 1
+    assert seen == 2
 
 
 @pytest.mark.parametrize("seed", range(40))
