@@ -190,6 +190,9 @@ def test_depthwise(dtype, stride):
                                             (2, 16, 32, 48, 2),
                                             (3, 40, 7, 7, 1),       # many small planes per CTA
                                             (2, 24, 14, 14, 2),
+                                            (2, 24, 14, 14, 1),     # whole-row items, 14 wide
+                                            (2, 16, 28, 28, 1),     # 28-wide rows in 2 pieces (fp16)
+                                            (2, 16, 28, 28, 2),
                                             (1, 4, 9, 2100, 1),     # rows too wide to stage whole
                                             (1, 4, 9, 2100, 2)])
 def test_depthwise_vector_and_tiled(dtype, N, C, H, W, stride):
@@ -199,6 +202,21 @@ def test_depthwise_vector_and_tiled(dtype, N, C, H, W, stride):
     b = (rng.standard_normal(C) * 0.1).astype(np.float32)
     check(Wd, x, b, 1.0, stride, depthwise=True, dtype=dtype, guard=64)
     check(Wd, x, b, 0.7, stride, relu=False, depthwise=True, dtype=dtype, guard=64)
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.float16])
+@pytest.mark.parametrize("H,stride", [(7, 1), (14, 1), (14, 2)])
+def test_depthwise_other_library(dtype, H, stride):
+    """A library other than the compiled one: the depthwise kernels take the taps from the masks
+    (the default library's pattern-specialised row bodies do not apply)."""
+    rng = np.random.default_rng(41 + H)
+    C = 40
+    masks = [OP.mask_of(t) for t in ([0, 4, 5, 8], [1, 4, 6, 7], [2, 3, 4, 8])]
+    Wd = (rng.standard_normal((C, 1, 3, 3)) * np.sqrt(2 / 9)).astype(np.float32)
+    x = rnd((3, C, H, H), 50 + H, dtype=_np_dt(dtype))
+    b = (rng.standard_normal(C) * 0.1).astype(np.float32)
+    check(Wd, x, b, 1.0, stride, depthwise=True, dtype=dtype, masks=masks)
+    check(Wd, x, b, 0.6, stride, depthwise=True, dtype=dtype, masks=masks)
 
 
 @pytest.mark.parametrize("dtype", [torch.float32, torch.float16])
