@@ -1564,12 +1564,17 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
             have_rect = true;
         }
     }
-    // the linear tile stages whole images (fewer channels per stage) and its lanes hit more bank
-    // conflicts; it must beat the best rectangle by that margin in estimated channel steps
+    // the linear tile stages whole images (fewer channels per stage, more stages) and its lanes
+    // hit more bank conflicts: a per-channel cost, worth about 1.3 kernel visits against 0.4 for
+    // a rectangle's window, so its estimated channel steps are weighed by (1.3 + k) / (0.4 + k), k
+    // the layer's mean kept kernels per (input channel, filter group).  Calibrated on 28x28 maps
+    // (VGG-16 and the sweep): rectangles win at k <= 2.4 (VGG-16 layers 8-10: -11, -2, +1 %), the
+    // linear tile at k = 8 (by 17-29 %: idle lanes) and mostly at k = 4
     Plan pr, pli;
     const double cr = have_rect ? finish(rect, rtx, rty, rtn, &pr) : 1e300;
     const int ltn = (int)(((long long)N * nby * nbx + lanes - 1) / lanes);
-    const double cl = have_lin ? 1.2 * finish(lin, 1, 1, ltn, &pli) : 1e300;
+    const double kpc = (double)L->beta / ((double)L->G * C);
+    const double cl = have_lin ? (1.3 + kpc) / (0.4 + kpc) * finish(lin, 1, 1, ltn, &pli) : 1e300;
     if (cr >= 1e300 && cl >= 1e300) return PP_ERR_SHAPE;
     *out = cl < cr ? pli : pr;
     if (S == 1) {   // the bank-group order where it lowers the window loads' wavefronts
