@@ -170,3 +170,22 @@ def test_other_paths_report_no_plan():
     gen = api.pp_pack(rng.standard_normal((8, 4, 3, 3)).astype(np.float32), masks, 0.5)
     assert gen.plan((1, 4, 9, 9), 0)["path"] == 3
     assert gen.workspace_bytes((1, 4, 9, 9)) == 0
+
+
+def test_linear_tile_weighed_by_density():
+    """28x28 maps (7 blocks a row): at VGG-16's keep 0.3 the planner takes 4x7 rectangles
+    without a split; at keep 1.0 the linear tile (every lane busy) pays for its per-channel cost."""
+    for L in WL.vgg16()[7:10]:
+        layer = api.pp_pack(WL.weights(L), None, L.keep)
+        shape = (32, L.cin, L.h, L.w)
+        pl = layer.plan(shape, layer.workspace_bytes(shape))
+        assert (pl["tile_by"], pl["tile_bx"], pl["tile_nb"], pl["splits"]) == (4, 7, 1, 1), L.name
+    rng = np.random.default_rng(7)
+    W = (rng.standard_normal((256, 256, 3, 3)) * np.sqrt(2 / (9 * 256))).astype(np.float32)
+    shape = (64, 256, 28, 28)
+    dense = api.pp_pack(W, None, 1.0)
+    pl = dense.plan(shape, dense.workspace_bytes(shape))
+    assert (pl["tile_by"], pl["tile_bx"]) == (7, 7) and pl["tile_nb"] > 1     # linear
+    sparse = api.pp_pack(W, None, 0.25)
+    pl = sparse.plan(shape, sparse.workspace_bytes(shape))
+    assert (pl["tile_by"], pl["tile_bx"], pl["tile_nb"]) == (4, 7, 1)
