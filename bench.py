@@ -517,7 +517,7 @@ def our_arm(args, rank, world, local_rank):
             "config": config_dict(),
             "useful_gflops": world * sum(flops) / (ms_step * 1e-3) / 1e9,
             "network_roofline_frac": roof_ms / tot_conv_ms,
-            "roofline": {"bound": "alu", "kernel": "pconv_tm<1,float> (+ split reduce)",
+            "roofline": {"bound": "alu", "kernel": "pconv_tm<1,float,SORT> (+ split reduce)",
                          "achieved": achieved / 1e12, "peak": peak / 1e12, "unit": "TFLOP/s",
                          "frac": achieved / peak,
                          "peak_basis": f"{props.multi_processor_count} SMs x 128 FP32 lanes x 2 x {mhz:.0f} MHz",
