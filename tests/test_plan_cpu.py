@@ -47,6 +47,21 @@ def _stage_geometry(pl, stride):
     return ih, bw + 4 if bw % 8 == 0 else bw
 
 
+def _is_linear(pl, shape, stride):
+    """Whether the plan's tile is the linear one (None where its shape does not tell)."""
+    n = shape[0]
+    ho, wo = (shape[2] - 1) // stride + 1, (shape[3] - 1) // stride + 1
+    nby, nbx = (ho + 3) // 4, (wo + 3) // 4
+    if (pl["tile_by"], pl["tile_bx"]) != (nby, nbx) or pl["tile_nb"] == 1:
+        return False
+    bpi, lanes = nby * nbx, 32 * pl["spatial_warps"]
+    rect_nb = min(n, 256, max(1, lanes // bpi))
+    lin_nb = min(n, (lanes - 1) // bpi + 2)
+    if rect_nb == lin_nb or (bpi < lanes and lanes % bpi == 0):
+        return None if rect_nb == lin_nb and not (bpi < lanes and lanes % bpi == 0) else False
+    return pl["tile_nb"] == lin_nb
+
+
 def _window_wavefronts(pl, shape, stride, t, dealt):
     """Wavefronts of warp 0's 16-byte window loads in tile t: 4 phases of 8 lanes, each costing
     the most lanes on one of the 8 bank groups; lanes in raster order or dealt by
@@ -56,7 +71,7 @@ def _window_wavefronts(pl, shape, stride, t, dealt):
     nby, nbx = (ho + 3) // 4, (wo + 3) // 4
     by_t, bx_t, nb = pl["tile_by"], pl["tile_bx"], pl["tile_nb"]
     lanes = 32 * pl["spatial_warps"]
-    linear = by_t == nby and bx_t == nbx and nb > 1 and nby * nbx * nb != lanes and lanes % (nby * nbx) != 0
+    linear = bool(_is_linear(pl, shape, stride))
     ih, bw = _stage_geometry(pl, stride)
     grp = []
     for lane in range(32):
@@ -189,3 +204,29 @@ def test_linear_tile_weighed_by_density():
     sparse = api.pp_pack(W, None, 0.25)
     pl = sparse.plan(shape, sparse.workspace_bytes(shape))
     assert (pl["tile_by"], pl["tile_bx"], pl["tile_nb"]) == (4, 7, 1)
+
+
+@pytest.mark.parametrize("seed", range(30))
+def test_lane_order_random_shapes(seed):
+    """The planner's bank-group lane order agrees with an independent model of the window loads'
+    wavefronts on random stride-1 shapes (rectangles and linear tiles)."""
+    rng = np.random.default_rng(100 + seed)
+    c = int(rng.choice([16, 64, 128, 256]))
+    n = int(rng.choice([1, 2, 3, 8, 32]))
+    h, w = int(rng.integers(5, 120)), int(rng.integers(5, 120))
+    keep = float(rng.choice([1.0, 0.5, 0.3]))
+    W = rng.standard_normal((c, c, 3, 3)).astype(np.float32)
+    layer = api.pp_pack(W, None, keep)
+    shape = (n, c, h, w)
+    for ws in (0, layer.workspace_bytes(shape)):
+        pl = layer.plan(shape, ws)
+        linear = _is_linear(pl, shape, 1)
+        if linear is None:
+            continue
+        tiles = 1
+        if linear:
+            nby, nbx = (h + 3) // 4, (w + 3) // 4
+            tiles = min(64, (n * nby * nbx + 32 * pl["spatial_warps"] - 1) // (32 * pl["spatial_warps"]))
+        raster = sum(_window_wavefronts(pl, shape, 1, t, False) for t in range(tiles))
+        dealt = sum(_window_wavefronts(pl, shape, 1, t, True) for t in range(tiles))
+        assert pl["lane_sort"] == (1 if dealt < raster else 0), (shape, ws, raster, dealt, pl)
