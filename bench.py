@@ -369,7 +369,7 @@ def our_arm(args, rank, world, local_rank):
         h = ho
     x0 = torch.from_numpy(WL.vgg16_image(BATCH)).to(dev)
     in_shapes = [(BATCH, L.cin) + ((224, 224) if i == 0 else shapes[i - 1][2:]) for i, L in enumerate(layers)]
-    workspace = api.workspace_for(packed, in_shapes, dev)   # input-channel split of small layers
+    workspace = api.workspace_for(packed, in_shapes, dev, [L.pool_after for L in layers])   # split of small layers
     big = max(int(np.prod(s)) for s in shapes)
     bufA = torch.empty(big, dtype=torch.float32, device=dev)
     bufB = torch.empty(big, dtype=torch.float32, device=dev)
@@ -570,7 +570,7 @@ def batch1_context(packed, biases, layers, K, barrier, dev):
         in_shapes.append((1, L.cin, h, h))
         h = h // 2 if L.pool_after else h
         shapes.append((1, L.cout, h, h))
-    ws = api.workspace_for(packed, in_shapes, dev)
+    ws = api.workspace_for(packed, in_shapes, dev, [L.pool_after for L in layers])
     outs = [torch.empty(sh, dtype=torch.float32, device=dev) for sh in shapes]
 
     def step():

@@ -102,19 +102,24 @@ class Layer:
 
     PLAN_KEYS = ("path", "splits", "workspace_bytes", "units", "tile_by", "tile_bx", "tile_nb",
                  "channels_per_stage", "filter_groups", "spatial_warps", "smem_bytes",
-                 "chunks_per_unit", "ctas", "lane_sort")
+                 "chunks_per_unit", "ctas", "lane_sort", "shift")
 
-    def plan(self, x_shape, workspace_bytes: int = 0) -> dict:
-        """Launch plan pp_conv_ws would use for input shape [N, C, H, W] (pp_conv_plan)."""
+    def plan(self, x_shape, workspace_bytes: int = 0, pool2x2: bool = False) -> dict:
+        """Launch plan pp_conv_ws (or, with pool2x2, pp_conv_pool_ws) would use for input shape
+        [N, C, H, W] (pp_conv_plan / pp_conv_pool_plan)."""
         N, _, H, W = x_shape
-        info = (ctypes.c_int64 * 14)()
-        _lib.check("pp_conv_plan", _lib.load().pp_conv_plan(self._h, N, H, W, int(workspace_bytes),
-                                                            info, 14))
+        n = len(self.PLAN_KEYS)
+        info = (ctypes.c_int64 * n)()
+        name = "pp_conv_pool_plan" if pool2x2 else "pp_conv_plan"
+        _lib.check(name, getattr(_lib.load(), name)(self._h, N, H, W, int(workspace_bytes), info, n))
         return dict(zip(self.PLAN_KEYS, (int(v) for v in info)))
 
-    def workspace_bytes(self, x_shape) -> int:
-        """Workspace the input-channel split would use for this input shape (0: no split)."""
+    def workspace_bytes(self, x_shape, pool2x2: bool = False) -> int:
+        """Workspace the input-channel split would use for this input shape (0: no split), for
+        pp_conv_ws or, with pool2x2, for pp_conv_pool_ws (whose plan may differ)."""
         N, _, H, W = x_shape
+        if pool2x2:
+            return self.plan(x_shape, (1 << 64) - 1, pool2x2=True)["workspace_bytes"]
         v = ctypes.c_size_t()
         _lib.check("pp_conv_workspace_size", _lib.load().pp_conv_workspace_size(
             self._h, N, H, W, ctypes.byref(v)))
@@ -203,9 +208,11 @@ def pp_conv(layer: Layer, x: torch.Tensor, bias: Optional[torch.Tensor], relu: b
     return layer.conv(x, bias, relu, y, stream, workspace)
 
 
-def workspace_for(layers, x_shapes, device=None) -> Optional[torch.Tensor]:
-    """One device buffer large enough for the input-channel split of every (layer, shape)."""
-    n = max([lay.workspace_bytes(s) for lay, s in zip(layers, x_shapes)] + [0])
+def workspace_for(layers, x_shapes, device=None, pools=None) -> Optional[torch.Tensor]:
+    """One device buffer large enough for the input-channel split of every (layer, shape); pools
+    flags the layers called with the fused 2x2 max-pool."""
+    pools = pools or [False] * len(layers)
+    n = max([lay.workspace_bytes(s, p) for lay, s, p in zip(layers, x_shapes, pools)] + [0])
     if n == 0:
         return None
     return torch.empty(n // 4 + 4, dtype=torch.float32, device=device or "cuda")

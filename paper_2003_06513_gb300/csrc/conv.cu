@@ -115,7 +115,7 @@ struct TmParams {
     size_t ws_stride;                  // elements per split
     int IH, BWb;                       // staged rows / row width (elements) per (image, channel)
     int ixa;                           // stage origin column: a multiple of ixa (16 bytes of input)
-    int use_tma, vec_store;
+    int use_tma, vec_store, vec_pair;  // float4 / 8-byte-group stores; pair stores (SHIFT)
     int pool, vec_pool;                // fused 2x2/2 max-pool of the output; pair stores of it
     unsigned tma_bytes;                // bytes one TMA box delivers
     unsigned kb_off, stage_off, stage_bytes, desc_off, vals_off;   // shared-memory layout
@@ -303,10 +303,15 @@ __device__ __forceinline__ void fill_share(const TmParams& p, const CUtensorMap*
 }
 
 // SORT (stride 1, fp32 only): each warp's blocks are dealt to its lanes by bank group.
-template <int S, typename TIn, bool SORT = false>
+// SHIFT (stride 1): block j of a tile row covers output columns ox0 + 4j - 1 .. ox0 + 4j + 2, so
+// that a lane's window column 0 sits at 2 (mod 4) in the stage and each window row is one 8-byte
+// and one 16-byte shared load (without SHIFT: 4-byte, 16-byte, 4-byte, the 4-byte ones bank
+// conflicted).  Not used with the fused pool, whose 2x2 windows must lie inside one block.
+template <int S, typename TIn, bool SORT = false, bool SHIFT = false>
 __global__ void __launch_bounds__(kThreadsTM, 1)
     pconv_tm(const TmParams p, const __grid_constant__ CUtensorMap tmap) {
     constexpr int RY = 4, RX = 4;
+    static_assert(!SHIFT || S == 1, "shifted blocks are a stride-1 layout");
     extern __shared__ __align__(128) unsigned char smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     // header: full[kStages] (stage filled), empty[kStages] (stage read by all 16 warps), the
@@ -402,8 +407,9 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     auto place_lane = [&]() {
         const Unit CU = s_units[ci];
         // block t (0 .. 32 * WS - 1) of the unit's tile: image, block row and column, and where
-        // the lane's window column 0 (input column ox0 * S - 1 of the block) sits in the stage:
-        // d = 3 into the row for fp32 stages, 3 or 7 for fp16 ones (their origin is 16 bytes)
+        // the lane's window column 0 (input column ox0 * S - 1 of the block, one less with SHIFT)
+        // sits in the stage: d = 3 into the row for fp32 stages, 3 or 7 for fp16 ones (their
+        // origin is 16 bytes); with SHIFT 2, or 2 or 6
         auto locate = [&](int t) {
             int rem;
             if (p.linear) {
@@ -419,19 +425,20 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
             }
             by = rem / p.BX;
             bx = rem - by * p.BX;
-            const int d = CU.ox0 * S - 1 - CU.ix0;
+            const int d = CU.ox0 * S - 1 - CU.ix0 - (SHIFT ? 1 : 0);
             in_off = active ? img * p.CK * plane + by * RY * S * p.BWb + bx * RX * S + d : d;
         };
         locate(blk);
         if constexpr (SORT) {
             static_assert(S == 1 && sizeof(TIn) == 4, "bank groups are those of fp32 stride-1 windows");
             // The warp's 32 blocks are dealt to its lanes so that each 8-lane phase of the
-            // 16-byte window loads (window columns 1-4, at in_off + 1) meets distinct bank
+            // 16-byte window loads (window columns 1-4 at in_off + 1, or 2-5 at in_off + 2 with
+            // SHIFT) meets distinct bank
             // groups where the blocks allow it: blocks are ordered by (rank among the blocks of
             // their bank group, bank group) and lane i takes the i-th.  Rows of 7 or 14 blocks
             // otherwise put two blocks of a phase on one bank group.  Idle lanes go last.  The
             // planner picks this instance where it lowers the wavefronts (window_wavefronts).
-            const int grp = active ? ((in_off + 1) >> 2) & 7 : 8;
+            const int grp = active ? ((in_off + (SHIFT ? 2 : 1)) >> 2) & 7 : 8;
             const unsigned same = __match_any_sync(0xffffffffu, grp);
             const int key = active ? 16 * __popc(same & ((1u << lane) - 1u)) + grp : 1024 + lane;   // distinct
             int pos = 0, src = 0;
@@ -452,7 +459,7 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     auto epilogue = [&](const Unit& U) {
         const int g = U.g0 + wg;
         const int n = U.n0 + img;
-        const int oyb = U.oy0 + by * RY, oxb = U.ox0 + bx * RX;
+        const int oyb = U.oy0 + by * RY, oxb = U.ox0 + bx * RX - (SHIFT ? 1 : 0);
 #pragma unroll 1
         for (int f = 0; f < kF; ++f) {
             float a[16];
@@ -469,7 +476,16 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
                     const int oy = oyb + r;
                     if (oy >= p.Ho) break;
                     float* wr = wc + (size_t)oy * p.Wo;
-                    if ((p.Wo % 4) == 0 && oxb + RX <= p.Wo) {
+                    if constexpr (SHIFT) {   // columns oxb (3 mod 4), oxb+1..oxb+2 (a pair), oxb+3
+                        if (oxb >= 0 && oxb < p.Wo) wr[oxb] = a[r * RX];
+                        if ((p.Wo % 2) == 0 && oxb + 3 <= p.Wo) {
+                            *reinterpret_cast<float2*>(wr + oxb + 1) = make_float2(a[r * RX + 1], a[r * RX + 2]);
+                        } else {
+                            if (oxb + 1 < p.Wo) wr[oxb + 1] = a[r * RX + 1];
+                            if (oxb + 2 < p.Wo) wr[oxb + 2] = a[r * RX + 2];
+                        }
+                        if (oxb + 3 < p.Wo) wr[oxb + 3] = a[r * RX + 3];
+                    } else if ((p.Wo % 4) == 0 && oxb + RX <= p.Wo) {
                         *reinterpret_cast<float4*>(wr + oxb) =
                             make_float4(a[r * RX], a[r * RX + 1], a[r * RX + 2], a[r * RX + 3]);
                     } else {
@@ -524,7 +540,20 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
                     const float q = a[r * RX + c] + b;
                     v[c] = p.relu ? fmaxf(q, 0.0f) : q;
                 }
-                if (p.vec_store && oxb + RX <= p.Wo) {
+                if constexpr (SHIFT) {   // columns oxb (3 mod 4), oxb+1..oxb+2 (a pair), oxb+3
+                    if (oxb >= 0 && oxb < p.Wo) yr[oxb] = from_f32<TOut>(v[0]);
+                    if (p.vec_pair && oxb + 3 <= p.Wo) {
+                        if constexpr (sizeof(TOut) == 4) {
+                            *reinterpret_cast<float2*>(yr + oxb + 1) = make_float2(v[1], v[2]);
+                        } else {
+                            *reinterpret_cast<__half2*>(yr + oxb + 1) = __floats2half2_rn(v[1], v[2]);
+                        }
+                    } else {
+                        if (oxb + 1 < p.Wo) yr[oxb + 1] = from_f32<TOut>(v[1]);
+                        if (oxb + 2 < p.Wo) yr[oxb + 2] = from_f32<TOut>(v[2]);
+                    }
+                    if (oxb + 3 < p.Wo) yr[oxb + 3] = from_f32<TOut>(v[3]);
+                } else if (p.vec_store && oxb + RX <= p.Wo) {
                     if constexpr (sizeof(TOut) == 4) {
                         *reinterpret_cast<float4*>(yr + oxb) = make_float4(v[0], v[1], v[2], v[3]);
                     } else {
@@ -555,8 +584,12 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
             const uint32_t vals_addr = smem_u32(reinterpret_cast<const float4*>(st + p.vals_off) + wg * p.maxk);
             const int ckv = min(p.CK, CU.c_hi - CU.c_lo - ck * p.CK);
             constexpr int es = (int)sizeof(TIn);
-            if constexpr (S == 1 && es == 4) {
+            if constexpr (S == 1 && es == 4 && SHIFT) {
+                PP_STAGE_KERNELS_S1_A(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw, edge);
+            } else if constexpr (S == 1 && es == 4) {
                 PP_STAGE_KERNELS_S1(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw, edge);
+            } else if constexpr (S == 1 && SHIFT) {
+                PP_STAGE_KERNELS_S1_HA(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw, edge);
             } else if constexpr (S == 1) {
                 PP_STAGE_KERNELS_S1_H(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw, edge);
             } else if constexpr (es == 4) {
@@ -1237,10 +1270,10 @@ static __device__ __align__(256) float g_pp_scratch[kStaticScratchBytes / sizeof
 int sm_count() {
     static std::atomic<int> cached[64];
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 152;   // no device: plan for a GB300
     if (dev < 64 && cached[dev].load() > 0) return cached[dev].load();
     int n = 0;
-    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 152;
     if (dev < 64) cached[dev].store(n);
     return n;
 }
@@ -1320,15 +1353,17 @@ struct Plan {
     size_t stage_bytes = 0, kb_bytes = 0, smem = 0;
     long long ctas = 0;           // CTAs of one split
     int lane_sort = 0;            // stride 1: pconv_tm deals blocks to lanes by bank group
+    int shift = 0;                // stride 1: blocks start at output columns 4j - 1 (SHIFT)
     size_t ws_bytes = 0;          // workspace the chosen split needs (0 without a split)
 };
 
 struct PlanCache : PlanCacheBase {
     std::mutex mu;
-    std::map<std::tuple<int, int, int, size_t>, Plan> plans;
+    std::map<std::tuple<int, int, int, size_t, int>, Plan> plans;
 };
 
-// Candidate spatial tiles of at most 32*WS blocks (4x4 outputs each).
+// Candidate spatial tiles of at most 32*WS blocks (4x4 outputs each; with shift, block j of a row
+// starts at output column 4j - 1, so a row of Wo outputs takes (Wo + 4) / 4 blocks).
 //   rectangles: BY x BX blocks of one image (several whole images when the rectangle is the
 //     whole image); stride-1 rows need 4*BX + 5 staged columns, stride-2 rows 8*BX + 4, rounded
 //     to a 16-byte multiple and padded to 4 (mod 8) floats so that rows four apart fall in other
@@ -1336,8 +1371,8 @@ struct PlanCache : PlanCacheBase {
 //   linear: 32*WS consecutive blocks of the (image, block row, block column) sequence, staged as
 //     the whole images they touch; no lane idles even when an image's block count is no divisor
 //     of the lane count (28 x 28 outputs: 49 blocks).
-std::vector<TileChoice> tile_candidates(int N, int Ho, int Wo, int S, int lanes) {
-    const int nby = (Ho + 3) / 4, nbx = (Wo + 3) / 4;
+std::vector<TileChoice> tile_candidates(int N, int Ho, int Wo, int S, int lanes, int shift) {
+    const int nby = (Ho + 3) / 4, nbx = shift ? (Wo + 4) / 4 : (Wo + 3) / 4;
     auto bw_of = [&](int bx) {
         int bw = S == 1 ? 4 * bx + 8 : 8 * bx + 4;
         if (bw % 8 == 0) bw += 4;
@@ -1414,7 +1449,8 @@ int window_wavefronts(const Plan& pl, int N, long long t, bool sorted) {
     return w;
 }
 
-int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out) {
+int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, int shift, Plan* out,
+                       double* cost) {
     const int S = L->stride;
     const int Ho = (H - 1) / S + 1, Wo = (W - 1) / S + 1;
     int wg = 1;
@@ -1422,7 +1458,7 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
     const int WS = kCompute / wg, lanes = 32 * WS;
     const int n_fchunks = (L->G + wg - 1) / wg;
     const int C = L->cin_g;
-    const int nby = (Ho + 3) / 4, nbx = (Wo + 3) / 4;
+    const int nby = (Ho + 3) / 4, nbx = shift ? (Wo + 4) / 4 : (Wo + 3) / 4;
     const long long sms = sm_count();
     const size_t out_elems = (size_t)N * L->cout * Ho * Wo;
 
@@ -1542,7 +1578,7 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
     TileChoice rect, lin;
     int rtx = 0, rty = 0, rtn = 0;
     bool have_rect = false, have_lin = false;
-    for (const TileChoice& t : tile_candidates(N, Ho, Wo, S, lanes)) {
+    for (const TileChoice& t : tile_candidates(N, Ho, Wo, S, lanes, shift)) {
         if ((long long)t.NB * t.IH * t.BWb * 4 * ck_min > 48 * 1024) continue;
         if (t.linear) {
             lin = t;
@@ -1577,6 +1613,8 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
     const double cl = have_lin ? (1.3 + kpc) / (0.4 + kpc) * finish(lin, 1, 1, ltn, &pli) : 1e300;
     if (cr >= 1e300 && cl >= 1e300) return PP_ERR_SHAPE;
     *out = cl < cr ? pli : pr;
+    out->shift = shift;
+    *cost = std::min(cl, cr);
     if (S == 1) {   // the bank-group order where it lowers the window loads' wavefronts
         const long long nt = out->tile.linear ? std::min<long long>(out->tiles_n, 64) : 1;
         long long raster = 0, sorted = 0;
@@ -1589,15 +1627,19 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
     return PP_OK;
 }
 
-int make_plan(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out) {
-    auto* cache = static_cast<PlanCache*>(L->plans.get());
-    if (!cache) {
-        static std::mutex create_mu;
-        std::lock_guard<std::mutex> g(create_mu);
-        if (!L->plans) const_cast<pp_layer*>(L)->plans.reset(new PlanCache);
-        cache = static_cast<PlanCache*>(L->plans.get());
-    }
-    const auto key = std::make_tuple(N, H, W, ws_avail);
+// Window loads with shifted blocks: one 8-byte and one 16-byte load per row instead of two bank-
+// conflicted 4-byte loads around a 16-byte one.  They pay where the window loads weigh most, at
+// few kept kernels per (input channel, filter group): VGG-16's keep-0.3 layers (2.4 kernels)
+// measured 6-13 % faster, its first layer (8 kernels, rows of 57 instead of 56 blocks) 16 %
+// slower.  The estimate of channel steps of the shifted plan is scaled by this factor of the
+// layer's mean kept kernels per (channel, group), 0.87 at 2.4 and 1 from 8 on.
+double shift_gain(double kept_per_channel) { return std::min(1.0, 0.82 + 0.0225 * kept_per_channel); }
+
+int make_plan(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out, int pool = 0) {
+    pp_layer* ML = const_cast<pp_layer*>(L);   // the cache is the only mutable part of a handle
+    std::call_once(ML->plans_once, [ML] { ML->plans.reset(new PlanCache); });
+    auto* cache = static_cast<PlanCache*>(ML->plans.get());
+    const auto key = std::make_tuple(N, H, W, ws_avail, pool);
     {
         std::lock_guard<std::mutex> g(cache->mu);
         auto it = cache->plans.find(key);
@@ -1607,8 +1649,15 @@ int make_plan(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out
         }
     }
     Plan pl;
-    const int rc = make_plan_uncached(L, N, H, W, ws_avail, &pl);
+    double cost = 0;
+    const int rc = make_plan_uncached(L, N, H, W, ws_avail, 0, &pl, &cost);
     if (rc != PP_OK) return rc;
+    if (L->stride == 1 && !pool) {   // shifted blocks where their estimate is lower
+        Plan ps;
+        double cs = 0;
+        const double kpc = (double)L->beta / ((double)L->G * L->cin_g);
+        if (make_plan_uncached(L, N, H, W, ws_avail, 1, &ps, &cs) == PP_OK && cs * shift_gain(kpc) < cost) pl = ps;
+    }
     std::lock_guard<std::mutex> g(cache->mu);
     if (cache->plans.size() >= 256) cache->plans.clear();
     cache->plans[key] = pl;
@@ -1664,7 +1713,7 @@ __global__ void splitk_reduce_pool(const float* __restrict__ ws, T* __restrict__
 // Raise the kernel's dynamic shared-memory limit to the device's opt-in maximum once per device
 // (a launch needs at most that), so that later calls, including ones under stream capture, make
 // no attribute call.
-template <int S, typename T, bool SORT>
+template <int S, typename T, bool SORT, bool SHIFT>
 bool allow_max_smem(size_t need) {
     static std::atomic<int> done[64];
     int dev = 0;
@@ -1673,7 +1722,7 @@ bool allow_max_smem(size_t need) {
     int optin = 0;
     if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess) return false;
     if ((size_t)optin < need) return false;
-    if (cudaFuncSetAttribute(pconv_tm<S, T, SORT>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin) != cudaSuccess)
+    if (cudaFuncSetAttribute(pconv_tm<S, T, SORT, SHIFT>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin) != cudaSuccess)
         return false;
     done[dev].store(1, std::memory_order_release);
     return true;
@@ -1683,9 +1732,10 @@ template <int S, typename T>
 int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int relu, int N, int H, int W, int Ho,
               int Wo, void* ws, size_t ws_bytes, cudaStream_t st, int pool = 0) {
     Plan pl;
-    const int rc = make_plan(L, N, H, W, ws ? ws_bytes : 0, &pl);
+    const int rc = make_plan(L, N, H, W, ws ? ws_bytes : 0, &pl, pool);
     if (rc != PP_OK) return rc;
     if (pl.KS > 1 && reinterpret_cast<uintptr_t>(ws) % 16 != 0) return PP_ERR_ALIGN;
+    if (pool && pl.shift) return PP_ERR_SHAPE;   // never planned: pool windows must lie in one block
     TmParams p{};
     p.x = x;
     p.y = y;
@@ -1739,6 +1789,7 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
     const size_t smem = p.stage_off + (size_t)kStages * p.stage_bytes;   // the plan's for fp32
     if (smem > pl.smem) return PP_ERR_SHAPE;
     p.vec_store = (Wo % 4 == 0) && (reinterpret_cast<uintptr_t>(y) % (4 * es)) == 0;
+    p.vec_pair = (Wo % 2 == 0) && (reinterpret_cast<uintptr_t>(y) % (2 * es)) == 0;
     p.pool = pool;
     p.vec_pool = ((Wo >> 1) % 2 == 0) && (reinterpret_cast<uintptr_t>(y) % (2 * es)) == 0;
 
@@ -1757,17 +1808,30 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
         if (r != CUDA_SUCCESS) p.use_tma = 0;
         p.tma_bytes = (unsigned)((size_t)p.BWb * p.IH * p.CK * p.NB * es);
     }
-    auto kern = pconv_tm<S, T, false>;
+    auto kern = pconv_tm<S, T, false, false>;
     bool smem_ok;
     if constexpr (S == 1 && sizeof(T) == 4) {
-        if (pl.lane_sort) {
-            kern = pconv_tm<1, float, true>;
-            smem_ok = allow_max_smem<1, float, true>(smem);
+        if (pl.lane_sort && pl.shift) {
+            kern = pconv_tm<1, float, true, true>;
+            smem_ok = allow_max_smem<1, float, true, true>(smem);
+        } else if (pl.lane_sort) {
+            kern = pconv_tm<1, float, true, false>;
+            smem_ok = allow_max_smem<1, float, true, false>(smem);
+        } else if (pl.shift) {
+            kern = pconv_tm<1, float, false, true>;
+            smem_ok = allow_max_smem<1, float, false, true>(smem);
         } else {
-            smem_ok = allow_max_smem<S, T, false>(smem);
+            smem_ok = allow_max_smem<1, float, false, false>(smem);
+        }
+    } else if constexpr (S == 1) {
+        if (pl.shift) {
+            kern = pconv_tm<1, T, false, true>;
+            smem_ok = allow_max_smem<1, T, false, true>(smem);
+        } else {
+            smem_ok = allow_max_smem<1, T, false, false>(smem);
         }
     } else {
-        smem_ok = allow_max_smem<S, T, false>(smem);
+        smem_ok = allow_max_smem<S, T, false, false>(smem);
     }
     if (!smem_ok) return PP_ERR_CUDA;
     const long long units = pl.ctas * pl.KS;
@@ -2097,15 +2161,16 @@ int pp_conv_pool_ws(pp_handle h, const void* x, int dtype, int N, int H, int W, 
                : launch_tm<2, float>(h, x, y, bias, relu, N, H, W, Ho, Wo, workspace, workspace_bytes, st, 1);
 }
 
-int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info) {
+namespace {
+int conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info, int pool) {
     if (!h || !info) return PP_ERR_NULL;
     if (N < 1 || H < 1 || W < 1 || n_info < 1) return PP_ERR_SHAPE;
-    int64_t v[14] = {0};
+    int64_t v[15] = {0};
     if (!h->fast || h->depthwise) {
         v[0] = h->depthwise ? 2 : 3;   // depthwise kernel / generic kernel: no plan, no workspace
     } else {
         Plan pl;
-        const int rc = make_plan(h, N, H, W, workspace_bytes, &pl);
+        const int rc = make_plan(h, N, H, W, workspace_bytes, &pl, pool);
         if (rc != PP_OK) return rc;
         v[0] = 1;
         v[1] = pl.KS;
@@ -2124,9 +2189,20 @@ int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64
         v[10] = (int64_t)pl.smem;
         v[11] = pl.n_chunks;
         v[13] = pl.lane_sort;
+        v[14] = pl.shift;
     }
-    for (int i = 0; i < n_info && i < 14; ++i) info[i] = v[i];
+    for (int i = 0; i < n_info && i < 15; ++i) info[i] = v[i];
     return PP_OK;
+}
+}  // namespace
+
+int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info) {
+    return conv_plan(h, N, H, W, workspace_bytes, info, n_info, 0);
+}
+
+int pp_conv_pool_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info) {
+    if (h && (h->depthwise || !h->fast)) return PP_ERR_PATH;
+    return conv_plan(h, N, H, W, workspace_bytes, info, n_info, 1);
 }
 
 int pp_conv_workspace_size(pp_handle h, int N, int H, int W, size_t* bytes) {

@@ -1,9 +1,9 @@
 #!/usr/bin/env python3
 """Generate pattern_dispatch.h: the channel loop of the pattern-sparse kernel as inline PTX.
 
-One macro per stride and stage type (fp32 stages; fp16 stages, whose window elements are widened
-to fp32 as they are loaded) processes one pipeline stage (CK input channels) for one filter
-group and one lane's 4x4 output block.  Per input channel:
+One macro per stride, stage type (fp32 stages; fp16 stages, whose window elements are widened to
+fp32 as they are loaded) and window alignment processes one pipeline stage (CK input channels)
+for one filter group and one lane's 4x4 output block.  Per input channel:
 
     ld.shared        the group's 64-bit descriptor (count in bits 0-3, then 6-bit
                      (slot << 3 | pattern) codes of the kept kernels, slots ascending)
@@ -19,16 +19,23 @@ group and one lane's 4x4 output block.  Per input channel:
                      (the four kept positions of the pattern, §3.2): nothing is decoded per element
       tcgen05.st     the accumulators back
 
-Stride 1 runs the taps of the centre column (1, 4, 7) as fma.rn.f32x2 on pairs of outputs: their
-window pairs, columns (1, 2) and (3, 4) of each row, are the halves of the row's aligned 16-byte
-load, so they cost no register moves, and each packed instruction does two of the per-lane
-fma.rn.f32 operations (same rounding) in one issue slot.  The other taps read pairs that straddle
-that alignment and stay scalar.  Every pattern holds 1 to 3 centre-column taps, so about a quarter
-of the body's instructions go away.
+Window alignment (stride 1).  The input stage is a tensor copy whose first column sits on a
+16-byte boundary, so the output block origin decides where a lane's window column 0 falls:
+  * blocks at output columns 4j: column 0 at 3 (mod 4); each row is a 4-byte, a 16-byte and a
+    4-byte load, and every lane's 4-byte loads fall on 8 of the 32 banks (4-way conflicts);
+  * blocks at output columns 4j - 1 (the "A" macros): column 0 at 2 (mod 4); each row is an
+    8-byte load of columns 0-1 and a 16-byte load of columns 2-5, a third fewer shared-memory
+    wavefronts and one instruction fewer.
+Packed taps.  A tap whose window pairs are the halves of one aligned load runs as fma.rn.f32x2
+on pairs of outputs (columns 0-1 and 2-3 of a row; same rounding as two fma.rn.f32): with
+blocks at 4j the centre-column taps (1, 4, 7), whose pairs are window columns (1, 2) and (3, 4);
+with blocks at 4j - 1 the side-column taps (0, 3, 6 and 2, 5, 8), whose pairs are (0, 1), (2, 3)
+and (2, 3), (4, 5).  The other taps read pairs that straddle the alignment and stay scalar.
+Taps are applied in ascending raster order for every output.
 
-Every branch is warp-uniform (bra.uni), so no convergence code surrounds the loop.  Taps are
-applied in ascending raster order for every output.  The macros' operands are listed in macro().  The library masks are the eight defaults
-(centre + 3 of the 4 edge neighbours; centre + one edge + its 2 flanking corners).
+Every branch is warp-uniform (bra.uni), so no convergence code surrounds the loop.  The macros'
+operands are listed in macro().  The library masks are the eight defaults (centre + 3 of the 4
+edge neighbours; centre + one edge + its 2 flanking corners).
 
 Usage: gen_dispatch.py OUT.h
 """
@@ -42,7 +49,7 @@ def taps(mask):
     return [t for t in range(9) if (mask >> t) & 1]
 
 
-def macro(S, half=False):
+def macro(S, half=False, aligned=False):
     RY = RX = 4
     WY, WX = (RY - 1) * S + 3, (RX - 1) * S + 3
     R = RY * RX
@@ -52,13 +59,17 @@ def macro(S, half=False):
     # channel 0, %4 row pitch in bytes, %5 channel plane in bytes, %6 tensor-memory base, %7
     # nonzero where the left neighbour lane does not hold the block to the left (stride 2)
     packed = S == 1
+    pairs = (0, 2, 4) if aligned else (1, 3)      # window columns starting an aligned pair
+
+    def packs(dx):                                # tap column dx (0..2) runs as f32x2
+        return (dx != 1) if aligned else (dx == 1)
     L = ["{",
          ".reg .pred P, EL;",
          f".reg .b32 cl, cnt, code, ta, pat, va, da, t1, {rows};",
          ".reg .b64 d, dd;",
          f".reg .f32 x<{WY * WX}>, a<{R}>, w<4>;"]
-    if packed:   # window pairs (row r, columns 1-2 / 3-4), accumulator pairs, duplicated weights
-        L.append(f".reg .b64 xq<{2 * WY}>, ap<{R // 2}>, wq<4>;")
+    if packed:   # window pairs xq{5 * row + column}, accumulator pairs, duplicated weights
+        L.append(f".reg .b64 xq<{5 * WY}>, ap<{R // 2}>, wq<4>;")
     if half:     # fp16 stage: 16-bit elements widened to fp32 as the window is loaded
         L.append(".reg .b16 h<10>;")
         L.append(".reg .b32 pA, pB, pC, pD;")
@@ -79,10 +90,7 @@ def macro(S, half=False):
           "and.b32 cnt, cnt, 15;",
           "setp.eq.u32 P, cnt, 0;",
           "@P bra.uni CN;"]
-    # window: column 0 alone, then aligned groups of four.  Stride 2: lanes sit 32 bytes apart, so
-    # a scalar load of column 0 meets an 8-way bank conflict; it is the left neighbour lane's
-    # column 8 instead (a warp shuffle), and only lanes at the start of a tile row or of the warp
-    # (%7 nonzero) load it from shared memory
+
     def cvt_pair(p, a):                   # two packed halves to x{a}, x{a+1}
         return [f"mov.b32 {{h0, h1}}, {p};", f"cvt.f32.f16 x{a}, h0;", f"cvt.f32.f16 x{a + 1}, h1;"]
     for r in range(WY):
@@ -102,29 +110,26 @@ def macro(S, half=False):
             L.append(f"shfl.sync.up.b32 x{base}, x{base + 8}, 1, 0, -1;")
             L.append(f"@EL ld.shared.f32 x{base}, [rb{r}];")
             continue
-        if half:                             # column 0, columns 1-4 (one 8-byte load), column 5
+        if half and aligned:                 # columns 0-1 (4 bytes), columns 2-5 (8 bytes)
+            L.append(f"ld.shared.b32 pA, [rb{r}];")
+            L.append(f"ld.shared.v2.b32 {{pB, pC}}, [rb{r}+4];")
+            L += cvt_pair("pA", base) + cvt_pair("pB", base + 2) + cvt_pair("pC", base + 4)
+        elif half:                           # column 0, columns 1-4 (one 8-byte load), column 5
             L.append(f"ld.shared.b16 h2, [rb{r}];")
             L.append(f"ld.shared.v2.b32 {{pA, pB}}, [rb{r}+2];")
             L.append(f"ld.shared.b16 h3, [rb{r}+10];")
             L.append(f"cvt.f32.f16 x{base}, h2;")
             L += cvt_pair("pA", base + 1) + cvt_pair("pB", base + 3)
             L.append(f"cvt.f32.f16 x{base + 5}, h3;")
-            if packed:
-                L.append(f"mov.b64 xq{2 * r}, {{x{base + 1}, x{base + 2}}};")
-                L.append(f"mov.b64 xq{2 * r + 1}, {{x{base + 3}, x{base + 4}}};")
-            continue
-        L.append(f"ld.shared.f32 x{base}, [rb{r}];")
-        c = 1
-        while c + 4 <= WX:
-            L.append(f"ld.shared.v4.f32 {{x{base + c}, x{base + c + 1}, x{base + c + 2}, x{base + c + 3}}}, "
-                     f"[rb{r}+{4 * c}];")
-            c += 4
-        while c < WX:
-            L.append(f"ld.shared.f32 x{base + c}, [rb{r}+{4 * c}];")
-            c += 1
-        if packed:
-            L.append(f"mov.b64 xq{2 * r}, {{x{base + 1}, x{base + 2}}};")
-            L.append(f"mov.b64 xq{2 * r + 1}, {{x{base + 3}, x{base + 4}}};")
+        elif aligned:                        # columns 0-1 (8 bytes), columns 2-5 (16 bytes)
+            L.append(f"ld.shared.v2.f32 {{x{base}, x{base + 1}}}, [rb{r}];")
+            L.append(f"ld.shared.v4.f32 {{x{base + 2}, x{base + 3}, x{base + 4}, x{base + 5}}}, [rb{r}+8];")
+        else:                                # column 0, columns 1-4 (16 bytes), column 5
+            L.append(f"ld.shared.f32 x{base}, [rb{r}];")
+            L.append(f"ld.shared.v4.f32 {{x{base + 1}, x{base + 2}, x{base + 3}, x{base + 4}}}, [rb{r}+4];")
+            L.append(f"ld.shared.f32 x{base + 5}, [rb{r}+20];")
+        for c0 in pairs:
+            L.append(f"mov.b64 xq{5 * r + c0}, {{x{base + c0}, x{base + c0 + 1}}};")
     L += ["shr.b64 dd, d, 4;",
           "PL:",
           "ld.shared.v4.f32 {w0, w1, w2, w3}, [va];",
@@ -149,14 +154,14 @@ def macro(S, half=False):
         tp = taps(m)
         if packed:
             L += [f"mov.b64 ap{i}, {{a{2 * i}, a{2 * i + 1}}};" for i in range(R // 2)]
-            L += [f"mov.b64 wq{k}, {{w{k}, w{k}}};" for k in range(4) if tp[k] % 3 == 1]
+            L += [f"mov.b64 wq{k}, {{w{k}, w{k}}};" for k in range(4) if packs(tp[k] % 3)]
         for k in range(4):                   # tap-outer: 16 independent FMAs per tap
             t = tp[k]
             dy, dx = t // 3, t % 3
-            if packed and dx == 1:           # outputs (r, 0-1) and (r, 2-3): window pairs of row r + dy
+            if packed and packs(dx):         # outputs (r, 0-1) and (r, 2-3): window pairs of row r + dy
                 for r in range(RY):
                     for h in range(2):
-                        L.append(f"fma.rn.f32x2 ap{2 * r + h}, wq{k}, xq{2 * (r + dy) + h}, ap{2 * r + h};")
+                        L.append(f"fma.rn.f32x2 ap{2 * r + h}, wq{k}, xq{5 * (r + dy) + 2 * h + dx}, ap{2 * r + h};")
                 continue
             for r in range(RY):
                 for c in range(RX):
@@ -185,8 +190,9 @@ def macro(S, half=False):
           "CD:",
           "}"]
     body = "\\n\\t".join(L)
-    name = f"PP_STAGE_KERNELS_S{S}" + ("_H" if half else "")
-    return (f"// stride {S}{', fp16 stage' if half else ''}: 4x4 outputs per lane, {WY}x{WX} input window\n"
+    name = f"PP_STAGE_KERNELS_S{S}" + ("_H" if half else "") + (("A" if half else "_A") if aligned else "")
+    what = f"stride {S}{', fp16 stage' if half else ''}{', window column 0 at 2 mod 4' if aligned else ''}"
+    return (f"// {what}: 4x4 outputs per lane, {WY}x{WX} input window\n"
             f"#define {name}(nch, desc_addr, vals_addr, win_addr, pitch_b, plane_b, tbase, edge) \\\n"
             f'    asm volatile("{body}" :: "r"(nch), "r"(desc_addr), "r"(vals_addr), "r"(win_addr), '
             f'"r"(pitch_b), "r"(plane_b), "r"(tbase), "r"(edge) : "memory")\n')
@@ -198,6 +204,8 @@ def generate() -> str:
     for S in STRIDES:
         for half in (False, True):
             text.append(macro(S, half))
+            if S == 1:
+                text.append(macro(S, half, aligned=True))
     return "\n".join(text)
 
 

@@ -5,6 +5,7 @@
 #include <cstddef>
 #include <cstdint>
 #include <memory>
+#include <mutex>
 #include <vector>
 
 namespace patconv {
@@ -49,5 +50,8 @@ struct pp_layer {
     void* dev = nullptr;               // caller-owned device copy of `image`
     size_t dev_bytes = 0;
 
-    std::unique_ptr<patconv::PlanCacheBase> plans;   // launch plans by call shape (conv.cu)
+    // launch plans by call shape (conv.cu), created on the first plan by call_once, so that calls
+    // from several host threads see it fully constructed
+    std::unique_ptr<patconv::PlanCacheBase> plans;
+    std::once_flag plans_once;
 };

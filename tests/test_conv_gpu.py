@@ -348,20 +348,21 @@ def test_conv_pool_fused(dtype, N, Cin, Cout, H, W, stride, relu):
 
 
 def test_conv_pool_fused_with_split_equals_unfused_pool():
-    """Small images with a workspace: the split path pools in its reduction; the result equals
-    pp_conv_ws followed by the library's max-pool bit for bit (same sums, same order)."""
+    """Small images with a workspace: the split path pools in its reduction; the result matches
+    pp_conv_ws followed by the library's max-pool (the two calls may plan different splits, so
+    their fp32 sums differ only in rounding order) and the oracle."""
     L = WL.vgg16()[12]                                     # 512 -> 512 at 14x14, pooled
     W, b = WL.weights(L), WL.bias(L)
     x = torch.from_numpy(WL.layer_input(L, 16)).cuda()
     bt = torch.from_numpy(b).cuda()
     layer = api.pp_pack(W, None, L.keep).bind("cuda")
-    nb = layer.workspace_bytes(x.shape)
-    assert nb > 0 and layer.plan(x.shape, nb)["splits"] > 1
+    nb = max(layer.workspace_bytes(x.shape, pool2x2=True), layer.workspace_bytes(x.shape))
+    assert layer.plan(x.shape, nb, pool2x2=True)["splits"] > 1
     ws = torch.full((nb // 4,), float("nan"), device="cuda")
     fused = layer.conv(x, bt, True, workspace=ws, pool2x2=True)
     plain = api.pp_maxpool2x2(layer.conv(x, bt, True, workspace=ws))
-    assert torch.equal(fused, plain)
     ref, den = _pool_ref(W, x[:2].cpu().numpy(), b, L.keep, 1, True)
+    assert OC.max_norm_err(fused[:2].double().cpu().numpy(), plain[:2].double().cpu().numpy(), den) <= 1e-5
     assert OC.max_norm_err(fused[:2].double().cpu().numpy(), ref, den) <= 1e-4
 
 
@@ -374,7 +375,7 @@ def test_vgg16_pool_layer_fused_batch32(idx):
     W, b = WL.weights(L), WL.bias(L)
     layer = api.pp_pack(W, None, L.keep).bind("cuda")
     xt = torch.from_numpy(x).cuda()
-    nb = layer.workspace_bytes(xt.shape)
+    nb = layer.workspace_bytes(xt.shape, pool2x2=True)
     ws = torch.empty(max(nb // 4, 1), device="cuda") if nb else None
     y = layer.conv(xt, torch.from_numpy(b).cuda(), True, workspace=ws, pool2x2=True)
     ref, den = _pool_ref(W, x[[0, 31]], b, L.keep, 1, True)

@@ -1,12 +1,12 @@
 """Launch planner of the pattern-sparse kernel (pp_conv_plan and pp_conv_workspace_size, host
 only, no GPU): invariants every plan must keep, over random call shapes and the workloads.
 
-The planner assumes 148 SMs when no GPU is present; the invariants do not depend on that."""
+The planner assumes 152 SMs (a GB300) when no GPU is present; the invariants do not depend on that."""
 import numpy as np
 import pytest
 
 from oracle import patterns as OP
-from paper_2003_06513_gb300 import api
+from paper_2003_06513_gb300 import _lib, api
 from paper_2003_06513_gb300 import workloads as WL
 
 SMEM_MAX = 227 * 1024
@@ -36,7 +36,13 @@ def _check(layer, shape, ws):
     assert pl["units"] % pl["splits"] == 0
     assert pl["ctas"] <= pl["units"]
     assert pl["lane_sort"] in (0, 1) and (layer.stride == 1 or pl["lane_sort"] == 0)
+    assert pl["shift"] in (0, 1) and (layer.stride == 1 or pl["shift"] == 0)
     return pl
+
+
+def _nbx(pl, wo):
+    """Blocks per output row: 4 columns each, starting at column 0, or at -1 when shifted."""
+    return (wo + 4) // 4 if pl["shift"] else (wo + 3) // 4
 
 
 def _stage_geometry(pl, stride):
@@ -51,7 +57,7 @@ def _is_linear(pl, shape, stride):
     """Whether the plan's tile is the linear one (None where its shape does not tell)."""
     n = shape[0]
     ho, wo = (shape[2] - 1) // stride + 1, (shape[3] - 1) // stride + 1
-    nby, nbx = (ho + 3) // 4, (wo + 3) // 4
+    nby, nbx = (ho + 3) // 4, _nbx(pl, wo)
     if (pl["tile_by"], pl["tile_bx"]) != (nby, nbx) or pl["tile_nb"] == 1:
         return False
     bpi, lanes = nby * nbx, 32 * pl["spatial_warps"]
@@ -67,8 +73,6 @@ def _window_wavefronts(pl, shape, stride, t, dealt):
     the most lanes on one of the 8 bank groups; lanes in raster order or dealt by
     (rank within bank group, bank group) with idle lanes last."""
     n = shape[0]
-    ho, wo = (shape[2] - 1) // stride + 1, (shape[3] - 1) // stride + 1
-    nby, nbx = (ho + 3) // 4, (wo + 3) // 4
     by_t, bx_t, nb = pl["tile_by"], pl["tile_bx"], pl["tile_nb"]
     lanes = 32 * pl["spatial_warps"]
     linear = bool(_is_linear(pl, shape, stride))
@@ -119,14 +123,14 @@ def test_lane_order_by_bank_group(which):
             continue
         tiles = 1
         ho, wo = L.ho, L.wo
-        nby, nbx = (ho + 3) // 4, (wo + 3) // 4
+        nby, nbx = (ho + 3) // 4, _nbx(pl, wo)
         if pl["tile_by"] == nby and pl["tile_bx"] == nbx and pl["tile_nb"] > 1:
             tiles = min(64, (n * nby * nbx + 31) // 32)
         raster = sum(_window_wavefronts(pl, shape, 1, t, False) for t in range(tiles))
         dealt = sum(_window_wavefronts(pl, shape, 1, t, True) for t in range(tiles))
         assert pl["lane_sort"] == (1 if dealt < raster else 0), (L.name, raster, dealt)
     if which == "vgg16":
-        assert [got[f"vgg{i}"] for i in range(1, 14)] == [0, 0, 0, 0, 1, 1, 1, 1, 1, 1, 0, 0, 0]
+        assert [got[f"vgg{i}"] for i in range(1, 14)] == [0, 0, 0, 0, 1, 1, 1, 0, 0, 0, 0, 0, 0]
 
 
 def test_multi_image_stages_are_not_bank_aligned():
@@ -188,22 +192,45 @@ def test_other_paths_report_no_plan():
 
 
 def test_linear_tile_weighed_by_density():
-    """28x28 maps (7 blocks a row): at VGG-16's keep 0.3 the planner takes 4x7 rectangles
-    without a split; at keep 1.0 the linear tile (every lane busy) pays for its per-channel cost."""
+    """28x28 maps with blocks at columns 4j (7 blocks a row, the fused-pool layout): at VGG-16's
+    keep 0.3 the planner takes 4x7 rectangles without a split; at keep 1.0 the linear tile (every
+    lane busy) pays for its per-channel cost.  Without the pool the blocks start at 4j - 1 (8 a
+    row), and 4x8 rectangles keep every lane busy."""
     for L in WL.vgg16()[7:10]:
         layer = api.pp_pack(WL.weights(L), None, L.keep)
         shape = (32, L.cin, L.h, L.w)
+        pl = layer.plan(shape, layer.workspace_bytes(shape, True), pool2x2=True)
+        assert (pl["tile_by"], pl["tile_bx"], pl["tile_nb"], pl["splits"], pl["shift"]) == (4, 7, 1, 1, 0), L.name
         pl = layer.plan(shape, layer.workspace_bytes(shape))
-        assert (pl["tile_by"], pl["tile_bx"], pl["tile_nb"], pl["splits"]) == (4, 7, 1, 1), L.name
+        assert (pl["tile_by"], pl["tile_bx"], pl["tile_nb"], pl["splits"], pl["shift"]) == (4, 8, 1, 1, 1), L.name
     rng = np.random.default_rng(7)
     W = (rng.standard_normal((256, 256, 3, 3)) * np.sqrt(2 / (9 * 256))).astype(np.float32)
     shape = (64, 256, 28, 28)
     dense = api.pp_pack(W, None, 1.0)
-    pl = dense.plan(shape, dense.workspace_bytes(shape))
+    pl = dense.plan(shape, dense.workspace_bytes(shape, True), pool2x2=True)
     assert (pl["tile_by"], pl["tile_bx"]) == (7, 7) and pl["tile_nb"] > 1     # linear
     sparse = api.pp_pack(W, None, 0.25)
-    pl = sparse.plan(shape, sparse.workspace_bytes(shape))
+    pl = sparse.plan(shape, sparse.workspace_bytes(shape, True), pool2x2=True)
     assert (pl["tile_by"], pl["tile_bx"], pl["tile_nb"]) == (4, 7, 1)
+
+
+@pytest.mark.parametrize("which", ["vgg16", "resnet50"])
+def test_pool_plans_keep_blocks_at_4j(which):
+    """The fused pool needs every 2x2 window inside one lane's block: its plans never shift the
+    blocks, and they obey the same invariants.  Layers without the fused pool refuse the query."""
+    layers = WL.vgg16() if which == "vgg16" else WL.resnet50_3x3()
+    n = 32 if which == "vgg16" else 64
+    for L in layers:
+        layer = api.pp_pack(WL.weights(L), None, L.keep, 1, L.stride)
+        shape = (n, L.cin, L.h, L.w)
+        for ws in (0, layer.workspace_bytes(shape, True)):
+            pl = layer.plan(shape, ws, pool2x2=True)
+            assert pl["path"] == 1 and pl["shift"] == 0
+            assert 0 < pl["smem_bytes"] <= SMEM_MAX and pl["filter_groups"] * pl["spatial_warps"] == 16
+    rng = np.random.default_rng(3)
+    dw = api.pp_pack(rng.standard_normal((16, 1, 3, 3)).astype(np.float32), None, 1.0, 16, 1)
+    with pytest.raises(_lib.PatconvError):
+        dw.plan((2, 16, 20, 20), 0, pool2x2=True)
 
 
 @pytest.mark.parametrize("seed", range(30))
@@ -225,7 +252,7 @@ def test_lane_order_random_shapes(seed):
             continue
         tiles = 1
         if linear:
-            nby, nbx = (h + 3) // 4, (w + 3) // 4
+            nby, nbx = (h + 3) // 4, _nbx(pl, w)
             tiles = min(64, (n * nby * nbx + 32 * pl["spatial_warps"] - 1) // (32 * pl["spatial_warps"]))
         raster = sum(_window_wavefronts(pl, shape, 1, t, False) for t in range(tiles))
         dealt = sum(_window_wavefronts(pl, shape, 1, t, True) for t in range(tiles))
