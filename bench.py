@@ -259,7 +259,8 @@ def reference_arm(args, rank, world):
             "ms_per_step": 1e3 * t_total / max(k_done, 1), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": config_dict(),
-            "cpu_baseline": {"value": value, "unit": "img/s", "cores": threads, "kind": "oracle",
+            "cpu_baseline": {"value": value, "unit": "img/s", "cores": threads, "cpu_count": os.cpu_count(),
+                             "kind": "oracle",
                              "sample": "1 image through the 13-layer stack per step (numpy float64)"},
             "e2e": {"value": value, "unit": "img/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
@@ -269,7 +270,8 @@ def reference_arm(args, rank, world):
 # ------------------------------------------------------------------------------ our arm
 
 def fp32_peak(props, clocks):
-    """FP32 CUDA-core peak: SMs x 128 FMA lanes x 2 FLOP x max SM clock."""
+    """Nominal FP32 CUDA-core peak (context beside the measured one): SMs x 128 FMA lanes x 2 FLOP
+    x max SM clock."""
     mhz = None
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -279,6 +281,29 @@ def fp32_peak(props, clocks):
     if not mhz:
         mhz = clocks.get("sm_max_mhz") or 2070.0
     return props.multi_processor_count * 128 * 2 * mhz * 1e6, mhz
+
+
+_MEASURED_PEAK = {}
+
+
+def measured_fp32_peak(dev):
+    """The FP32 FMA peak measured on this GPU by the library (independent FFMA chains on every SM,
+    best of 50 launches of about 2 ms, CUDA events), the clocks sampled meanwhile, and a one-line
+    basis; cached per device."""
+    import torch
+    from paper_2003_06513_gb300 import api
+    key = int(getattr(dev, "index", dev) or 0)
+    if key not in _MEASURED_PEAK:
+        with torch.cuda.device(key), ClockSampler(key) as clk:
+            peak = api.measure_fp32_peak(50)
+        props = torch.cuda.get_device_properties(key)
+        nominal, mhz = fp32_peak(props, {})
+        cl = clk.summary()
+        basis = (f"measured: FFMA chains on {props.multi_processor_count} SMs, best of 50 x ~2 ms "
+                 f"(SM clock median {cl.get('sm_mhz')} MHz); nominal {nominal / 1e12:.1f} TFLOP/s = "
+                 f"{props.multi_processor_count} SMs x 128 x 2 x {mhz:.0f} MHz")
+        _MEASURED_PEAK[key] = (peak, basis, cl, nominal)
+    return _MEASURED_PEAK[key]
 
 
 def hbm_peak():
@@ -404,6 +429,8 @@ def our_arm(args, rank, world, local_rank):
     for _ in range(max(args.warmup, 3)):
         step(x0)
     barrier()
+    peak_meas, peak_basis, peak_clocks, peak_nominal = measured_fp32_peak(dev)   # the roofline denominator
+    barrier()
 
     K = args.steps
     launches_per_step = len(layers) + sum(
@@ -495,9 +522,8 @@ def our_arm(args, rank, world, local_rank):
     elapsed_ms, e2e_ms, graph_ms = max_over_ranks(dist, [elapsed_ms, e2e_ms, graph_ms], dev)
 
     if rank == 0:
-        props = torch.cuda.get_device_properties(dev)
         clocks = clk.summary()
-        peak, mhz = fp32_peak(props, clocks)
+        peak = peak_meas
         hbm, hbm_kind = hbm_peak()
         flops = [c[0] for c in costs]
         bytes_ = [c[1] for c in costs]
@@ -519,8 +545,8 @@ def our_arm(args, rank, world, local_rank):
             "network_roofline_frac": roof_ms / tot_conv_ms,
             "roofline": {"bound": "alu", "kernel": "pconv_tm<1,float,SORT> (+ split reduce)",
                          "achieved": achieved / 1e12, "peak": peak / 1e12, "unit": "TFLOP/s",
-                         "frac": achieved / peak,
-                         "peak_basis": f"{props.multi_processor_count} SMs x 128 FP32 lanes x 2 x {mhz:.0f} MHz",
+                         "frac": achieved / peak, "peak_kind": "measured", "peak_basis": peak_basis,
+                         "peak_nominal": peak_nominal / 1e12, "peak_clocks": peak_clocks,
                          "traffic": (trec or {}).get("dram_bytes_per_launch"),
                          "algorithmic_bytes_per_launch": sum(bytes_) / len(bytes_),
                          "hbm_peak_gbs": hbm / 1e9, "hbm_peak_kind": hbm_kind},
@@ -549,7 +575,8 @@ def our_arm(args, rank, world, local_rank):
                                                    "weights + bias + ReLU, max_pool2d; fp32, TF32 off"}
         if world == 1 and not args.no_cpu_baseline:
             n, dt, thr = oracle_forward_images(args.cpu_seconds, max_images=BATCH)
-            line["cpu_baseline"] = {"value": n / dt, "unit": "img/s", "cores": thr, "kind": "oracle",
+            line["cpu_baseline"] = {"value": n / dt, "unit": "img/s", "cores": thr, "cpu_count": os.cpu_count(),
+                                    "kind": "oracle",
                                     "sample": f"{n} image(s) through the 13-layer stack, numpy float64"}
         print(json.dumps(line), flush=True)
     if dist is not None:
@@ -640,11 +667,9 @@ def dense_context(packed, biases, layers, x0, K, barrier):
 
 
 def _peaks(dev):
-    import torch
-    props = torch.cuda.get_device_properties(dev)
-    peak, mhz = fp32_peak(props, {})
+    peak, basis, _, _ = measured_fp32_peak(dev)
     hbm, kind = hbm_peak()
-    return peak, hbm, kind, f"{props.multi_processor_count} SMs x 128 FP32 lanes x 2 x {mhz:.0f} MHz"
+    return peak, hbm, kind, basis
 
 
 def _time_layer(lay, x, b, relu, ws, K, warmup=3):
@@ -731,7 +756,7 @@ def layer_suite(args):
     if which == "single" and not args.no_cpu_baseline:
         orc = oracle_single_layer()
         line["cpu_baseline"] = {"value": tot_flops / (orc[0]["ms"] * 1e-3) / 1e9, "unit": "GFLOP/s",
-                                "cores": orc[0]["threads"], "kind": "oracle",
+                                "cores": orc[0]["threads"], "cpu_count": os.cpu_count(), "kind": "oracle",
                                 "sample": "the whole layer, median of up to 30 runs (numpy float64)",
                                 "rows": orc}
     print(json.dumps(line), flush=True)

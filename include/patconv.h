@@ -213,12 +213,18 @@ int pp_conv_pool_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, 
  * exits.  Nothing is allocated and no allocating routine is called.
  *   - the first call on a device looks up the array's device address (once per device, with
  *     that device current); make that first call before any stream capture;
- *   - a call whose split would need more scratch than the array holds (see
- *     pp_conv_workspace_size) returns PP_ERR_SCRATCH without launching anything;
+ *   - the call runs the plan pp_conv_ws would run with an unlimited workspace; where that plan's
+ *     split needs more scratch than the array holds (pp_conv_workspace_size reports the need)
+ *     it returns PP_ERR_SCRATCH without launching anything, rather than falling back to a plan
+ *     that fits.  Such shapes (wide layers on many small images) are rejected here although
+ *     pp_conv, which never splits, and pp_conv_ws with a smaller workspace accept them;
+ *   - the argument errors of pp_conv_ws (PP_ERR_NULL, _ARG, _ALIGN, _BUFFER, ...) are checked
+ *     first and take precedence over PP_ERR_SCRATCH;
  *   - every call on a device shares the one array, which keeps the previous call's contents;
- *     nothing needs clearing (each call writes every partial sum it reads), but calls that
- *     overlap on the GPU (different streams, or different host threads) race on it: order them;
- *   - otherwise identical to pp_conv_ws (same plan, same result, same errors). */
+ *     nothing needs clearing (each call writes every partial sum it reads before reading it),
+ *     but calls that overlap on the GPU (different streams, or different host threads) race on
+ *     it: order them;
+ *   - otherwise identical to pp_conv_ws with an unlimited workspace (same plan, same result). */
 #define PP_STATIC_SCRATCH_BYTES 33554432
 int pp_conv_static_scratch(pp_handle h, const void* x, int dtype, int N, int H, int W,
                            const float* bias, int relu, void* y, void* stream);
@@ -238,6 +244,22 @@ int pp_maxpool2x2(const void* x, int dtype, int N, int C, int H, int W, void* y,
  * (a device-to-host copy); call it between launches, e.g. at the end of a test.
  * Errors: PP_ERR_NULL, PP_ERR_CUDA. */
 int pp_device_status(int clear, unsigned int* status);
+
+/* Measured FP32 fused multiply-add peak of the current device in FLOP/s (2 per FMA), the
+ * roofline denominator of the dense kernel (the paper has no counterpart): independent
+ * fma.rn.f32 chains on every SM, no memory traffic, timed with CUDA events on the legacy default
+ * stream, best of `reps` launches of about 2 ms after one warm-up launch.  Synchronous.
+ * Errors: PP_ERR_NULL, PP_ERR_ARG (reps outside 1..1000), PP_ERR_CUDA. */
+int pp_measure_fp32_peak(int reps, double* flop_per_s);
+
+/* Test hook for the failure path above (the paper has no counterpart): the next launch of the
+ * dense pattern-sparse kernel, from any thread, issues none of its input-stage copies and waits
+ * only about 10 us for them, so the first pipeline wait of every CTA runs out.  That launch
+ * records bit 1 in the status word, writes nothing to y (the call itself returns PP_OK: the
+ * failure is on the device) and returns with nothing in flight; the context stays usable and
+ * later calls run normally.  One-shot; depthwise and generic kernels ignore it.  Never needed in
+ * use.  Returns PP_OK. */
+int pp_debug_inject_timeout(void);
 
 /* Release the handle's host memory (the bound device image stays the caller's).  NULL is OK. */
 int pp_destroy(pp_handle h);

@@ -14,6 +14,8 @@ Plain, slow, obviously-correct numpy in IEEE float64:
                    compressed weight storage), written from this library's layout specification.
 * ``conv``      -- the layer forward sigma(W X + b) (§4.1, Eq. 1) as a dense 3x3 convolution over
                    the projected weights with the zeros in place, and the normalised error metric.
+* ``admm``      -- the layer-wise ADMM pruning of Algorithm 1 (§4.3-4.5, Eq. 4-7) with a hand-written
+                   gradient, for the training-side module of the library.
 
 Every function is pinned by ``tests/test_oracle_*.py`` against something other than itself:
 brute-force enumeration, torch's CPU convolution, hand-computed fixtures under
@@ -23,4 +25,4 @@ weights from the sections; its byte-level encoding itself is a specification of 
 not a result the paper prints ("parity unpinned" against the paper for the byte encoding).
 """
 
-from . import conv, layout, patterns, project  # noqa: F401
+from . import admm, conv, layout, patterns, project  # noqa: F401

@@ -38,6 +38,8 @@ SIGNATURES = {
     "pp_conv_static_scratch": (_c_int, [_c_void_p, _c_void_p, _c_int, _c_int, _c_int, _c_int, _c_void_p,
                                         _c_int, _c_void_p, _c_void_p]),
     "pp_static_scratch_bytes": (_c_int, [ctypes.POINTER(_c_size_t)]),
+    "pp_debug_inject_timeout": (_c_int, []),
+    "pp_measure_fp32_peak": (_c_int, [_c_int, ctypes.POINTER(ctypes.c_double)]),
     "pp_maxpool2x2": (_c_int, [_c_void_p, _c_int, _c_int, _c_int, _c_int, _c_int, _c_void_p,
                                _c_void_p]),
     "pp_device_status": (_c_int, [_c_int, ctypes.POINTER(ctypes.c_uint)]),

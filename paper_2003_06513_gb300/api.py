@@ -218,6 +218,13 @@ def workspace_for(layers, x_shapes, device=None, pools=None) -> Optional[torch.T
     return torch.empty(n // 4 + 4, dtype=torch.float32, device=device or "cuda")
 
 
+def measure_fp32_peak(reps: int = 10) -> float:
+    """Measured FP32 FMA peak of the current CUDA device in FLOP/s (pp_measure_fp32_peak)."""
+    v = ctypes.c_double()
+    _lib.check("pp_measure_fp32_peak", _lib.load().pp_measure_fp32_peak(int(reps), ctypes.byref(v)))
+    return float(v.value)
+
+
 def pp_maxpool2x2(x: torch.Tensor, out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
     """2x2/2 max-pool of a contiguous CUDA NCHW tensor via the library's kernel."""
     if not x.is_cuda or x.dtype not in _DT or not x.is_contiguous() or x.dim() != 4:

@@ -1,21 +1,28 @@
 // CUDA kernels and launchers of libpatconv (sm_103a): pattern-sparse 3x3 convolution.
 //
-// Work decomposition of the main kernel (pconv_main):
-//   * a lane owns an RY x RX block of output pixels of one image;
-//   * a warp owns one filter group (8 filters, "filter kernel reorder" of §3.4) for the 32
-//     blocks of its CTA's spatial tile and keeps 8 x RY*RX fp32 accumulators in registers;
-//   * a CTA is 8 warps = 8 filter groups (64 filters) over one spatial tile, so every input
-//     element staged in shared memory is reused by 64 filters;
-//   * input channels stream through a multi-stage cp.async pipeline: the tile of CK channels,
-//     with its zero halo (padding 1), lands in shared memory together with each group's
-//     descriptors and kept weights for those channels;
-//   * per input channel a lane loads its (RY-1)*S+3 x (RX-1)*S+3 input window into registers
-//     once and applies it to every kept kernel of its group: the 6-bit (slot, pattern) code of
-//     each kept kernel selects one of 64 compile-time bodies whose four tap offsets are
-//     constants (the 4 taps of §3.2), so no per-element index is decoded;
-//   * epilogue: + bias, ReLU, fp32 or fp16 (round to nearest even) vector stores to the
-//     original channel of each slot.
-// The path is a gathered sparse contraction, so it runs on the CUDA-core FFMA pipe.
+// Dense layers, main kernel pconv_tm<S, T, SORT, SHIFT>:
+//   * a lane owns a 4x4 block of output pixels of one image; a warp owns one filter group (8
+//     filter slots, the "filter kernel reorder" of §3.4) for its 32 blocks; a CTA is 16 warps =
+//     WG filter groups x WS spatial warps over one spatial tile;
+//   * accumulators live in tensor memory: 16 warps x 8 slots x 16 fp32 = all 512 columns; a kept
+//     kernel is applied by tcgen05.ld of its slot, 64 FMAs, tcgen05.st;
+//   * input channels stream through a 3-stage mbarrier pipeline: one TMA box per stage (the tile
+//     of CK channels with its zero halo, padding 1) or, where rows are not 16-byte multiples, a
+//     copy shared by all 512 threads; each group's descriptors and kept weights for those channels
+//     arrive by cp.async beside it;
+//   * per input channel a lane loads its input window into registers once and applies it to every
+//     kept kernel of its group: the 6-bit (slot, pattern) code of each kept kernel selects one of
+//     8 compile-time pattern bodies (generated inline PTX, gen_dispatch.py) whose four tap
+//     operands are fixed registers (the 4 taps of §3.2), so no per-element index is decoded;
+//   * persistent CTAs (one per SM unless the units overflow a CTA's table) walk their units
+//     (tile, filter chunk, input-channel split) as one chunk stream;
+//   * epilogue: + bias, ReLU, optionally the 2x2 max-pool, fp32 or fp16 (round to nearest even)
+//     stores to the original channel of each slot, or raw partial sums to the split workspace;
+//   * every pipeline wait is bounded; a wait that runs out records a bit in the status word and
+//     the kernel drains its copies, frees tensor memory and returns.
+// Depthwise layers: pconv_depthwise / pconv_depthwise_staged (HBM-bound).  Other pattern
+// libraries: pconv_generic.  The path is a gathered sparse contraction, so it runs on the
+// CUDA-core FFMA pipe.
 #include <cuda_fp16.h>
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -103,6 +110,8 @@ struct TmParams {
     const uint32_t* kofs;
     const float4* vals;
     unsigned* status;
+    long long wait_limit;              // SM cycles a pipeline (full / empty) wait may take
+    int no_fill;                       // test only: issue no stage fills (every first wait runs out)
     int N, C, H, W, Cout, Ho, Wo, G, relu;
     int WG, WS;                        // filter groups x spatial warps per CTA (WG * WS = 16)
     int BY, BX, NB;                    // spatial tile: BY x BX blocks (4x4 outputs) of NB images
@@ -135,7 +144,8 @@ __device__ __forceinline__ void cp_async_arrive(uint32_t a) {
     asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(a) : "memory");
 }
 // Bounded wait for the completion of the phase with the given parity.
-__device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity, unsigned* status, unsigned code) {
+__device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity, unsigned* status, unsigned code,
+                                          long long limit = kTimeoutCycles) {
     const long long t0 = clock64();
     while (true) {
         uint32_t done;
@@ -145,7 +155,7 @@ __device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity, unsigned*
             "selp.u32 %0, 1, 0, P;\n\t}"
             : "=r"(done) : "r"(a), "r"(parity) : "memory");
         if (done) return true;
-        if (clock64() - t0 > kTimeoutCycles) {
+        if (clock64() - t0 > limit) {
             atomicOr(status, code);
             return false;
         }
@@ -155,8 +165,9 @@ __device__ __forceinline__ void mbar_arrive(uint32_t a) {
     asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(a) : "memory");
 }
 // mbar_wait by a whole warp with one outcome for all its lanes
-__device__ __forceinline__ bool mbar_wait_warp(uint32_t a, uint32_t parity, unsigned* status, unsigned code) {
-    return __all_sync(0xffffffffu, mbar_wait(a, parity, status, code));
+__device__ __forceinline__ bool mbar_wait_warp(uint32_t a, uint32_t parity, unsigned* status, unsigned code,
+                                               long long limit) {
+    return __all_sync(0xffffffffu, mbar_wait(a, parity, status, code, limit));
 }
 __device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map, int x, int y, int c, int n,
                                             uint32_t mbar) {
@@ -386,7 +397,7 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     };
     fetch_range();
     {   // prologue: every thread's share of the first kStages chunks
-        const int first = min(kStages, Q);
+        const int first = p.no_fill ? 0 : min(kStages, Q);
         for (int q = 0; q < first; ++q) fill(q);
         if (threadIdx.x == 0) *s_issued = first;
     }
@@ -575,7 +586,7 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
 
     for (int q = 0; q < Q; ++q) {
         const int s = q % kStages;
-        if (!mbar_wait_warp(full0 + 8 * s, (q / kStages) & 1, p.status, kStatusFullTimeout)) break;
+        if (!mbar_wait_warp(full0 + 8 * s, (q / kStages) & 1, p.status, kStatusFullTimeout, p.wait_limit)) break;
         const Unit CU = s_units[ci];
         if (CU.g0 + wg < p.G) {
             const unsigned char* st = smem + p.stage_off + (size_t)s * p.stage_bytes;
@@ -604,7 +615,8 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
         if (lane == 0) mbar_arrive(empty0 + 8 * s);
         const int j = q + kStages - 1;
         if (q >= 1 && j < Q) {
-            if (!mbar_wait_warp(empty0 + 8 * (j % kStages), ((q - 1) / kStages) & 1, p.status, kStatusEmptyTimeout))
+            if (!mbar_wait_warp(empty0 + 8 * (j % kStages), ((q - 1) / kStages) & 1, p.status, kStatusEmptyTimeout,
+                                p.wait_limit))
                 break;
             fill(j);
             if (threadIdx.x == 0) *s_issued = j + 1;
@@ -1258,6 +1270,31 @@ __global__ void maxpool2x2(const T* __restrict__ x, T* __restrict__ y, long long
 }
 
 
+// ------------------------------------------------------------------------------ FP32 peak
+// The roofline denominator of the pattern-sparse kernel, measured instead of taken from the
+// nominal lane count: 16 independent fma.rn.f32 chains per thread (4-cycle latency hidden by 16
+// warps per SM scheduler), 4 CTAs of 512 threads per SM, no memory traffic.
+constexpr int kPeakChains = 16, kPeakUnroll = 4;
+__device__ float g_fma_sink;
+
+__global__ void __launch_bounds__(512, 4) fma_peak(int iters) {
+    float a[kPeakChains];
+#pragma unroll
+    for (int i = 0; i < kPeakChains; ++i) a[i] = 1e-3f * (float)(threadIdx.x + i);
+    const float m = 0.999f, c = 1e-7f;
+    for (int it = 0; it < iters; ++it) {
+#pragma unroll
+        for (int i = 0; i < kPeakChains; ++i) {
+#pragma unroll
+            for (int u = 0; u < kPeakUnroll; ++u) asm volatile("fma.rn.f32 %0, %0, %1, %2;" : "+f"(a[i]) : "f"(m), "f"(c));
+        }
+    }
+    float sum = 0.0f;
+#pragma unroll
+    for (int i = 0; i < kPeakChains; ++i) sum += a[i];
+    if (sum == 12345.0f) g_fma_sink = sum;   // keeps the chains live; never true in practice
+}
+
 // ------------------------------------------------------------------------------ static scratch
 // Scratch for pp_conv_static_scratch: a fixed array in the library's own device image, so that
 // callers which may not allocate device memory still get the input-channel split.  It exists on
@@ -1324,6 +1361,11 @@ EncodeTiledFn encode_tiled() {
     }();
     return fn;
 }
+
+// Test hook (pp_debug_inject_timeout): the next pattern-sparse launch issues no stage fills and
+// waits this many SM cycles (about 10 us) for them, so every CTA's first pipeline wait runs out.
+std::atomic<int> g_inject_timeout{0};
+constexpr long long kInjectedWaitCycles = 20000;
 
 unsigned* status_word() {
     static std::atomic<unsigned*> cached[64];
@@ -1747,6 +1789,9 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
     p.vals = reinterpret_cast<const float4*>(img + L->off_vals);
     p.status = status_word();
     if (!p.status) return PP_ERR_CUDA;
+    const bool inject = g_inject_timeout.exchange(0) != 0;
+    p.wait_limit = inject ? kInjectedWaitCycles : kTimeoutCycles;
+    p.no_fill = inject ? 1 : 0;
     p.N = N;
     p.C = L->cin_g;
     p.H = H;
@@ -2216,11 +2261,9 @@ int pp_conv_workspace_size(pp_handle h, int N, int H, int W, size_t* bytes) {
 
 int pp_conv_static_scratch(pp_handle h, const void* x, int dtype, int N, int H, int W, const float* bias, int relu,
                            void* y, void* stream) {
-    if (!h) return PP_ERR_NULL;
-    if (!h->dev) return PP_ERR_NOT_BOUND;
-    if (dtype != PP_F32 && dtype != PP_F16) return PP_ERR_DTYPE;
-    if (N < 0 || H < 1 || W < 1) return PP_ERR_SHAPE;
-    if (N == 0) return pp_conv_ws(h, x, dtype, N, H, W, bias, relu, y, nullptr, 0, stream);
+    // the argument errors of pp_conv_ws come first, before the scratch size is considered
+    const int v = validate_conv(h, x, dtype, N, H, W, bias, relu, y);
+    if (v != PP_OK || N == 0) return v;
     size_t need = 0;
     const int rc = pp_conv_workspace_size(h, N, H, W, &need);
     if (rc != PP_OK) return rc;
@@ -2233,6 +2276,40 @@ int pp_conv_static_scratch(pp_handle h, const void* x, int dtype, int N, int H, 
 int pp_static_scratch_bytes(size_t* bytes) {
     if (!bytes) return PP_ERR_NULL;
     *bytes = kStaticScratchBytes;
+    return PP_OK;
+}
+
+int pp_measure_fp32_peak(int reps, double* flop_per_s) {
+    if (!flop_per_s) return PP_ERR_NULL;
+    if (reps < 1 || reps > 1000) return PP_ERR_ARG;
+    const int sms = sm_count(), ctas = 4 * sms, threads = 512, iters = 4096;
+    cudaEvent_t e0, e1;
+    if (cudaEventCreate(&e0) != cudaSuccess) return PP_ERR_CUDA;
+    if (cudaEventCreate(&e1) != cudaSuccess) {
+        cudaEventDestroy(e0);
+        return PP_ERR_CUDA;
+    }
+    float best = 0.0f;
+    bool ok = true;
+    fma_peak<<<ctas, threads>>>(16);                      // warm-up
+    for (int r = 0; r < reps && ok; ++r) {
+        float ms = 0.0f;
+        ok = cudaEventRecord(e0) == cudaSuccess;
+        fma_peak<<<ctas, threads>>>(iters);
+        ok = ok && cudaGetLastError() == cudaSuccess && cudaEventRecord(e1) == cudaSuccess &&
+             cudaEventSynchronize(e1) == cudaSuccess && cudaEventElapsedTime(&ms, e0, e1) == cudaSuccess;
+        if (ok && ms > 0.0f && (best == 0.0f || ms < best)) best = ms;
+    }
+    cudaEventDestroy(e0);
+    cudaEventDestroy(e1);
+    if (!ok || best <= 0.0f) return PP_ERR_CUDA;
+    const double flop = 2.0 * kPeakChains * kPeakUnroll * (double)iters * threads * ctas;
+    *flop_per_s = flop / (best * 1e-3);
+    return PP_OK;
+}
+
+int pp_debug_inject_timeout(void) {
+    g_inject_timeout.store(1);
     return PP_OK;
 }
 

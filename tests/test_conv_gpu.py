@@ -5,6 +5,8 @@ Error metric: |y_gpu - y_ref| / (sum |W_hat| |x| + |b| + 2^-1000) per output, ma
 bar 1e-4 for fp32 I/O and 2e-3 for fp16 I/O.  The oracle projects the weights itself: nothing
 it uses comes from the CUDA path.
 """
+import ctypes
+
 import numpy as np
 import pytest
 import torch
@@ -12,12 +14,23 @@ import torch
 from oracle import conv as OC
 from oracle import patterns as OP
 from oracle import project as OPR
-from paper_2003_06513_gb300 import api
+from paper_2003_06513_gb300 import _lib, api
 from paper_2003_06513_gb300 import workloads as WL
 
 pytestmark = pytest.mark.gpu
 
 TOL = {torch.float32: 1e-4, torch.float16: 2e-3}
+
+
+@pytest.fixture(autouse=True)
+def _no_pipeline_timeout():
+    """After every test: no kernel of the test recorded a pipeline wait that ran out (the status
+    word of the conv kernels, read and cleared through pp_device_status)."""
+    yield
+    torch.cuda.synchronize()
+    st = ctypes.c_uint(0)
+    assert _lib.load().pp_device_status(1, ctypes.byref(st)) == 0
+    assert st.value == 0, f"a conv kernel recorded pipeline timeout bits {st.value:#x}"
 
 
 def _np_dt(dt):

@@ -145,6 +145,63 @@ def test_layout_hand_packed_fixture():
     assert s["header"][:14].tolist() == [int(v) for v in g["header"]]
 
 
+def _snake_fixture():
+    g = golden_kv("layout_snake.txt")
+    pa, pb = [int(v) for v in g["pa"]], [int(v) for v in g["pb"]]
+    W = np.zeros((20, 2, 9), np.float32)
+    for co in range(20):
+        for ci, p in enumerate((pa[co], pb[co])):
+            for k, t in enumerate(P.taps_of(P.default8()[p])):
+                W[co, ci, t] = co + 0.25 * ci + 0.0625 * k + 1
+    return W.reshape(20, 2, 3, 3), g
+
+
+def _snake_expected(g):
+    """desc words assembled by the specification's bit rule from the fixture's codes, and the
+    vals rows: the (co, ci) kernels in (g, ci, slot) order, values by the fixture's rule."""
+    desc, rows = [], []
+    perm = [int(v) for v in g["perm"]]
+    for grp in range(3):
+        for ci in range(2):
+            cnt, *codes = [int(v) for v in g[f"desc_g{grp}c{ci}"]]
+            assert len(codes) == cnt
+            desc.append(cnt | sum(c << (4 + 6 * j) for j, c in enumerate(codes)))
+            for c in codes:
+                co = perm[8 * grp + (c >> 3)]
+                rows.append([co + 0.25 * ci + 0.0625 * k + 1 for k in range(4)])
+    return desc, rows
+
+
+def test_layout_snake_deal_hand_fixture():
+    """Three groups: the sorted filters are dealt in snake order (round r fills slot r of every
+    group, direction alternating), which the hand-dealt fixture pins exactly."""
+    W, g = _snake_fixture()
+    lib = P.default8()
+    r = PR.project(W, lib, 1.0)
+    assert r["beta"] == 40
+    pa, pb = [int(v) for v in g["pa"]], [int(v) for v in g["pb"]]
+    assert r["pid"].tolist() == [[a, b] for a, b in zip(pa, pb)]
+    assert L.filter_order(r["pid"]) == [int(v) for v in g["order"]]
+    s = L.build(W, r["pid"], lib, 1, 1, r["beta"])
+    desc, rows = _snake_expected(g)
+    assert s["perm"].tolist() == [int(v) for v in g["perm"]]
+    assert s["desc"].tolist() == desc
+    assert s["kofs"].tolist() == [int(v) for v in g["kofs"]]
+    assert s["vals"].tolist() == rows
+
+
+def test_packer_snake_deal_hand_fixture():
+    """The C++ packer (pp_export) on the same hand-dealt fixture."""
+    from paper_2003_06513_gb300 import api
+    W, g = _snake_fixture()
+    layer = api.pp_pack(W, None, 1.0)
+    desc, rows = _snake_expected(g)
+    assert layer.export("perm").tolist() == [int(v) for v in g["perm"]]
+    assert layer.export("desc").tolist() == desc
+    assert layer.export("kofs").tolist() == [int(v) for v in g["kofs"]]
+    assert layer.export("vals").reshape(-1, 4).tolist() == rows
+
+
 @pytest.mark.parametrize("cout,cin,keep,dw", [(3, 2, 0.5, False), (8, 8, 1.0, False), (13, 5, 0.3, False),
                                               (17, 1, 0.6, False), (20, 20, 1.0, True), (9, 9, 0.5, True),
                                               (64, 3, 1.0, False)])

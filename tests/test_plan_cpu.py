@@ -257,3 +257,31 @@ def test_lane_order_random_shapes(seed):
         raster = sum(_window_wavefronts(pl, shape, 1, t, False) for t in range(tiles))
         dealt = sum(_window_wavefronts(pl, shape, 1, t, True) for t in range(tiles))
         assert pl["lane_sort"] == (1 if dealt < raster else 0), (shape, ws, raster, dealt, pl)
+
+
+def test_one_handle_planned_from_many_threads():
+    """pp_conv_plan from 8 host threads on one fresh handle at once: every thread gets the same
+    plans (the per-handle plan cache is created once and guarded; ctypes releases the GIL)."""
+    import threading
+    rng = np.random.default_rng(21)
+    W = rng.standard_normal((256, 128, 3, 3)).astype(np.float32)
+    layer = api.pp_pack(W, None, 0.3)
+    shapes = [(n, 128, h, h) for n in (1, 8, 32) for h in (7, 14, 28, 56)]
+    out, errors = [None] * 8, []
+
+    def work(i):
+        try:
+            got = []
+            for rep in range(5):
+                for sh in shapes[i % 3:] + shapes[:i % 3]:
+                    got.append((sh, tuple(layer.plan(sh, 1 << 30).items())))
+            out[i] = sorted(set(got))
+        except Exception as e:        # pragma: no cover - reported below
+            errors.append(e)
+    threads = [threading.Thread(target=work, args=(i,)) for i in range(8)]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    assert not errors
+    assert all(o == out[0] for o in out) and len(out[0]) == len(shapes)

@@ -1,0 +1,138 @@
+"""GPU parity of every launch plan the planner can choose, and of the single-layer sweep at its
+full batch.
+
+Each case states the plan outcome it exercises and asserts it through layer.plan (the same plan
+the launch uses): linear tiles, rectangles of several whole images, the bank-group lane order,
+blocks shifted to start at output columns 4j - 1, the copy fallback for rows that are not a
+multiple of 16 bytes, fp16 stages through TMA without the fused pool, input-channel splits up to
+32 ways, more units than one persistent CTA per SM can hold in its table, and the fused pool.
+Outputs are compared with the float64 oracle (§4.1 Eq. 1 over the projection of §4.3-4.4) on
+two sampled images of the full batch; the bar is 1e-4 of sum|W_hat||x| for fp32 I/O and 2e-3 for
+fp16 I/O.  Inputs come from the seeded generators only."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import conv as OC
+from oracle import patterns as OP
+from oracle import project as OPR
+from paper_2003_06513_gb300 import api
+from paper_2003_06513_gb300 import workloads as WL
+
+pytestmark = pytest.mark.gpu
+
+TOL = {"f32": 1e-4, "f16": 2e-3}
+SMS_TABLE = 64        # units one persistent CTA holds in its table
+
+
+def _run(cout, cin, n, h, w, keep, io, pool=False, stride=1, seed=0, relu_in=True):
+    rng = np.random.default_rng(seed)
+    W = (rng.standard_normal((cout, cin, 3, 3)) * np.sqrt(2 / (9 * cin))).astype(np.float32)
+    b = (rng.standard_normal(cout) * 0.1).astype(np.float32)
+    x = WL.activations((n, cin, h, w), seed + 17, relu=relu_in,
+                       dtype=np.float32 if io == "f32" else np.float16)
+    layer = api.pp_pack(W, None, keep, 1, stride).bind("cuda")
+    xt = torch.from_numpy(x).cuda()
+    nb = layer.workspace_bytes(xt.shape, pool)
+    ws = torch.empty(max(nb // 4, 1), device="cuda") if nb else None
+    plan = layer.plan(xt.shape, nb, pool2x2=pool)
+    y = layer.conv(xt, torch.from_numpy(b).cuda(), True, workspace=ws, pool2x2=pool)
+    idx = [0, n - 1] if n > 1 else [0]
+    Wh = OPR.project(W, OP.default8(), keep)["W_hat"]
+    xs = x[idx].astype(np.float64)
+    ref = OC.conv_ref(xs, Wh, b, stride, True)
+    den = OC.denominator(xs, Wh, b, stride)
+    if pool:
+        ref, den = OC.maxpool2x2(ref), OC.maxpool2x2(den)
+    err = OC.max_norm_err(y[idx].double().cpu().numpy(), ref, den)
+    assert err <= TOL[io], f"max normalised error {err:.3e}"
+    return plan, y
+
+
+def _sms():
+    return torch.cuda.get_device_properties(0).multi_processor_count
+
+
+def test_units_overflow_the_persistent_table():
+    """VGG-16 layer 1 shape at batch 256: more units than one CTA per SM holds, so the launch
+    takes ceil(units / 64) persistent CTAs."""
+    plan, _ = _run(64, 3, 256, 224, 224, 1.0, "f32", seed=1)
+    assert plan["units"] > SMS_TABLE * _sms()
+    assert plan["ctas"] == -(-plan["units"] // SMS_TABLE) > _sms()
+
+
+@pytest.mark.parametrize("pool", [False, True])
+def test_linear_tile(pool):
+    """28x28 maps at keep 1.0: lanes take consecutive blocks across image boundaries (whole
+    images staged, several per tile), with a split."""
+    plan, _ = _run(256, 256, 64, 28, 28, 1.0, "f32", pool=pool, seed=2)
+    nb_rect = max(1, 32 * plan["spatial_warps"] // (plan["tile_by"] * plan["tile_bx"]))
+    assert (plan["tile_by"], plan["tile_bx"]) == (7, 7) and plan["tile_nb"] > nb_rect   # linear
+    assert plan["shift"] == 0 and plan["splits"] > 1
+
+
+@pytest.mark.parametrize("pool", [False, True])
+def test_bank_group_lane_order(pool):
+    """56x56 maps at keep 0.3: rows of 14 (or 15 shifted) blocks, each warp's blocks dealt to
+    lanes by shared-memory bank group; shifted blocks without the pool, blocks at 4j with it."""
+    plan, _ = _run(128, 128, 16, 56, 56, 0.3, "f32", pool=pool, seed=3)
+    assert plan["lane_sort"] == 1 and plan["shift"] == (0 if pool else 1)
+
+
+def test_multi_image_rectangles_with_split():
+    """7x7 maps: rectangles of 8 whole images (2x2 blocks each) and an 8-way split."""
+    plan, _ = _run(256, 256, 64, 7, 7, 0.5, "f32", seed=4)
+    assert plan["tile_nb"] == 8 and plan["splits"] > 1
+
+
+def test_batch_one_split_32_ways():
+    plan, _ = _run(256, 256, 1, 14, 14, 0.25, "f32", seed=5)
+    assert plan["splits"] == 32 and plan["shift"] == 1
+
+
+@pytest.mark.parametrize("io", ["f32", "f16"])
+def test_copy_fallback_rows(io):
+    """Rows of 30 elements (120 / 60 bytes: no tensor copy), shifted blocks, split."""
+    plan, _ = _run(64, 32, 4, 20, 30, 0.5, io, seed=6)
+    assert plan["shift"] == 1 and plan["splits"] > 1
+
+
+@pytest.mark.parametrize("pool", [False, True])
+def test_fp16_through_tma(pool):
+    """fp16 rows of 56 elements (112 bytes): fp16 stages through TMA, with and without the pool."""
+    plan, _ = _run(128, 128, 16, 56, 56, 0.3, "f16", pool=pool, seed=7)
+    assert plan["shift"] == (0 if pool else 1)
+
+
+@pytest.mark.parametrize("io", ["f32", "f16"])
+def test_stride2_heads(io):
+    plan, _ = _run(128, 128, 16, 56, 56, 0.4, io, stride=2, seed=8)
+    assert plan["shift"] == 0 and plan["lane_sort"] == 0
+
+
+# the single-layer sweep (C = Cin = Cout, H = W, batch, keep, io) at full batch
+SWEEP = [(128, 56, 64, 1.0, "f32"), (256, 28, 256, 0.25, "f16"), (512, 14, 256, 0.5, "f32"),
+         (512, 7, 256, 0.25, "f16"), (256, 56, 16, 0.25, "f16"), (128, 28, 64, 1.0, "f16"),
+         (256, 14, 1, 1.0, "f32"), (512, 28, 16, 0.5, "f32"), (128, 7, 16, 1.0, "f32")]
+
+
+@pytest.mark.parametrize("c,hw,n,keep,io", SWEEP)
+def test_sweep_point_full_batch(c, hw, n, keep, io):
+    """Points of the 288-point sweep at their full batch, with the sweep's own seeds (weights,
+    bias) and N(0,1) inputs as the sweep draws them."""
+    pts = [(L, nn, dt) for L, nn, dt in WL.sweep() if (L.cin, L.h, nn, L.keep, dt) == (c, hw, n, keep, io)]
+    assert len(pts) == 1
+    L, _, _ = pts[0]
+    W, b = WL.weights(L), WL.bias(L)
+    x = WL.activations((n, c, hw, hw), L.x_seed, dtype=np.float32 if io == "f32" else np.float16)
+    layer = api.pp_pack(W, None, keep).bind("cuda")
+    xt = torch.from_numpy(x).cuda()
+    nb = layer.workspace_bytes(xt.shape)
+    ws = torch.empty(max(nb // 4, 1), device="cuda") if nb else None
+    y = layer.conv(xt, torch.from_numpy(b).cuda(), True, workspace=ws)
+    idx = [0, n - 1] if n > 1 else [0]
+    Wh = OPR.project(W, OP.default8(), keep)["W_hat"]
+    xs = x[idx].astype(np.float64)
+    err = OC.max_norm_err(y[idx].double().cpu().numpy(), OC.conv_ref(xs, Wh, b, 1, True),
+                          OC.denominator(xs, Wh, b, 1))
+    assert err <= TOL[io], f"max normalised error {err:.3e}"

@@ -2,10 +2,13 @@
 
 Such callers (code inside a host runtime that owns every device allocation, plugins that must
 not allocate while serving) still pass x, y and bias, and the split of the input channels keeps
-its partial sums in the library's own static device array instead of a caller workspace.  This
-test calls the entry point through the C ABI, twice in a row, and checks both results against
-the workspace entry point pp_conv_ws within the tolerance of the other conv tests.  The file
-sorts last so that a run stopping at the first failure has already run every other test.
+its partial sums in the library's own static device array instead of a caller workspace.  The
+test calls the entry point through the C ABI.  It first fills the array with wrong partial sums
+(the same layer on the negated input), then runs the checked call twice in a row and compares
+both results with the workspace entry point pp_conv_ws and with the oracle on two sampled
+images, within the tolerance of the other conv tests: a call that read a partial sum it did not
+write would fail.  The file sorts last so that a run stopping at the first failure has already
+run every other test.
 """
 import ctypes
 
@@ -21,13 +24,15 @@ from paper_2003_06513_gb300 import workloads as WL
 
 pytestmark = pytest.mark.gpu
 
+PP_ERR_NULL = -1
+PP_ERR_ARG = -11
 PP_ERR_SCRATCH = -13
 
 
-def _call_static(lib, layer, x, b, y):
-    N, _, H, W = x.shape
-    return lib.pp_conv_static_scratch(layer._h, ctypes.c_void_p(x.data_ptr()), 0, N, H, W,
-                                      ctypes.c_void_p(b.data_ptr()), 1,
+def _call_static(lib, layer, x, b, y, relu=1):
+    N, _, H, W = x.shape if x is not None else y.shape
+    xp = ctypes.c_void_p(x.data_ptr()) if x is not None else None
+    return lib.pp_conv_static_scratch(layer._h, xp, 0, N, H, W, ctypes.c_void_p(b.data_ptr()), relu,
                                       ctypes.c_void_p(y.data_ptr()), None)
 
 
@@ -50,15 +55,26 @@ def test_static_scratch_entry_point_matches_workspace_entry_point():
     ref = layer.conv(x, b, True, workspace=ws)
     torch.cuda.synchronize()
 
+    # leave wrong partial sums in the array: same layer and split on the negated input
+    junk = torch.empty_like(ref)
+    assert _call_static(lib, layer, -x, b, junk, relu=0) == 0
+    torch.cuda.synchronize()
+    assert (junk - ref).abs().max().item() > 0.1
+
     Wh = OPR.project(W, OP.default8(), L.keep)["W_hat"]
-    den = OC.denominator(x_np, Wh, bias, 1)
+    idx = [0, 15]
+    oracle = OC.conv_ref(x_np[idx].astype(np.float64), Wh, bias, 1, True)
+    den = OC.denominator(x_np.astype(np.float64), Wh, bias, 1)
     ref_h = ref.double().cpu().numpy()
     for _ in range(2):                                # two calls in a row share the array
         y = torch.full_like(ref, float("nan"))
         assert _call_static(lib, layer, x, b, y) == 0
         torch.cuda.synchronize()
-        err = OC.max_norm_err(y.double().cpu().numpy(), ref_h, den)
+        y_h = y.double().cpu().numpy()
+        err = OC.max_norm_err(y_h, ref_h, den)
         assert err <= 1e-4, f"static-scratch result differs from pp_conv_ws: {err:.3e}"
+        err = OC.max_norm_err(y_h[idx], oracle, den[idx])
+        assert err <= 1e-4, f"static-scratch result differs from the oracle: {err:.3e}"
 
 
 def test_static_scratch_rejects_calls_beyond_its_size():
@@ -77,5 +93,8 @@ def test_static_scratch_rejects_calls_beyond_its_size():
     x = torch.zeros(shape, device="cuda")
     y = torch.zeros(shape, device="cuda")
     b = torch.zeros(C, device="cuda")
+    # argument errors come before the size check
+    assert _call_static(lib, layer, None, b, y) == PP_ERR_NULL
+    assert _call_static(lib, layer, x, b, y, relu=2) == PP_ERR_ARG
     assert _call_static(lib, layer, x, b, y) == PP_ERR_SCRATCH
     assert b"static scratch" in lib.pp_status_string(PP_ERR_SCRATCH)
