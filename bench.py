@@ -730,7 +730,7 @@ def layer_suite(args):
                               stride=L.stride).bind("cuda")
             x = torch.from_numpy(WL.layer_input(L, batch, dtype=ndt)).cuda()
             b = torch.from_numpy(WL.bias(L)).cuda()
-            nb = lay.workspace_bytes(x.shape)
+            nb = lay.workspace_bytes(x.shape, dtype=x.dtype)
             ws = torch.empty(max(nb // 4, 1), device="cuda") if nb else None
             ms, ms_eager, ms_graph = _time_layer(lay, x, b, True, ws, K, warmup=10)
             G = (L.cout + 7) // 8
@@ -778,7 +778,7 @@ def sweep_run(args):
             g.manual_seed(L.x_seed)
             x = torch.randn((n, L.cin, L.h, L.w), generator=g, device="cuda").to(tdt)
             b = torch.from_numpy(WL.bias(L)).cuda()
-            nb = lay.workspace_bytes(x.shape)
+            nb = lay.workspace_bytes(x.shape, dtype=x.dtype)
             ws = torch.empty(max(nb // 4, 1), device="cuda") if nb else None
             ms = _time_layer(lay, x, b, True, ws, K)[0]
             fl, by = conv_cost(lay.beta, L.cin, L.cout, L.h, L.w, L.ho, L.wo, n, (L.cout + 7) // 8, es)
@@ -820,7 +820,7 @@ def profile_layer(args):
     ndt = np.float16 if args.workload == "mobilenet" else np.float32
     x = torch.from_numpy(WL.layer_input(L, args.batch, relu=not L.depthwise, dtype=ndt)).cuda()
     b = torch.from_numpy(WL.bias(L)).cuda()
-    ws_n = lay.workspace_bytes(x.shape)
+    ws_n = lay.workspace_bytes(x.shape, dtype=x.dtype)
     ws = torch.empty(max(ws_n // 4, 1), device="cuda") if ws_n else None
     y = lay.conv(x, b, True, workspace=ws)
     torch.cuda.synchronize()
@@ -833,7 +833,7 @@ def profile_layer(args):
     ms = e0.elapsed_time(e1) / max(args.steps, 1)
     flops = 8.0 * lay.beta * args.batch * L.ho * L.wo
     print(json.dumps({"layer": L.name, "batch": args.batch, "ms": ms, "useful_tflops": flops / ms / 1e9,
-                      "plan": lay.plan(x.shape, ws_n)}))
+                      "plan": lay.plan(x.shape, ws_n, dtype=x.dtype)}))
 
 
 def main():

@@ -194,7 +194,14 @@ int pp_conv_workspace_size(pp_handle h, int N, int H, int W, size_t* bytes);
  * 4j - 1 instead of 4j (each lane's input window then starts 8 bytes into a 16-byte group, so a
  * window row is one 8-byte and one 16-byte shared load instead of two bank-conflicted 4-byte
  * loads around a 16-byte one; never for pp_conv_pool_ws, which keeps blocks at 4j so that every
- * 2x2 pooling window lies inside one block), else 0.  Writes min(n_info, 15) values.  Host-only. */
+ * 2x2 pooling window lies inside one block), else 0; [15] 1 where the launch takes the balanced
+ * schedule: one CTA per SM, each taking an equal share of all units' input-channel chunks
+ * instead of whole units (whole units leave the SMs of the last partial wave idle); a unit cut
+ * between two CTAs is finished by the CTA holding its first chunks, which adds the later ones'
+ * raw sums from their workspace slots (workspace: 256 KiB per SM + flags, reported in [2]; the
+ * launch is cooperative and resets the flags with a small memset first; the input must go
+ * through TMA, else the launch takes whole units), else 0.  Writes min(n_info, 16) values.
+ * Host-only. */
 int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info);
 
 /* Launch plan of pp_conv_pool_ws (conv with the fused 2x2 max-pool) for a call shape and
@@ -202,6 +209,16 @@ int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64
  * the fused pooling (depthwise, other pattern libraries) return PP_ERR_PATH.  Host-only. */
 int pp_conv_pool_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info,
                       int n_info);
+
+/* The plan of a call with a given dtype (PP_F32, PP_F16) and pool flag (0: pp_conv_ws, 1:
+ * pp_conv_pool_ws), fields as pp_conv_plan.  The dtype matters where the planner asks whether
+ * the input rows go through TMA (a multiple of 16 bytes), as the balanced schedule needs;
+ * pp_conv_plan, pp_conv_pool_plan and pp_conv_workspace_size answer for fp32 calls.  The
+ * workspace a call needs is info[2] of the plan with workspace_bytes = SIZE_MAX.  Errors:
+ * PP_ERR_DTYPE, PP_ERR_ARG (pool not 0/1), PP_ERR_PATH (pool on a layer without it), and those
+ * of pp_conv_plan.  Host-only. */
+int pp_conv_plan_dt(pp_handle h, int dtype, int pool, int N, int H, int W, size_t workspace_bytes,
+                    int64_t* info, int n_info);
 
 /* pp_conv_ws for callers that cannot allocate device memory (the paper has no counterpart to
  * this entry point).  Some callers are not allowed to call cudaMalloc or any allocating routine:

@@ -35,6 +35,8 @@ SIGNATURES = {
                               _c_int]),
     "pp_conv_pool_plan": (_c_int, [_c_void_p, _c_int, _c_int, _c_int, _c_size_t,
                                    ctypes.POINTER(ctypes.c_int64), _c_int]),
+    "pp_conv_plan_dt": (_c_int, [_c_void_p, _c_int, _c_int, _c_int, _c_int, _c_int, _c_size_t,
+                                 ctypes.POINTER(ctypes.c_int64), _c_int]),
     "pp_conv_static_scratch": (_c_int, [_c_void_p, _c_void_p, _c_int, _c_int, _c_int, _c_int, _c_void_p,
                                         _c_int, _c_void_p, _c_void_p]),
     "pp_static_scratch_bytes": (_c_int, [ctypes.POINTER(_c_size_t)]),

@@ -102,28 +102,23 @@ class Layer:
 
     PLAN_KEYS = ("path", "splits", "workspace_bytes", "units", "tile_by", "tile_bx", "tile_nb",
                  "channels_per_stage", "filter_groups", "spatial_warps", "smem_bytes",
-                 "chunks_per_unit", "ctas", "lane_sort", "shift")
+                 "chunks_per_unit", "ctas", "lane_sort", "shift", "streamk")
 
-    def plan(self, x_shape, workspace_bytes: int = 0, pool2x2: bool = False) -> dict:
-        """Launch plan pp_conv_ws (or, with pool2x2, pp_conv_pool_ws) would use for input shape
-        [N, C, H, W] (pp_conv_plan / pp_conv_pool_plan)."""
+    def plan(self, x_shape, workspace_bytes: int = 0, pool2x2: bool = False,
+             dtype=torch.float32) -> dict:
+        """Launch plan pp_conv_ws (or, with pool2x2, pp_conv_pool_ws) would use for an input of
+        shape [N, C, H, W] and dtype (pp_conv_plan_dt)."""
         N, _, H, W = x_shape
         n = len(self.PLAN_KEYS)
         info = (ctypes.c_int64 * n)()
-        name = "pp_conv_pool_plan" if pool2x2 else "pp_conv_plan"
-        _lib.check(name, getattr(_lib.load(), name)(self._h, N, H, W, int(workspace_bytes), info, n))
+        _lib.check("pp_conv_plan_dt", _lib.load().pp_conv_plan_dt(
+            self._h, _DT[dtype], 1 if pool2x2 else 0, N, H, W, int(workspace_bytes), info, n))
         return dict(zip(self.PLAN_KEYS, (int(v) for v in info)))
 
-    def workspace_bytes(self, x_shape, pool2x2: bool = False) -> int:
-        """Workspace the input-channel split would use for this input shape (0: no split), for
-        pp_conv_ws or, with pool2x2, for pp_conv_pool_ws (whose plan may differ)."""
-        N, _, H, W = x_shape
-        if pool2x2:
-            return self.plan(x_shape, (1 << 64) - 1, pool2x2=True)["workspace_bytes"]
-        v = ctypes.c_size_t()
-        _lib.check("pp_conv_workspace_size", _lib.load().pp_conv_workspace_size(
-            self._h, N, H, W, ctypes.byref(v)))
-        return int(v.value)
+    def workspace_bytes(self, x_shape, pool2x2: bool = False, dtype=torch.float32) -> int:
+        """Workspace the call would use for this input shape and dtype (0: none): the input-channel
+        split or the balanced schedule, for pp_conv_ws or, with pool2x2, pp_conv_pool_ws."""
+        return self.plan(x_shape, (1 << 64) - 1, pool2x2, dtype)["workspace_bytes"]
 
     def conv(self, x: torch.Tensor, bias: Optional[torch.Tensor] = None, relu: bool = False,
              out: Optional[torch.Tensor] = None, stream=None,

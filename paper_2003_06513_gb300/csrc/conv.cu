@@ -1,6 +1,6 @@
 // CUDA kernels and launchers of libpatconv (sm_103a): pattern-sparse 3x3 convolution.
 //
-// Dense layers, main kernel pconv_tm<S, T, SORT, SHIFT>:
+// Dense layers, main kernel pconv_tm<S, T, SORT, SHIFT, SK>:
 //   * a lane owns a 4x4 block of output pixels of one image; a warp owns one filter group (8
 //     filter slots, the "filter kernel reorder" of §3.4) for its 32 blocks; a CTA is 16 warps =
 //     WG filter groups x WS spatial warps over one spatial tile;
@@ -16,6 +16,9 @@
 //     operands are fixed registers (the 4 taps of §3.2), so no per-element index is decoded;
 //   * persistent CTAs (one per SM unless the units overflow a CTA's table) walk their units
 //     (tile, filter chunk, input-channel split) as one chunk stream;
+//   * SK (balanced schedule, stride 1): one CTA per SM takes an equal range of all units'
+//     channel chunks; a unit cut between CTAs is finished by the CTA holding its first chunks,
+//     which adds the later CTAs' raw sums (a cooperative launch: every CTA is resident);
 //   * epilogue: + bias, ReLU, optionally the 2x2 max-pool, fp32 or fp16 (round to nearest even)
 //     stores to the original channel of each slot, or raw partial sums to the split workspace;
 //   * every pipeline wait is bounded; a wait that runs out records a bit in the status word and
@@ -99,7 +102,9 @@ constexpr int kMaxUnitsPerCta = 64;                // units one persistent CTA h
 // Device status word: a wait that ran out of time records its code here and the kernel returns
 // early instead of hanging (read back by pp_device_status).
 __device__ unsigned int g_pp_status;
-enum : unsigned { kStatusFullTimeout = 1u, kStatusEmptyTimeout = 2u, kStatusDrainTimeout = 4u };
+enum : unsigned { kStatusFullTimeout = 1u, kStatusEmptyTimeout = 2u, kStatusDrainTimeout = 4u,
+                  kStatusPartTimeout = 8u };
+constexpr int kSlotFloats = kCompute * 8 * 16 * 32;   // a CTA's accumulators: 16 warps x 8 slots x 16 x 32 lanes
 
 struct TmParams {
     const void* x;
@@ -122,6 +127,10 @@ struct TmParams {
     int KS, c_split;                   // input-channel splits; channels per split (multiple of CK)
     float* ws;                         // KS > 1: fp32 partial sums [KS][N][Cout][Ho][Wo]
     size_t ws_stride;                  // elements per split
+    int streamk;                       // balanced schedule: CTA b takes chunks [T b / P, T (b + 1) / P)
+    long long sk_total;                // T: chunks of all units (every unit has n_chunks of them)
+    float* sk_slots;                   // a CTA's part: its raw accumulators (kSlotFloats per CTA)
+    unsigned* sk_flags;                // [CTA][warp]: 1 once that warp's part slot is written
     int IH, BWb;                       // staged rows / row width (elements) per (image, channel)
     int ixa;                           // stage origin column: a multiple of ixa (16 bytes of input)
     int use_tma, vec_store, vec_pair;  // float4 / 8-byte-group stores; pair stores (SHIFT)
@@ -247,9 +256,14 @@ __device__ __forceinline__ void stage_input_share(const TmParams& p, TIn* s_in, 
 
 // One unit of work of a CTA: a spatial tile, a filter chunk (WG groups) and an input-channel
 // split.  Units are numbered with the filter chunk fastest, so CTAs working at the same time
-// share input tiles in L2.
+// share input tiles in L2.  With the balanced (stream-K) schedule a CTA may hold only a segment
+// of a unit's channel chunks: c_lo and nck then describe the segment, and role says whether it
+// is the whole unit, its head (the first chunks: this CTA adds the other segments' partial sums
+// and writes the result) or a later part (raw partial sums to the CTA's workspace slot); a head's
+// parts are the next CTAs up to pb1 (exclusive).  role and pb1 share one word: role | pb1 << 2.
+enum : int { kRoleFull = 0, kRoleHead = 1, kRolePart = 2 };
 struct __align__(16) Unit {
-    int ks, tn, n0, oy0, ox0, iy0, ix0, g0, c_lo, c_hi, nck, pad;
+    int ks, tn, n0, oy0, ox0, iy0, ix0, g0, c_lo, c_hi, nck, sk;
 };
 
 template <int S>
@@ -266,6 +280,7 @@ __device__ __forceinline__ Unit unit_of(const TmParams& p, int u) {
     U.c_lo = U.ks * p.c_split;
     U.c_hi = min(p.C, U.c_lo + p.c_split);
     U.nck = (U.c_hi - U.c_lo + p.CK - 1) / p.CK;
+    U.sk = kRoleFull;
     // linear tiles: tile tn holds blocks [tn * lanes, (tn + 1) * lanes) of the (image, block row,
     // block column) sequence and stages the whole images from n0 on
     U.n0 = p.linear ? (int)(((long long)U.tn * 32 * p.WS) / (p.BY * p.BX)) : U.tn * p.NB;
@@ -313,12 +328,82 @@ __device__ __forceinline__ void fill_share(const TmParams& p, const CUtensorMap*
     cp_async_arrive(fb);
 }
 
+__device__ __forceinline__ void tmem_st16(uint32_t ta, const float (&a)[16]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};\n\t"
+        "tcgen05.wait::st.sync.aligned;" ::"r"(ta),
+        "r"(__float_as_uint(a[0])), "r"(__float_as_uint(a[1])), "r"(__float_as_uint(a[2])), "r"(__float_as_uint(a[3])),
+        "r"(__float_as_uint(a[4])), "r"(__float_as_uint(a[5])), "r"(__float_as_uint(a[6])), "r"(__float_as_uint(a[7])),
+        "r"(__float_as_uint(a[8])), "r"(__float_as_uint(a[9])), "r"(__float_as_uint(a[10])), "r"(__float_as_uint(a[11])),
+        "r"(__float_as_uint(a[12])), "r"(__float_as_uint(a[13])), "r"(__float_as_uint(a[14])), "r"(__float_as_uint(a[15]))
+        : "memory");
+}
+
+// Balanced schedule, a part segment's end: the warp's raw accumulators (8 slots x 16 per lane) go
+// to this CTA's workspace slot ([warp][slot][16][lane]: coalesced), tensor memory is zeroed
+// behind, then the warp's flag is released once every lane's stores are visible.
+__device__ __noinline__ void sk_store_part(const TmParams& p, uint32_t tw, int warp, int lane) {
+    float* sl = p.sk_slots + (size_t)blockIdx.x * kSlotFloats + (size_t)warp * kF * 16 * 32 + lane;
+#pragma unroll 1
+    for (int f = 0; f < kF; ++f) {
+        float a[16];
+        __syncwarp();
+        tmem_ld16(tw + 16u * f, a);
+        tmem_zero16(tw + 16u * f);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) sl[(f * 16 + i) * 32] = a[i];
+    }
+    __threadfence();
+    __syncwarp();
+    if (lane == 0) {
+        unsigned* fl = p.sk_flags + (size_t)blockIdx.x * kCompute + warp;
+        asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(fl), "r"(1u) : "memory");
+    }
+}
+
+// Balanced schedule, a head segment's end: wait (bounded) for the flags of the unit's parts, held
+// by CTAs [pb0, pb1), then add their sums to the warp's accumulators in chunk order (a fixed
+// summation order).  A flag that never comes records a status bit and the parts are left out.
+__device__ __noinline__ void sk_add_parts(const TmParams& p, uint32_t tw, int warp, int lane, int pb0, int pb1) {
+    bool ok = true;
+    for (int b = pb0; b < pb1; ++b) {
+        unsigned ready = 0;
+        if (lane == 0) {
+            const unsigned* fl = p.sk_flags + (size_t)b * kCompute + warp;
+            const long long t0 = clock64();
+            while (true) {
+                asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(ready) : "l"(fl) : "memory");
+                if (ready) break;
+                if (clock64() - t0 > kTimeoutCycles) {
+                    atomicOr(p.status, kStatusPartTimeout);
+                    break;
+                }
+            }
+        }
+        ok = ok && __shfl_sync(0xffffffffu, ready, 0) != 0;
+    }
+    __syncwarp();   // the other lanes read the slots after lane 0's acquire
+    if (!ok) return;
+#pragma unroll 1
+    for (int f = 0; f < kF; ++f) {
+        float a[16];
+        __syncwarp();
+        tmem_ld16(tw + 16u * f, a);
+        for (int b = pb0; b < pb1; ++b) {
+            const float* sl = p.sk_slots + (size_t)b * kSlotFloats + (size_t)warp * kF * 16 * 32 + lane + f * 16 * 32;
+#pragma unroll
+            for (int i = 0; i < 16; ++i) a[i] += __ldcg(sl + 32 * i);
+        }
+        tmem_st16(tw + 16u * f, a);
+    }
+}
+
 // SORT (stride 1, fp32 only): each warp's blocks are dealt to its lanes by bank group.
 // SHIFT (stride 1): block j of a tile row covers output columns ox0 + 4j - 1 .. ox0 + 4j + 2, so
 // that a lane's window column 0 sits at 2 (mod 4) in the stage and each window row is one 8-byte
 // and one 16-byte shared load (without SHIFT: 4-byte, 16-byte, 4-byte, the 4-byte ones bank
 // conflicted).  Not used with the fused pool, whose 2x2 windows must lie inside one block.
-template <int S, typename TIn, bool SORT = false, bool SHIFT = false>
+template <int S, typename TIn, bool SORT = false, bool SHIFT = false, bool SK = false>
 __global__ void __launch_bounds__(kThreadsTM, 1)
     pconv_tm(const TmParams p, const __grid_constant__ CUtensorMap tmap) {
     constexpr int RY = 4, RX = 4;
@@ -333,11 +418,33 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     const uint32_t full0 = smem_u32(bar), empty0 = full0 + 8 * kStages;
 
     // this CTA's units: blockIdx.x, blockIdx.x + gridDim.x, ... (one per CTA unless the launch is
-    // persistent); their chunks form one stream q = 0 .. Q-1 through the three stages, so the
-    // next unit's first stages fill while the current one finishes
-    const int n_my = p.n_units > (int)blockIdx.x ? (p.n_units - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+    // persistent), or with the balanced schedule the units its chunk range [lo, hi) touches;
+    // their chunks form one stream q = 0 .. Q-1 through the three stages, so the next unit's
+    // first stages fill while the current one finishes
     Unit* s_units = reinterpret_cast<Unit*>(smem + p.kb_off);   // at most kMaxUnitsPerCta
-    if ((int)threadIdx.x < n_my) s_units[threadIdx.x] = unit_of<S>(p, blockIdx.x + threadIdx.x * gridDim.x);
+    int n_my;
+    if constexpr (SK) {
+        const long long P = gridDim.x, T = p.sk_total, nck = p.n_chunks;
+        const long long lo = T * blockIdx.x / P, hi = T * (blockIdx.x + 1) / P;
+        const long long u0 = lo / nck;
+        n_my = hi > lo ? (int)((hi - 1) / nck - u0 + 1) : 0;
+        if ((int)threadIdx.x < n_my) {
+            const long long u = u0 + threadIdx.x;
+            Unit U = unit_of<S>(p, (int)u);
+            const int k0 = (int)(max(lo, u * nck) - u * nck), k1 = (int)(min(hi, (u + 1) * nck) - u * nck);
+            U.c_lo += k0 * p.CK;
+            U.nck = k1 - k0;
+            U.sk = k0 > 0 ? kRolePart : (k1 < nck ? kRoleHead : kRoleFull);
+            if (U.sk == kRoleHead) {   // the CTAs holding chunks k1 .. nck-1: the next ones
+                const long long last = (u + 1) * nck - 1;   // CTA of chunk c: ceil((c+1) P / T) - 1
+                U.sk |= (int)(((last + 1) * P + T - 1) / T) << 2;
+            }
+            s_units[threadIdx.x] = U;
+        }
+    } else {
+        n_my = p.n_units > (int)blockIdx.x ? (p.n_units - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+        if ((int)threadIdx.x < n_my) s_units[threadIdx.x] = unit_of<S>(p, blockIdx.x + threadIdx.x * gridDim.x);
+    }
 
     if (!p.use_tma) {   // the fallback writes only in-image elements: zero all stages once
         float* z = reinterpret_cast<float*>(smem + p.stage_off);
@@ -471,6 +578,15 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
         const int g = U.g0 + wg;
         const int n = U.n0 + img;
         const int oyb = U.oy0 + by * RY, oxb = U.ox0 + bx * RX - (SHIFT ? 1 : 0);
+        // balanced schedule: a part only publishes its raw sums; a head first adds its unit's
+        // parts into tensor memory (out of line: the common path keeps its registers)
+        if constexpr (SK) {
+            if ((U.sk & 3) == kRolePart) {
+                sk_store_part(p, tw, warp, lane);
+                return;
+            }
+            if ((U.sk & 3) == kRoleHead) sk_add_parts(p, tw, warp, lane, blockIdx.x + 1, U.sk >> 2);
+        }
 #pragma unroll 1
         for (int f = 0; f < kF; ++f) {
             float a[16];
@@ -1328,12 +1444,19 @@ bool pdl_enabled() {
     return on;
 }
 
+// The balanced schedule can be switched off (PATCONV_BALANCED=0): plans then take whole units.
+bool balanced_enabled() {
+    static const bool on = [] {
+        const char* e = std::getenv("PATCONV_BALANCED");
+        return !(e && e[0] == '0');
+    }();
+    return on;
+}
+
 template <typename... KArgs, typename... Args>
-cudaError_t launch(void (*kern)(KArgs...), unsigned grid, unsigned block, size_t smem, cudaStream_t st,
-                   const Args&... args) {
+cudaError_t launch_ex(bool cooperative, void (*kern)(KArgs...), unsigned grid, unsigned block, size_t smem,
+                      cudaStream_t st, const Args&... args) {
     cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(block);
@@ -1342,10 +1465,24 @@ cudaError_t launch(void (*kern)(KArgs...), unsigned grid, unsigned block, size_t
     cfg.attrs = attr;
     cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
     const bool captured = cudaStreamIsCapturing(st, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone;
-    cfg.numAttrs = pdl_enabled() && !captured ? 1 : 0;
+    if (cooperative) {   // CTAs that wait on each other: all resident at once
+        attr[0].id = cudaLaunchAttributeCooperative;
+        attr[0].val.cooperative = 1;
+        cfg.numAttrs = 1;
+    } else {
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.numAttrs = pdl_enabled() && !captured ? 1 : 0;
+    }
     const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, args...);
     const cudaError_t l = cudaGetLastError();
     return e != cudaSuccess ? e : l;
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch(void (*kern)(KArgs...), unsigned grid, unsigned block, size_t smem, cudaStream_t st,
+                   const Args&... args) {
+    return launch_ex(false, kern, grid, block, smem, st, args...);
 }
 
 using EncodeTiledFn = PFN_cuTensorMapEncodeTiled_v12000;
@@ -1396,8 +1533,15 @@ struct Plan {
     long long ctas = 0;           // CTAs of one split
     int lane_sort = 0;            // stride 1: pconv_tm deals blocks to lanes by bank group
     int shift = 0;                // stride 1: blocks start at output columns 4j - 1 (SHIFT)
-    size_t ws_bytes = 0;          // workspace the chosen split needs (0 without a split)
+    int streamk = 0;              // balanced schedule over sm_count() CTAs (KS = 1)
+    size_t ws_bytes = 0;          // workspace the chosen split or schedule needs (0: none)
 };
+
+// Workspace of the balanced schedule over P CTAs: a slot of raw accumulators per CTA, then a flag
+// per (CTA, warp).
+size_t streamk_bytes(long long P) {
+    return align_up((size_t)P * kSlotFloats * sizeof(float), 256) + (size_t)P * kCompute * sizeof(unsigned);
+}
 
 struct PlanCache : PlanCacheBase {
     std::mutex mu;
@@ -1492,8 +1636,9 @@ int window_wavefronts(const Plan& pl, int N, long long t, bool sorted) {
 }
 
 int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, int shift, Plan* out,
-                       double* cost) {
+                       double* cost, bool allow_sk, int es) {
     const int S = L->stride;
+    const bool tma_rows = ((size_t)W * es) % 16 == 0;   // the input goes through TMA (if aligned)
     const int Ho = (H - 1) / S + 1, Wo = (W - 1) / S + 1;
     int wg = 1;
     while (wg < L->G && wg < kCompute) wg *= 2;
@@ -1530,7 +1675,7 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
             const size_t desc_b = align_up((size_t)wg * ck * 8, 16);
             const size_t vals_b = (size_t)wg * std::max(maxk, 1) * 16;
             *stage_bytes = align_up(in_b + desc_b + vals_b, 128);
-            *kb_bytes = (size_t)kMaxUnitsPerCta * sizeof(int) * 12;   // the CTA's unit table
+            *kb_bytes = (size_t)kMaxUnitsPerCta * sizeof(Unit);   // the CTA's unit table
             return align_up(64 + *kb_bytes, 128) + kStages * *stage_bytes;
         };
         int ck = std::min(C, 64);
@@ -1610,6 +1755,36 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
             }
             pl->smem = layout(pl->CK, pl->maxk, &pl->stage_bytes, &pl->kb_bytes);
         }
+        // balanced schedule: P = sm_count() CTAs take equal ranges of the units' chunk sequence
+        // (KS = 1); a unit cut at a range boundary is finished by the CTA holding its first
+        // chunks, which adds the later CTAs' raw sums from their workspace slots.  Every CTA gets
+        // T / P chunks instead of whole units, where the last partial wave of whole units leaves
+        // SMs idle (busy share <= 0.88) and there are at least 0.75 units per CTA.  It costs the
+        // slots' traffic (256 KiB per CTA out and in, about 14 us a launch measured on VGG-16)
+        // and the launch overlap of the previous kernel (a cooperative launch), so it is taken
+        // only with a 5 % margin.  Only for stride 1 and where the input goes through TMA
+        // (persistent CTAs)
+        pl->streamk = 0;
+        const long long U1 = pl->ctas;   // whole units without a split
+        const double busy = (double)U1 / ((double)sms * ((U1 + sms - 1) / sms));
+        if (S == 1 && allow_sk && balanced_enabled() && tma_rows && busy <= 0.88 && 4 * U1 >= 3 * sms) {
+            const long long T = U1 * nck_total;
+            const size_t skb = streamk_bytes(sms);
+            if (T >= 2 * sms && U1 <= (long long)(kMaxUnitsPerCta - 2) * sms && ws_avail >= skb) {
+                const double cost_sk = (double)U1 * (C + 2.0 * nck_total) / sms + 4.0 * ck + 42.0;
+                if (cost_sk < 0.95 * steps) {
+                    steps = cost_sk;
+                    pl->streamk = 1;
+                    pl->KS = 1;
+                    pl->CK = ck;
+                    pl->c_split = nck_total * ck;
+                    pl->n_chunks = nck_total;
+                    pl->maxk = std::max(maxk_for(ck), 1);
+                    pl->ws_bytes = skb;
+                    pl->smem = layout(pl->CK, pl->maxk, &pl->stage_bytes, &pl->kb_bytes);
+                }
+            }
+        }
         return steps;
     };
 
@@ -1677,11 +1852,12 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
 // layer's mean kept kernels per (channel, group), 0.87 at 2.4 and 1 from 8 on.
 double shift_gain(double kept_per_channel) { return std::min(1.0, 0.82 + 0.0225 * kept_per_channel); }
 
-int make_plan(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out, int pool = 0) {
+int make_plan(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out, int pool = 0,
+              bool allow_sk = true, int es = 4) {
     pp_layer* ML = const_cast<pp_layer*>(L);   // the cache is the only mutable part of a handle
     std::call_once(ML->plans_once, [ML] { ML->plans.reset(new PlanCache); });
     auto* cache = static_cast<PlanCache*>(ML->plans.get());
-    const auto key = std::make_tuple(N, H, W, ws_avail, pool);
+    const auto key = std::make_tuple(N, H, W, ws_avail, (pool * 2 + (allow_sk ? 1 : 0)) * 8 + es);
     {
         std::lock_guard<std::mutex> g(cache->mu);
         auto it = cache->plans.find(key);
@@ -1692,13 +1868,14 @@ int make_plan(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out
     }
     Plan pl;
     double cost = 0;
-    const int rc = make_plan_uncached(L, N, H, W, ws_avail, 0, &pl, &cost);
+    const int rc = make_plan_uncached(L, N, H, W, ws_avail, 0, &pl, &cost, allow_sk, es);
     if (rc != PP_OK) return rc;
     if (L->stride == 1 && !pool) {   // shifted blocks where their estimate is lower
         Plan ps;
         double cs = 0;
         const double kpc = (double)L->beta / ((double)L->G * L->cin_g);
-        if (make_plan_uncached(L, N, H, W, ws_avail, 1, &ps, &cs) == PP_OK && cs * shift_gain(kpc) < cost) pl = ps;
+        if (make_plan_uncached(L, N, H, W, ws_avail, 1, &ps, &cs, allow_sk, es) == PP_OK && cs * shift_gain(kpc) < cost)
+            pl = ps;
     }
     std::lock_guard<std::mutex> g(cache->mu);
     if (cache->plans.size() >= 256) cache->plans.clear();
@@ -1755,7 +1932,7 @@ __global__ void splitk_reduce_pool(const float* __restrict__ ws, T* __restrict__
 // Raise the kernel's dynamic shared-memory limit to the device's opt-in maximum once per device
 // (a launch needs at most that), so that later calls, including ones under stream capture, make
 // no attribute call.
-template <int S, typename T, bool SORT, bool SHIFT>
+template <int S, typename T, bool SORT, bool SHIFT, bool SK>
 bool allow_max_smem(size_t need) {
     static std::atomic<int> done[64];
     int dev = 0;
@@ -1764,19 +1941,35 @@ bool allow_max_smem(size_t need) {
     int optin = 0;
     if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess) return false;
     if ((size_t)optin < need) return false;
-    if (cudaFuncSetAttribute(pconv_tm<S, T, SORT, SHIFT>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin) != cudaSuccess)
+    if (cudaFuncSetAttribute(pconv_tm<S, T, SORT, SHIFT, SK>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin) != cudaSuccess)
         return false;
     done[dev].store(1, std::memory_order_release);
     return true;
+}
+
+using TmKernel = void (*)(const TmParams, const CUtensorMap);
+
+// The kernel variant for a plan: the balanced-schedule variants (SK) exist for stride 1 only,
+// where the planner takes that schedule.
+template <int S, typename T, bool SORT, bool SHIFT>
+TmKernel pick_tm(bool sk, size_t smem, bool* ok) {
+    if constexpr (S == 1) {
+        if (sk) {
+            *ok = allow_max_smem<S, T, SORT, SHIFT, true>(smem);
+            return pconv_tm<S, T, SORT, SHIFT, true>;
+        }
+    }
+    *ok = allow_max_smem<S, T, SORT, SHIFT, false>(smem);
+    return pconv_tm<S, T, SORT, SHIFT, false>;
 }
 
 template <int S, typename T>
 int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int relu, int N, int H, int W, int Ho,
               int Wo, void* ws, size_t ws_bytes, cudaStream_t st, int pool = 0) {
     Plan pl;
-    const int rc = make_plan(L, N, H, W, ws ? ws_bytes : 0, &pl, pool);
+    const int rc = make_plan(L, N, H, W, ws ? ws_bytes : 0, &pl, pool, true, (int)sizeof(T));
     if (rc != PP_OK) return rc;
-    if (pl.KS > 1 && reinterpret_cast<uintptr_t>(ws) % 16 != 0) return PP_ERR_ALIGN;
+    if ((pl.KS > 1 || pl.streamk) && reinterpret_cast<uintptr_t>(ws) % 16 != 0) return PP_ERR_ALIGN;
     if (pool && pl.shift) return PP_ERR_SHAPE;   // never planned: pool windows must lie in one block
     TmParams p{};
     p.x = x;
@@ -1853,35 +2046,38 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
         if (r != CUDA_SUCCESS) p.use_tma = 0;
         p.tma_bytes = (unsigned)((size_t)p.BWb * p.IH * p.CK * p.NB * es);
     }
-    auto kern = pconv_tm<S, T, false, false>;
-    bool smem_ok;
+    // balanced schedule (TMA path only: the copy fallback keeps one CTA per unit)
+    p.streamk = S == 1 && pl.streamk && p.use_tma ? 1 : 0;
+    const bool sk = p.streamk != 0;
+    TmKernel kern;
+    bool smem_ok = false;
     if constexpr (S == 1 && sizeof(T) == 4) {
-        if (pl.lane_sort && pl.shift) {
-            kern = pconv_tm<1, float, true, true>;
-            smem_ok = allow_max_smem<1, float, true, true>(smem);
-        } else if (pl.lane_sort) {
-            kern = pconv_tm<1, float, true, false>;
-            smem_ok = allow_max_smem<1, float, true, false>(smem);
-        } else if (pl.shift) {
-            kern = pconv_tm<1, float, false, true>;
-            smem_ok = allow_max_smem<1, float, false, true>(smem);
-        } else {
-            smem_ok = allow_max_smem<1, float, false, false>(smem);
-        }
+        if (pl.lane_sort && pl.shift) kern = pick_tm<1, float, true, true>(sk, smem, &smem_ok);
+        else if (pl.lane_sort) kern = pick_tm<1, float, true, false>(sk, smem, &smem_ok);
+        else if (pl.shift) kern = pick_tm<1, float, false, true>(sk, smem, &smem_ok);
+        else kern = pick_tm<1, float, false, false>(sk, smem, &smem_ok);
     } else if constexpr (S == 1) {
-        if (pl.shift) {
-            kern = pconv_tm<1, T, false, true>;
-            smem_ok = allow_max_smem<1, T, false, true>(smem);
-        } else {
-            smem_ok = allow_max_smem<1, T, false, false>(smem);
-        }
+        if (pl.shift) kern = pick_tm<1, T, false, true>(sk, smem, &smem_ok);
+        else kern = pick_tm<1, T, false, false>(sk, smem, &smem_ok);
     } else {
-        smem_ok = allow_max_smem<S, T, false, false>(smem);
+        kern = pick_tm<S, T, false, false>(false, smem, &smem_ok);
     }
     if (!smem_ok) return PP_ERR_CUDA;
     const long long units = pl.ctas * pl.KS;
     if (units > INT_MAX) return PP_ERR_SHAPE;
     p.n_units = (int)units;
+    if (p.streamk) {
+        const long long P = sm_count();
+        if (!ws || ws_bytes < streamk_bytes(P)) return PP_ERR_BUFFER;
+        p.sk_total = pl.ctas * pl.n_chunks;
+        p.sk_slots = static_cast<float*>(ws);
+        p.sk_flags = reinterpret_cast<unsigned*>(static_cast<unsigned char*>(ws) +
+                                                 align_up((size_t)P * kSlotFloats * sizeof(float), 256));
+        if (cudaMemsetAsync(p.sk_flags, 0, (size_t)P * kCompute * sizeof(unsigned), st) != cudaSuccess)
+            return PP_ERR_CUDA;
+        if (launch_ex(true, kern, (unsigned)P, kThreadsTM, smem, st, p, tmap) != cudaSuccess) return PP_ERR_CUDA;
+        return PP_OK;
+    }
     // TMA path: one persistent CTA per SM walks its units as one chunk stream (the halo is zero
     // filled by the TMA unit, so stages carry over between tiles); the copy fallback relies on
     // stages zeroed once, so there every unit gets its own CTA
@@ -2207,15 +2403,16 @@ int pp_conv_pool_ws(pp_handle h, const void* x, int dtype, int N, int H, int W, 
 }
 
 namespace {
-int conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info, int pool) {
+int conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info, int pool,
+              int es) {
     if (!h || !info) return PP_ERR_NULL;
     if (N < 1 || H < 1 || W < 1 || n_info < 1) return PP_ERR_SHAPE;
-    int64_t v[15] = {0};
+    int64_t v[16] = {0};
     if (!h->fast || h->depthwise) {
         v[0] = h->depthwise ? 2 : 3;   // depthwise kernel / generic kernel: no plan, no workspace
     } else {
         Plan pl;
-        const int rc = make_plan(h, N, H, W, workspace_bytes, &pl, pool);
+        const int rc = make_plan(h, N, H, W, workspace_bytes, &pl, pool, true, es);
         if (rc != PP_OK) return rc;
         v[0] = 1;
         v[1] = pl.KS;
@@ -2235,19 +2432,29 @@ int conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t*
         v[11] = pl.n_chunks;
         v[13] = pl.lane_sort;
         v[14] = pl.shift;
+        v[15] = pl.streamk;
+        if (pl.streamk) v[12] = sm_count();
     }
-    for (int i = 0; i < n_info && i < 15; ++i) info[i] = v[i];
+    for (int i = 0; i < n_info && i < 16; ++i) info[i] = v[i];
     return PP_OK;
 }
 }  // namespace
 
 int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info) {
-    return conv_plan(h, N, H, W, workspace_bytes, info, n_info, 0);
+    return conv_plan(h, N, H, W, workspace_bytes, info, n_info, 0, 4);
 }
 
 int pp_conv_pool_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info) {
     if (h && (h->depthwise || !h->fast)) return PP_ERR_PATH;
-    return conv_plan(h, N, H, W, workspace_bytes, info, n_info, 1);
+    return conv_plan(h, N, H, W, workspace_bytes, info, n_info, 1, 4);
+}
+
+int pp_conv_plan_dt(pp_handle h, int dtype, int pool, int N, int H, int W, size_t workspace_bytes, int64_t* info,
+                    int n_info) {
+    if (dtype != PP_F32 && dtype != PP_F16) return PP_ERR_DTYPE;
+    if (pool != 0 && pool != 1) return PP_ERR_ARG;
+    if (pool && h && (h->depthwise || !h->fast)) return PP_ERR_PATH;
+    return conv_plan(h, N, H, W, workspace_bytes, info, n_info, pool, dtype == PP_F32 ? 4 : 2);
 }
 
 int pp_conv_workspace_size(pp_handle h, int N, int H, int W, size_t* bytes) {
@@ -2264,9 +2471,15 @@ int pp_conv_static_scratch(pp_handle h, const void* x, int dtype, int N, int H, 
     // the argument errors of pp_conv_ws come first, before the scratch size is considered
     const int v = validate_conv(h, x, dtype, N, H, W, bias, relu, y);
     if (v != PP_OK || N == 0) return v;
+    // the input-channel split pp_conv_ws would choose with an unlimited workspace (the balanced
+    // schedule left out: the array holds split partial sums only)
     size_t need = 0;
-    const int rc = pp_conv_workspace_size(h, N, H, W, &need);
-    if (rc != PP_OK) return rc;
+    if (!h->depthwise && h->fast) {
+        Plan pl;
+        const int rc = make_plan(h, N, H, W, (size_t)-1, &pl, 0, false);
+        if (rc != PP_OK) return rc;
+        need = pl.ws_bytes;
+    }
     if (need > kStaticScratchBytes) return PP_ERR_SCRATCH;
     void* scratch = static_scratch_address();
     if (!scratch) return PP_ERR_CUDA;

@@ -470,10 +470,13 @@ def _split_case():
 
 
 def test_split_is_planned_for_small_images():
+    """14x14 maps leave SMs idle with whole units: with a workspace the input-channel split
+    (their 56-byte fp32 rows take the copy fallback, which keeps one CTA per unit, so not the
+    balanced schedule), without one a single pass."""
     L, W, b, x = _split_case()
     lay = api.pp_pack(W, None, L.keep)
     plan = lay.plan(x.shape, lay.workspace_bytes(x.shape))
-    assert plan["path"] == 1 and plan["splits"] > 1
+    assert plan["path"] == 1 and plan["splits"] > 1 and plan["streamk"] == 0
     assert lay.plan(x.shape, 0)["splits"] == 1
     big = api.pp_pack(WL.weights(WL.vgg16()[1]), None, 0.3)
     assert big.plan((32, 64, 224, 224), 1 << 34)["splits"] == 1
@@ -489,6 +492,24 @@ def test_split_matches_oracle_single_pass_and_is_deterministic():
     assert OC.max_norm_err(y_split[[0, 31]], ref, den) <= 1e-4
     d = np.abs(y_split - y_one) / np.maximum(np.abs(y_one), 1e-3)
     assert float(np.max(d)) < 1e-3                       # only fp32 summation order differs
+
+
+def test_balanced_schedule_matches_oracle_and_is_deterministic():
+    """VGG-16 layer 9 at batch 32 (the balanced schedule): the same result on every run (the
+    head of a cut unit adds its parts in chunk order), the oracle's within tolerance, and the
+    whole-unit schedule's up to fp32 summation order (the schedule off: no workspace)."""
+    L = WL.vgg16()[8]
+    W, b, x = WL.weights(L), WL.bias(L), WL.layer_input(L, 32)
+    lay = api.pp_pack(W, None, L.keep)
+    assert lay.plan(x.shape, lay.workspace_bytes(x.shape))["streamk"] == 1
+    y1, _ = run_gpu(W, x, b, L.keep, ws=True)
+    y2, _ = run_gpu(W, x, b, L.keep, ws=True)
+    y0, _ = run_gpu(W, x, b, L.keep, ws=False)
+    assert np.array_equal(y1, y2)
+    ref, den = oracle(W, x[[0, 31]], b, L.keep)
+    assert OC.max_norm_err(y1[[0, 31]], ref, den) <= 1e-4
+    full_den = OC.denominator(x[[7]].astype(np.float64), OPR.project(W, OP.default8(), L.keep)["W_hat"], b, 1)
+    assert OC.max_norm_err(y1[[7]], y0[[7]], full_den) <= 1e-5
 
 
 def test_split_with_small_workspace_and_fp16():

@@ -11,6 +11,10 @@ from paper_2003_06513_gb300 import workloads as WL
 
 SMEM_MAX = 227 * 1024
 MAX_CHUNKS = 256      # input-channel stages one unit may walk
+SMS = 152             # the planner's SM count without a GPU (a GB300)
+# balanced schedule: a slot of 16 warps x 8 slots x 16 x 32 fp32 accumulators per CTA, then a flag
+# per (CTA, warp)
+STREAMK_BYTES = SMS * 16 * 8 * 16 * 32 * 4 + SMS * 16 * 4
 
 
 def _check(layer, shape, ws):
@@ -24,7 +28,11 @@ def _check(layer, shape, ws):
     assert 1 <= pl["chunks_per_unit"] <= MAX_CHUNKS
     # a split needs its workspace, and never more than the caller gave
     out_bytes = 4 * shape[0] * layer.cout * ((shape[2] - 1) // layer.stride + 1) * ((shape[3] - 1) // layer.stride + 1)
-    if pl["splits"] == 1:
+    if pl["streamk"]:
+        assert pl["splits"] == 1 and pl["ctas"] == SMS
+        assert pl["workspace_bytes"] == STREAMK_BYTES <= ws
+        assert pl["chunks_per_unit"] * pl["units"] >= 2 * SMS
+    elif pl["splits"] == 1:
         assert pl["workspace_bytes"] == 0
     else:
         assert pl["workspace_bytes"] == pl["splits"] * out_bytes <= ws
@@ -34,9 +42,10 @@ def _check(layer, shape, ws):
     assert per_split * pl["splits"] >= cin > per_split * (pl["splits"] - 1)
     # units: tiles x filter chunks x splits; persistent CTAs never exceed the units
     assert pl["units"] % pl["splits"] == 0
-    assert pl["ctas"] <= pl["units"]
+    assert pl["ctas"] <= pl["units"] or pl["streamk"]
     assert pl["lane_sort"] in (0, 1) and (layer.stride == 1 or pl["lane_sort"] == 0)
     assert pl["shift"] in (0, 1) and (layer.stride == 1 or pl["shift"] == 0)
+    assert pl["streamk"] in (0, 1)
     return pl
 
 

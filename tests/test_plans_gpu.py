@@ -25,7 +25,10 @@ TOL = {"f32": 1e-4, "f16": 2e-3}
 SMS_TABLE = 64        # units one persistent CTA holds in its table
 
 
-def _run(cout, cin, n, h, w, keep, io, pool=False, stride=1, seed=0, relu_in=True):
+CAP = 32 << 20        # a workspace below the balanced schedule's (39 MB): the channel split
+
+
+def _run(cout, cin, n, h, w, keep, io, pool=False, stride=1, seed=0, relu_in=True, ws_cap=None):
     rng = np.random.default_rng(seed)
     W = (rng.standard_normal((cout, cin, 3, 3)) * np.sqrt(2 / (9 * cin))).astype(np.float32)
     b = (rng.standard_normal(cout) * 0.1).astype(np.float32)
@@ -33,9 +36,11 @@ def _run(cout, cin, n, h, w, keep, io, pool=False, stride=1, seed=0, relu_in=Tru
                        dtype=np.float32 if io == "f32" else np.float16)
     layer = api.pp_pack(W, None, keep, 1, stride).bind("cuda")
     xt = torch.from_numpy(x).cuda()
-    nb = layer.workspace_bytes(xt.shape, pool)
+    nb = layer.workspace_bytes(xt.shape, pool, xt.dtype)
+    if ws_cap is not None:
+        nb = min(nb, ws_cap)
     ws = torch.empty(max(nb // 4, 1), device="cuda") if nb else None
-    plan = layer.plan(xt.shape, nb, pool2x2=pool)
+    plan = layer.plan(xt.shape, nb, pool, xt.dtype)
     y = layer.conv(xt, torch.from_numpy(b).cuda(), True, workspace=ws, pool2x2=pool)
     idx = [0, n - 1] if n > 1 else [0]
     Wh = OPR.project(W, OP.default8(), keep)["W_hat"]
@@ -68,7 +73,7 @@ def test_linear_tile(pool):
     plan, _ = _run(256, 256, 64, 28, 28, 1.0, "f32", pool=pool, seed=2)
     nb_rect = max(1, 32 * plan["spatial_warps"] // (plan["tile_by"] * plan["tile_bx"]))
     assert (plan["tile_by"], plan["tile_bx"]) == (7, 7) and plan["tile_nb"] > nb_rect   # linear
-    assert plan["shift"] == 0 and plan["splits"] > 1
+    assert plan["shift"] == 0 and plan["splits"] > 1 and plan["streamk"] == 0
 
 
 @pytest.mark.parametrize("pool", [False, True])
@@ -80,9 +85,34 @@ def test_bank_group_lane_order(pool):
 
 
 def test_multi_image_rectangles_with_split():
-    """7x7 maps: rectangles of 8 whole images (2x2 blocks each) and an 8-way split."""
-    plan, _ = _run(256, 256, 64, 7, 7, 0.5, "f32", seed=4)
-    assert plan["tile_nb"] == 8 and plan["splits"] > 1
+    """7x7 maps: rectangles of 8 whole images (2x2 blocks each) and an 8-way split (a workspace
+    too small for the balanced schedule)."""
+    plan, _ = _run(256, 256, 64, 7, 7, 0.5, "f32", seed=4, ws_cap=CAP)
+    assert plan["tile_nb"] == 8 and plan["splits"] > 1 and plan["streamk"] == 0
+
+
+@pytest.mark.parametrize("pool", [False, True])
+def test_balanced_schedule(pool):
+    """VGG-16 layer 9's shape (512 -> 512, 28x28, keep 0.3, batch 32, fp32): 256 whole units
+    would take 1.7 waves; the balanced schedule spreads their chunks over 152 CTAs and every
+    unit cut between two CTAs is summed by its head CTA."""
+    plan, _ = _run(512, 512, 32, 28, 28, 0.3, "f32", pool=pool, seed=11)
+    assert plan["streamk"] == 1 and plan["splits"] == 1 and plan["ctas"] == _sms()
+    assert plan["units"] % _sms() != 0
+
+
+def test_balanced_schedule_fp16():
+    """fp16 rows of 56 elements (112 bytes, through TMA), 154 units (just over one wave) on 152
+    CTAs: almost every CTA holds a head of one unit and a part of the next."""
+    plan, _ = _run(256, 256, 11, 56, 56, 0.3, "f16", seed=12)
+    assert plan["streamk"] == 1 and _sms() < plan["units"] < 2 * _sms()
+
+
+def test_no_balanced_schedule_without_tma_rows():
+    """fp16 rows of 28 elements (56 bytes: the copy fallback, one CTA per unit): the planner
+    keeps whole units (and the channel split) there."""
+    plan, _ = _run(512, 512, 32, 28, 28, 0.3, "f16", seed=13)
+    assert plan["streamk"] == 0
 
 
 def test_batch_one_split_32_ways():
@@ -127,7 +157,7 @@ def test_sweep_point_full_batch(c, hw, n, keep, io):
     x = WL.activations((n, c, hw, hw), L.x_seed, dtype=np.float32 if io == "f32" else np.float16)
     layer = api.pp_pack(W, None, keep).bind("cuda")
     xt = torch.from_numpy(x).cuda()
-    nb = layer.workspace_bytes(xt.shape)
+    nb = layer.workspace_bytes(xt.shape, dtype=xt.dtype)
     ws = torch.empty(max(nb // 4, 1), device="cuda") if nb else None
     y = layer.conv(xt, torch.from_numpy(b).cuda(), True, workspace=ws)
     idx = [0, n - 1] if n > 1 else [0]
