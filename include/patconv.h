@@ -190,11 +190,12 @@ int pp_conv_workspace_size(pp_handle h, int N, int H, int W, size_t* bytes);
  * bytes: persistent CTAs, at most one per SM unless the units overflow a CTA's unit table; the
  * copy fallback launches one CTA per unit), [13] 1 where a stride-1 fp32 launch deals each warp's
  * blocks to its lanes by shared-memory bank group (fewer conflicting window loads; rows of 7 or
- * 14 blocks), else 0; [14] 1 where the stride-1 blocks of a tile row start at output columns
- * 4j - 1 instead of 4j (each lane's input window then starts 8 bytes into a 16-byte group, so a
- * window row is one 8-byte and one 16-byte shared load instead of two bank-conflicted 4-byte
- * loads around a 16-byte one; never for pp_conv_pool_ws, which keeps blocks at 4j so that every
- * 2x2 pooling window lies inside one block), else 0; [15] 1 where the launch takes the balanced
+ * 14 blocks), else 0; [14] s where the stride-1 blocks of a tile row start at output columns
+ * 4j - s instead of 4j: s = 1 (each lane's input window then starts 8 bytes into a 16-byte group,
+ * so a window row is one 8-byte and one 16-byte shared load instead of two bank-conflicted 4-byte
+ * loads around a 16-byte one; never for pp_conv_pool_ws, whose 2x2 pooling windows must lie
+ * inside one block), s = 2 (fp32 pp_conv_pool_ws only: the window starts 4 bytes into a 16-byte
+ * group and a row is two 16-byte loads; block origins stay even), else 0; [15] 1 where the launch takes the balanced
  * schedule: one CTA per SM, each taking an equal share of all units' input-channel chunks
  * instead of whole units (whole units leave the SMs of the last partial wave idle); a unit cut
  * between two CTAs is finished by the CTA holding its first chunks, which adds the later ones'
@@ -205,7 +206,7 @@ int pp_conv_workspace_size(pp_handle h, int N, int H, int W, size_t* bytes);
 int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info);
 
 /* Launch plan of pp_conv_pool_ws (conv with the fused 2x2 max-pool) for a call shape and
- * workspace size: the same fields as pp_conv_plan; info[14] is always 0 here.  Layers without
+ * workspace size: the same fields as pp_conv_plan; info[14] is 0 or 2 here.  Layers without
  * the fused pooling (depthwise, other pattern libraries) return PP_ERR_PATH.  Host-only. */
 int pp_conv_pool_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info,
                       int n_info);

@@ -399,15 +399,18 @@ __device__ __noinline__ void sk_add_parts(const TmParams& p, uint32_t tw, int wa
 }
 
 // SORT (stride 1, fp32 only): each warp's blocks are dealt to its lanes by bank group.
-// SHIFT (stride 1): block j of a tile row covers output columns ox0 + 4j - 1 .. ox0 + 4j + 2, so
-// that a lane's window column 0 sits at 2 (mod 4) in the stage and each window row is one 8-byte
-// and one 16-byte shared load (without SHIFT: 4-byte, 16-byte, 4-byte, the 4-byte ones bank
-// conflicted).  Not used with the fused pool, whose 2x2 windows must lie inside one block.
-template <int S, typename TIn, bool SORT = false, bool SHIFT = false, bool SK = false>
+// SHIFT (stride 1): block j of a tile row covers output columns ox0 + 4j - SHIFT .. ox0 + 4j + 3
+// - SHIFT.  SHIFT 1: a lane's window column 0 sits at 2 (mod 4) in the stage and each window row
+// is one 8-byte and one 16-byte shared load (SHIFT 0: 4-byte, 16-byte, 4-byte, the 4-byte ones
+// bank conflicted); its blocks split 2x2 pooling windows, so the fused pool never uses it.
+// SHIFT 2 (fp32): column 0 at 1 (mod 4), each row two 16-byte loads, and blocks start at even
+// columns, so the fused pool's windows stay inside a block.
+template <int S, typename TIn, bool SORT = false, int SHIFT = 0, bool SK = false>
 __global__ void __launch_bounds__(kThreadsTM, 1)
     pconv_tm(const TmParams p, const __grid_constant__ CUtensorMap tmap) {
     constexpr int RY = 4, RX = 4;
     static_assert(!SHIFT || S == 1, "shifted blocks are a stride-1 layout");
+    static_assert(SHIFT != 2 || sizeof(TIn) == 4, "blocks at 4j - 2 are an fp32 layout");
     extern __shared__ __align__(128) unsigned char smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     // header: full[kStages] (stage filled), empty[kStages] (stage read by all 16 warps), the
@@ -525,9 +528,10 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     auto place_lane = [&]() {
         const Unit CU = s_units[ci];
         // block t (0 .. 32 * WS - 1) of the unit's tile: image, block row and column, and where
-        // the lane's window column 0 (input column ox0 * S - 1 of the block, one less with SHIFT)
-        // sits in the stage: d = 3 into the row for fp32 stages, 3 or 7 for fp16 ones (their
-        // origin is 16 bytes); with SHIFT 2, or 2 or 6
+        // the lane's window column 0 (input column ox0 * S - 1 of the block, SHIFT less) sits in
+        // the stage: d = 3 into the row for fp32 stages, 3 or 7 for fp16 ones (their origin is 16
+        // bytes); with SHIFT 1, 2 or 6; with SHIFT 2 the window address is that of column -1, at
+        // d = 0
         auto locate = [&](int t) {
             int rem;
             if (p.linear) {
@@ -543,20 +547,20 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
             }
             by = rem / p.BX;
             bx = rem - by * p.BX;
-            const int d = CU.ox0 * S - 1 - CU.ix0 - (SHIFT ? 1 : 0);
+            const int d = CU.ox0 * S - 1 - CU.ix0 - SHIFT - (SHIFT == 2 ? 1 : 0);
             in_off = active ? img * p.CK * plane + by * RY * S * p.BWb + bx * RX * S + d : d;
         };
         locate(blk);
         if constexpr (SORT) {
             static_assert(S == 1 && sizeof(TIn) == 4, "bank groups are those of fp32 stride-1 windows");
             // The warp's 32 blocks are dealt to its lanes so that each 8-lane phase of the
-            // 16-byte window loads (window columns 1-4 at in_off + 1, or 2-5 at in_off + 2 with
-            // SHIFT) meets distinct bank
+            // 16-byte window loads (window columns 1-4 at in_off + 1, 2-5 at in_off + 2 with
+            // SHIFT 1, -1..2 and 3..6 at in_off and in_off + 4 with SHIFT 2) meets distinct bank
             // groups where the blocks allow it: blocks are ordered by (rank among the blocks of
             // their bank group, bank group) and lane i takes the i-th.  Rows of 7 or 14 blocks
             // otherwise put two blocks of a phase on one bank group.  Idle lanes go last.  The
             // planner picks this instance where it lowers the wavefronts (window_wavefronts).
-            const int grp = active ? ((in_off + (SHIFT ? 2 : 1)) >> 2) & 7 : 8;
+            const int grp = active ? ((in_off + (SHIFT == 0 ? 1 : SHIFT == 1 ? 2 : 0)) >> 2) & 7 : 8;
             const unsigned same = __match_any_sync(0xffffffffu, grp);
             const int key = active ? 16 * __popc(same & ((1u << lane) - 1u)) + grp : 1024 + lane;   // distinct
             int pos = 0, src = 0;
@@ -577,7 +581,7 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     auto epilogue = [&](const Unit& U) {
         const int g = U.g0 + wg;
         const int n = U.n0 + img;
-        const int oyb = U.oy0 + by * RY, oxb = U.ox0 + bx * RX - (SHIFT ? 1 : 0);
+        const int oyb = U.oy0 + by * RY, oxb = U.ox0 + bx * RX - SHIFT;
         // balanced schedule: a part only publishes its raw sums; a head first adds its unit's
         // parts into tensor memory (out of line: the common path keeps its registers)
         if constexpr (SK) {
@@ -603,7 +607,7 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
                     const int oy = oyb + r;
                     if (oy >= p.Ho) break;
                     float* wr = wc + (size_t)oy * p.Wo;
-                    if constexpr (SHIFT) {   // columns oxb (3 mod 4), oxb+1..oxb+2 (a pair), oxb+3
+                    if constexpr (SHIFT == 1) {   // columns oxb (3 mod 4), oxb+1..oxb+2 (a pair), oxb+3
                         if (oxb >= 0 && oxb < p.Wo) wr[oxb] = a[r * RX];
                         if ((p.Wo % 2) == 0 && oxb + 3 <= p.Wo) {
                             *reinterpret_cast<float2*>(wr + oxb + 1) = make_float2(a[r * RX + 1], a[r * RX + 2]);
@@ -612,6 +616,18 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
                             if (oxb + 2 < p.Wo) wr[oxb + 2] = a[r * RX + 2];
                         }
                         if (oxb + 3 < p.Wo) wr[oxb + 3] = a[r * RX + 3];
+                    } else if constexpr (SHIFT == 2) {   // pairs at oxb (2 mod 4) and oxb+2; oxb >= -2
+#pragma unroll
+                        for (int h = 0; h < 2; ++h) {
+                            const int c = oxb + 2 * h;
+                            if (c < 0) continue;
+                            if ((p.Wo % 2) == 0 && c + 2 <= p.Wo) {
+                                *reinterpret_cast<float2*>(wr + c) = make_float2(a[r * RX + 2 * h], a[r * RX + 2 * h + 1]);
+                            } else {
+                                if (c < p.Wo) wr[c] = a[r * RX + 2 * h];
+                                if (c + 1 < p.Wo) wr[c + 1] = a[r * RX + 2 * h + 1];
+                            }
+                        }
                     } else if ((p.Wo % 4) == 0 && oxb + RX <= p.Wo) {
                         *reinterpret_cast<float4*>(wr + oxb) =
                             make_float4(a[r * RX], a[r * RX + 1], a[r * RX + 2], a[r * RX + 3]);
@@ -624,7 +640,8 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
                 continue;
             }
             const float b = p.bias ? p.bias[co] : 0.0f;
-            if (p.pool) {   // 2x2/2 max-pool inside the lane's 4x4 block (block origins are even)
+            if (p.pool) {   // 2x2/2 max-pool inside the lane's 4x4 block (block origins are even;
+                            // with SHIFT 2 the first pooled column is -1 in a row's first block)
                 const int Hp = p.Ho >> 1, Wp = p.Wo >> 1;
                 const int py0 = oyb >> 1, px0 = oxb >> 1;
                 TOut* yc = y + ((size_t)n * p.Cout + co) * Hp * Wp;
@@ -641,7 +658,11 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
                         v[c] = p.relu ? fmaxf(q, 0.0f) : q;
                     }
                     TOut* yr = yc + (size_t)py * Wp + px0;
-                    if (p.vec_pool && px0 + 2 <= Wp) {
+                    if constexpr (SHIFT == 2) {   // px0 odd: no pair store
+#pragma unroll
+                        for (int c = 0; c < 2; ++c)
+                            if (px0 + c >= 0 && px0 + c < Wp) yr[c] = from_f32<TOut>(v[c]);
+                    } else if (p.vec_pool && px0 + 2 <= Wp) {
                         if constexpr (sizeof(TOut) == 4) {
                             *reinterpret_cast<float2*>(yr) = make_float2(v[0], v[1]);
                         } else {
@@ -667,7 +688,7 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
                     const float q = a[r * RX + c] + b;
                     v[c] = p.relu ? fmaxf(q, 0.0f) : q;
                 }
-                if constexpr (SHIFT) {   // columns oxb (3 mod 4), oxb+1..oxb+2 (a pair), oxb+3
+                if constexpr (SHIFT == 1) {   // columns oxb (3 mod 4), oxb+1..oxb+2 (a pair), oxb+3
                     if (oxb >= 0 && oxb < p.Wo) yr[oxb] = from_f32<TOut>(v[0]);
                     if (p.vec_pair && oxb + 3 <= p.Wo) {
                         if constexpr (sizeof(TOut) == 4) {
@@ -680,6 +701,18 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
                         if (oxb + 2 < p.Wo) yr[oxb + 2] = from_f32<TOut>(v[2]);
                     }
                     if (oxb + 3 < p.Wo) yr[oxb + 3] = from_f32<TOut>(v[3]);
+                } else if constexpr (SHIFT == 2) {   // pairs at oxb (2 mod 4) and oxb+2; oxb >= -2
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        const int c = oxb + 2 * h;
+                        if (c < 0) continue;
+                        if (p.vec_pair && c + 2 <= p.Wo) {
+                            *reinterpret_cast<float2*>(yr + c) = make_float2(v[2 * h], v[2 * h + 1]);
+                        } else {
+                            if (c < p.Wo) yr[c] = from_f32<TOut>(v[2 * h]);
+                            if (c + 1 < p.Wo) yr[c + 1] = from_f32<TOut>(v[2 * h + 1]);
+                        }
+                    }
                 } else if (p.vec_store && oxb + RX <= p.Wo) {
                     if constexpr (sizeof(TOut) == 4) {
                         *reinterpret_cast<float4*>(yr + oxb) = make_float4(v[0], v[1], v[2], v[3]);
@@ -711,7 +744,9 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
             const uint32_t vals_addr = smem_u32(reinterpret_cast<const float4*>(st + p.vals_off) + wg * p.maxk);
             const int ckv = min(p.CK, CU.c_hi - CU.c_lo - ck * p.CK);
             constexpr int es = (int)sizeof(TIn);
-            if constexpr (S == 1 && es == 4 && SHIFT) {
+            if constexpr (S == 1 && es == 4 && SHIFT == 2) {
+                PP_STAGE_KERNELS_S1_B(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw, edge);
+            } else if constexpr (S == 1 && es == 4 && SHIFT == 1) {
                 PP_STAGE_KERNELS_S1_A(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw, edge);
             } else if constexpr (S == 1 && es == 4) {
                 PP_STAGE_KERNELS_S1(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw, edge);
@@ -1532,7 +1567,7 @@ struct Plan {
     size_t stage_bytes = 0, kb_bytes = 0, smem = 0;
     long long ctas = 0;           // CTAs of one split
     int lane_sort = 0;            // stride 1: pconv_tm deals blocks to lanes by bank group
-    int shift = 0;                // stride 1: blocks start at output columns 4j - 1 (SHIFT)
+    int shift = 0;                // stride 1: blocks start at output columns 4j - shift (SHIFT)
     int streamk = 0;              // balanced schedule over sm_count() CTAs (KS = 1)
     size_t ws_bytes = 0;          // workspace the chosen split or schedule needs (0: none)
 };
@@ -1549,7 +1584,7 @@ struct PlanCache : PlanCacheBase {
 };
 
 // Candidate spatial tiles of at most 32*WS blocks (4x4 outputs each; with shift, block j of a row
-// starts at output column 4j - 1, so a row of Wo outputs takes (Wo + 4) / 4 blocks).
+// starts at output column 4j - shift, so a row of Wo outputs takes (Wo + shift + 3) / 4 blocks).
 //   rectangles: BY x BX blocks of one image (several whole images when the rectangle is the
 //     whole image); stride-1 rows need 4*BX + 5 staged columns, stride-2 rows 8*BX + 4, rounded
 //     to a 16-byte multiple and padded to 4 (mod 8) floats so that rows four apart fall in other
@@ -1558,7 +1593,7 @@ struct PlanCache : PlanCacheBase {
 //     the whole images they touch; no lane idles even when an image's block count is no divisor
 //     of the lane count (28 x 28 outputs: 49 blocks).
 std::vector<TileChoice> tile_candidates(int N, int Ho, int Wo, int S, int lanes, int shift) {
-    const int nby = (Ho + 3) / 4, nbx = shift ? (Wo + 4) / 4 : (Wo + 3) / 4;
+    const int nby = (Ho + 3) / 4, nbx = (Wo + shift + 3) / 4;
     auto bw_of = [&](int bx) {
         int bw = S == 1 ? 4 * bx + 8 : 8 * bx + 4;
         if (bw % 8 == 0) bw += 4;
@@ -1645,7 +1680,7 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
     const int WS = kCompute / wg, lanes = 32 * WS;
     const int n_fchunks = (L->G + wg - 1) / wg;
     const int C = L->cin_g;
-    const int nby = (Ho + 3) / 4, nbx = shift ? (Wo + 4) / 4 : (Wo + 3) / 4;
+    const int nby = (Ho + 3) / 4, nbx = (Wo + shift + 3) / 4;
     const long long sms = sm_count();
     const size_t out_elems = (size_t)N * L->cout * Ho * Wo;
 
@@ -1844,12 +1879,13 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
     return PP_OK;
 }
 
-// Window loads with shifted blocks: one 8-byte and one 16-byte load per row instead of two bank-
-// conflicted 4-byte loads around a 16-byte one.  They pay where the window loads weigh most, at
-// few kept kernels per (input channel, filter group): VGG-16's keep-0.3 layers (2.4 kernels)
-// measured 6-13 % faster, its first layer (8 kernels, rows of 57 instead of 56 blocks) 16 %
-// slower.  The estimate of channel steps of the shifted plan is scaled by this factor of the
-// layer's mean kept kernels per (channel, group), 0.87 at 2.4 and 1 from 8 on.
+// Window loads with shifted blocks: one 8-byte and one 16-byte load per row (blocks at 4j - 1),
+// or two 16-byte loads (4j - 2), instead of two bank-conflicted 4-byte loads around a 16-byte
+// one.  They pay where the window loads weigh most, at few kept kernels per (input channel,
+// filter group): VGG-16's keep-0.3 layers (2.4 kernels) measured 6-13 % faster with blocks at
+// 4j - 1, its first layer (8 kernels, rows of 57 instead of 56 blocks) 16 % slower.  The estimate
+// of channel steps of a shifted plan is scaled by this factor of the layer's mean kept kernels per
+// (channel, group), 0.87 at 2.4 and 1 from 8 on.
 double shift_gain(double kept_per_channel) { return std::min(1.0, 0.82 + 0.0225 * kept_per_channel); }
 
 int make_plan(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out, int pool = 0,
@@ -1870,11 +1906,13 @@ int make_plan(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out
     double cost = 0;
     const int rc = make_plan_uncached(L, N, H, W, ws_avail, 0, &pl, &cost, allow_sk, es);
     if (rc != PP_OK) return rc;
-    if (L->stride == 1 && !pool) {   // shifted blocks where their estimate is lower
+    if (L->stride == 1 && (!pool || es == 4)) {   // shifted blocks where their estimate is lower:
+        // at 4j - 1 without the fused pool, at 4j - 2 (fp32 only) with it
         Plan ps;
         double cs = 0;
         const double kpc = (double)L->beta / ((double)L->G * L->cin_g);
-        if (make_plan_uncached(L, N, H, W, ws_avail, 1, &ps, &cs, allow_sk, es) == PP_OK && cs * shift_gain(kpc) < cost)
+        if (make_plan_uncached(L, N, H, W, ws_avail, pool ? 2 : 1, &ps, &cs, allow_sk, es) == PP_OK &&
+            cs * shift_gain(kpc) < cost)
             pl = ps;
     }
     std::lock_guard<std::mutex> g(cache->mu);
@@ -1932,7 +1970,7 @@ __global__ void splitk_reduce_pool(const float* __restrict__ ws, T* __restrict__
 // Raise the kernel's dynamic shared-memory limit to the device's opt-in maximum once per device
 // (a launch needs at most that), so that later calls, including ones under stream capture, make
 // no attribute call.
-template <int S, typename T, bool SORT, bool SHIFT, bool SK>
+template <int S, typename T, bool SORT, int SHIFT, bool SK>
 bool allow_max_smem(size_t need) {
     static std::atomic<int> done[64];
     int dev = 0;
@@ -1951,7 +1989,7 @@ using TmKernel = void (*)(const TmParams, const CUtensorMap);
 
 // The kernel variant for a plan: the balanced-schedule variants (SK) exist for stride 1 only,
 // where the planner takes that schedule.
-template <int S, typename T, bool SORT, bool SHIFT>
+template <int S, typename T, bool SORT, int SHIFT>
 TmKernel pick_tm(bool sk, size_t smem, bool* ok) {
     if constexpr (S == 1) {
         if (sk) {
@@ -1970,7 +2008,8 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
     const int rc = make_plan(L, N, H, W, ws ? ws_bytes : 0, &pl, pool, true, (int)sizeof(T));
     if (rc != PP_OK) return rc;
     if ((pl.KS > 1 || pl.streamk) && reinterpret_cast<uintptr_t>(ws) % 16 != 0) return PP_ERR_ALIGN;
-    if (pool && pl.shift) return PP_ERR_SHAPE;   // never planned: pool windows must lie in one block
+    // never planned: pool windows must lie in one block; blocks at 4j - 2 are fp32 only
+    if ((pool && pl.shift == 1) || (pl.shift == 2 && sizeof(T) != 4)) return PP_ERR_SHAPE;
     TmParams p{};
     p.x = x;
     p.y = y;
@@ -2052,15 +2091,20 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
     TmKernel kern;
     bool smem_ok = false;
     if constexpr (S == 1 && sizeof(T) == 4) {
-        if (pl.lane_sort && pl.shift) kern = pick_tm<1, float, true, true>(sk, smem, &smem_ok);
-        else if (pl.lane_sort) kern = pick_tm<1, float, true, false>(sk, smem, &smem_ok);
-        else if (pl.shift) kern = pick_tm<1, float, false, true>(sk, smem, &smem_ok);
-        else kern = pick_tm<1, float, false, false>(sk, smem, &smem_ok);
+        if (pl.lane_sort) {
+            if (pl.shift == 2) kern = pick_tm<1, float, true, 2>(sk, smem, &smem_ok);
+            else if (pl.shift == 1) kern = pick_tm<1, float, true, 1>(sk, smem, &smem_ok);
+            else kern = pick_tm<1, float, true, 0>(sk, smem, &smem_ok);
+        } else {
+            if (pl.shift == 2) kern = pick_tm<1, float, false, 2>(sk, smem, &smem_ok);
+            else if (pl.shift == 1) kern = pick_tm<1, float, false, 1>(sk, smem, &smem_ok);
+            else kern = pick_tm<1, float, false, 0>(sk, smem, &smem_ok);
+        }
     } else if constexpr (S == 1) {
-        if (pl.shift) kern = pick_tm<1, T, false, true>(sk, smem, &smem_ok);
-        else kern = pick_tm<1, T, false, false>(sk, smem, &smem_ok);
+        if (pl.shift) kern = pick_tm<1, T, false, 1>(sk, smem, &smem_ok);
+        else kern = pick_tm<1, T, false, 0>(sk, smem, &smem_ok);
     } else {
-        kern = pick_tm<S, T, false, false>(false, smem, &smem_ok);
+        kern = pick_tm<S, T, false, 0>(false, smem, &smem_ok);
     }
     if (!smem_ok) return PP_ERR_CUDA;
     const long long units = pl.ctas * pl.KS;

@@ -25,12 +25,17 @@ Window alignment (stride 1).  The input stage is a tensor copy whose first colum
     4-byte load, and every lane's 4-byte loads fall on 8 of the 32 banks (4-way conflicts);
   * blocks at output columns 4j - 1 (the "A" macros): column 0 at 2 (mod 4); each row is an
     8-byte load of columns 0-1 and a 16-byte load of columns 2-5, a third fewer shared-memory
-    wavefronts and one instruction fewer.
+    wavefronts and one instruction fewer;
+  * blocks at output columns 4j - 2 (the "B" macros, fp32): column 0 at 1 (mod 4); each row is
+    two 16-byte loads, of columns -1..2 and 3..6 (the window address is that of column -1), as
+    few wavefronts as the "A" layout, and every 2x2 pooling window of the block's outputs stays
+    inside the block.
 Packed taps.  A tap whose window pairs are the halves of one aligned load runs as fma.rn.f32x2
 on pairs of outputs (columns 0-1 and 2-3 of a row; same rounding as two fma.rn.f32): with
-blocks at 4j the centre-column taps (1, 4, 7), whose pairs are window columns (1, 2) and (3, 4);
-with blocks at 4j - 1 the side-column taps (0, 3, 6 and 2, 5, 8), whose pairs are (0, 1), (2, 3)
-and (2, 3), (4, 5).  The other taps read pairs that straddle the alignment and stay scalar.
+blocks at 4j or 4j - 2 the centre-column taps (1, 4, 7), whose pairs are window columns (1, 2)
+and (3, 4); with blocks at 4j - 1 the side-column taps (0, 3, 6 and 2, 5, 8), whose pairs are
+(0, 1), (2, 3) and (2, 3), (4, 5).  The other taps read pairs that straddle the alignment and
+stay scalar.
 Taps are applied in ascending raster order for every output.
 
 Every branch is warp-uniform (bra.uni), so no convergence code surrounds the loop.  The macros'
@@ -49,16 +54,18 @@ def taps(mask):
     return [t for t in range(9) if (mask >> t) & 1]
 
 
-def macro(S, half=False, aligned=False):
+def macro(S, half=False, shift=0):
     RY = RX = 4
     WY, WX = (RY - 1) * S + 3, (RX - 1) * S + 3
     R = RY * RX
     acc = ", ".join(f"a{i}" for i in range(R))
     rows = ", ".join(f"rb{r}" for r in range(WY))
     # operands: %0 channels, %1 descriptor address, %2 weights address, %3 window address of
-    # channel 0, %4 row pitch in bytes, %5 channel plane in bytes, %6 tensor-memory base, %7
-    # nonzero where the left neighbour lane does not hold the block to the left (stride 2)
+    # channel 0 (of window column -1 for shift 2), %4 row pitch in bytes, %5 channel plane in
+    # bytes, %6 tensor-memory base, %7 nonzero where the left neighbour lane does not hold the
+    # block to the left (stride 2)
     packed = S == 1
+    aligned = shift == 1
     pairs = (0, 2, 4) if aligned else (1, 3)      # window columns starting an aligned pair
 
     def packs(dx):                                # tap column dx (0..2) runs as f32x2
@@ -67,7 +74,7 @@ def macro(S, half=False, aligned=False):
          ".reg .pred P, EL;",
          f".reg .b32 cl, cnt, code, ta, pat, va, da, t1, {rows};",
          ".reg .b64 d, dd;",
-         f".reg .f32 x<{WY * WX}>, a<{R}>, w<4>;"]
+         f".reg .f32 x<{WY * WX}>, a<{R}>, w<4>, xs<2>;"]
     if packed:   # window pairs xq{5 * row + column}, accumulator pairs, duplicated weights
         L.append(f".reg .b64 xq<{5 * WY}>, ap<{R // 2}>, wq<4>;")
     if half:     # fp16 stage: 16-bit elements widened to fp32 as the window is loaded
@@ -121,6 +128,9 @@ def macro(S, half=False, aligned=False):
             L.append(f"cvt.f32.f16 x{base}, h2;")
             L += cvt_pair("pA", base + 1) + cvt_pair("pB", base + 3)
             L.append(f"cvt.f32.f16 x{base + 5}, h3;")
+        elif shift == 2:                     # columns -1..2 and 3..6 (16 bytes each)
+            L.append(f"ld.shared.v4.f32 {{xs0, x{base}, x{base + 1}, x{base + 2}}}, [rb{r}];")
+            L.append(f"ld.shared.v4.f32 {{x{base + 3}, x{base + 4}, x{base + 5}, xs1}}, [rb{r}+16];")
         elif aligned:                        # columns 0-1 (8 bytes), columns 2-5 (16 bytes)
             L.append(f"ld.shared.v2.f32 {{x{base}, x{base + 1}}}, [rb{r}];")
             L.append(f"ld.shared.v4.f32 {{x{base + 2}, x{base + 3}, x{base + 4}, x{base + 5}}}, [rb{r}+8];")
@@ -190,8 +200,10 @@ def macro(S, half=False, aligned=False):
           "CD:",
           "}"]
     body = "\\n\\t".join(L)
-    name = f"PP_STAGE_KERNELS_S{S}" + ("_H" if half else "") + (("A" if half else "_A") if aligned else "")
-    what = f"stride {S}{', fp16 stage' if half else ''}{', window column 0 at 2 mod 4' if aligned else ''}"
+    tag = {0: "", 1: "A", 2: "B"}[shift]
+    name = f"PP_STAGE_KERNELS_S{S}" + ("_H" if half else "") + ((tag if half else "_" + tag) if tag else "")
+    where = {0: "", 1: ", window column 0 at 2 mod 4", 2: ", window column 0 at 1 mod 4"}[shift]
+    what = f"stride {S}{', fp16 stage' if half else ''}{where}"
     return (f"// {what}: 4x4 outputs per lane, {WY}x{WX} input window\n"
             f"#define {name}(nch, desc_addr, vals_addr, win_addr, pitch_b, plane_b, tbase, edge) \\\n"
             f'    asm volatile("{body}" :: "r"(nch), "r"(desc_addr), "r"(vals_addr), "r"(win_addr), '
@@ -205,7 +217,9 @@ def generate() -> str:
         for half in (False, True):
             text.append(macro(S, half))
             if S == 1:
-                text.append(macro(S, half, aligned=True))
+                text.append(macro(S, half, shift=1))
+                if not half:
+                    text.append(macro(S, half, shift=2))
     return "\n".join(text)
 
 

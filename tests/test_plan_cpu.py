@@ -4,6 +4,7 @@ only, no GPU): invariants every plan must keep, over random call shapes and the 
 The planner assumes 152 SMs (a GB300) when no GPU is present; the invariants do not depend on that."""
 import numpy as np
 import pytest
+import torch
 
 from oracle import patterns as OP
 from paper_2003_06513_gb300 import _lib, api
@@ -44,14 +45,14 @@ def _check(layer, shape, ws):
     assert pl["units"] % pl["splits"] == 0
     assert pl["ctas"] <= pl["units"] or pl["streamk"]
     assert pl["lane_sort"] in (0, 1) and (layer.stride == 1 or pl["lane_sort"] == 0)
-    assert pl["shift"] in (0, 1) and (layer.stride == 1 or pl["shift"] == 0)
+    assert pl["shift"] in (0, 1, 2) and (layer.stride == 1 or pl["shift"] == 0)
     assert pl["streamk"] in (0, 1)
     return pl
 
 
 def _nbx(pl, wo):
-    """Blocks per output row: 4 columns each, starting at column 0, or at -1 when shifted."""
-    return (wo + 4) // 4 if pl["shift"] else (wo + 3) // 4
+    """Blocks per output row: 4 columns each, starting at column 0, or at -1 or -2 when shifted."""
+    return (wo + pl["shift"] + 3) // 4
 
 
 def _stage_geometry(pl, stride):
@@ -201,32 +202,36 @@ def test_other_paths_report_no_plan():
 
 
 def test_linear_tile_weighed_by_density():
-    """28x28 maps with blocks at columns 4j (7 blocks a row, the fused-pool layout): at VGG-16's
-    keep 0.3 the planner takes 4x7 rectangles without a split; at keep 1.0 the linear tile (every
-    lane busy) pays for its per-channel cost.  Without the pool the blocks start at 4j - 1 (8 a
-    row), and 4x8 rectangles keep every lane busy."""
+    """28x28 maps with blocks at columns 4j (7 blocks a row, the fp16 fused-pool layout): at
+    VGG-16's keep 0.3 the planner takes 4x7 rectangles without a split; at keep 1.0 the linear
+    tile (every lane busy) pays for its per-channel cost.  With blocks at 4j - 1 (no pool) or
+    4j - 2 (fp32 pool) a row has 8 blocks, and 4x8 rectangles keep every lane busy."""
+    f16 = torch.float16
     for L in WL.vgg16()[7:10]:
         layer = api.pp_pack(WL.weights(L), None, L.keep)
         shape = (32, L.cin, L.h, L.w)
-        pl = layer.plan(shape, layer.workspace_bytes(shape, True), pool2x2=True)
+        pl = layer.plan(shape, layer.workspace_bytes(shape, True, f16), pool2x2=True, dtype=f16)
         assert (pl["tile_by"], pl["tile_bx"], pl["tile_nb"], pl["splits"], pl["shift"]) == (4, 7, 1, 1, 0), L.name
+        pl = layer.plan(shape, layer.workspace_bytes(shape, True), pool2x2=True)
+        assert (pl["tile_by"], pl["tile_bx"], pl["tile_nb"], pl["splits"], pl["shift"]) == (4, 8, 1, 1, 2), L.name
         pl = layer.plan(shape, layer.workspace_bytes(shape))
         assert (pl["tile_by"], pl["tile_bx"], pl["tile_nb"], pl["splits"], pl["shift"]) == (4, 8, 1, 1, 1), L.name
     rng = np.random.default_rng(7)
     W = (rng.standard_normal((256, 256, 3, 3)) * np.sqrt(2 / (9 * 256))).astype(np.float32)
     shape = (64, 256, 28, 28)
     dense = api.pp_pack(W, None, 1.0)
-    pl = dense.plan(shape, dense.workspace_bytes(shape, True), pool2x2=True)
+    pl = dense.plan(shape, dense.workspace_bytes(shape, True, f16), pool2x2=True, dtype=f16)
     assert (pl["tile_by"], pl["tile_bx"]) == (7, 7) and pl["tile_nb"] > 1     # linear
     sparse = api.pp_pack(W, None, 0.25)
-    pl = sparse.plan(shape, sparse.workspace_bytes(shape, True), pool2x2=True)
+    pl = sparse.plan(shape, sparse.workspace_bytes(shape, True, f16), pool2x2=True, dtype=f16)
     assert (pl["tile_by"], pl["tile_bx"], pl["tile_nb"]) == (4, 7, 1)
 
 
 @pytest.mark.parametrize("which", ["vgg16", "resnet50"])
-def test_pool_plans_keep_blocks_at_4j(which):
-    """The fused pool needs every 2x2 window inside one lane's block: its plans never shift the
-    blocks, and they obey the same invariants.  Layers without the fused pool refuse the query."""
+def test_pool_plans_keep_block_origins_even(which):
+    """The fused pool needs every 2x2 window inside one lane's block: its plans start blocks at
+    4j, or at 4j - 2 for fp32, never at 4j - 1, and they obey the same invariants.  Layers without
+    the fused pool refuse the query."""
     layers = WL.vgg16() if which == "vgg16" else WL.resnet50_3x3()
     n = 32 if which == "vgg16" else 64
     for L in layers:
@@ -234,7 +239,8 @@ def test_pool_plans_keep_blocks_at_4j(which):
         shape = (n, L.cin, L.h, L.w)
         for ws in (0, layer.workspace_bytes(shape, True)):
             pl = layer.plan(shape, ws, pool2x2=True)
-            assert pl["path"] == 1 and pl["shift"] == 0
+            assert pl["path"] == 1 and pl["shift"] in (0, 2)
+            assert layer.plan(shape, ws, pool2x2=True, dtype=torch.float16)["shift"] == 0
             assert 0 < pl["smem_bytes"] <= SMEM_MAX and pl["filter_groups"] * pl["spatial_warps"] == 16
     rng = np.random.default_rng(3)
     dw = api.pp_pack(rng.standard_normal((16, 1, 3, 3)).astype(np.float32), None, 1.0, 16, 1)

@@ -3,9 +3,10 @@ full batch.
 
 Each case states the plan outcome it exercises and asserts it through layer.plan (the same plan
 the launch uses): linear tiles, rectangles of several whole images, the bank-group lane order,
-blocks shifted to start at output columns 4j - 1, the copy fallback for rows that are not a
-multiple of 16 bytes, fp16 stages through TMA without the fused pool, input-channel splits up to
-32 ways, more units than one persistent CTA per SM can hold in its table, and the fused pool.
+blocks shifted to start at output columns 4j - 1 (4j - 2 under the fp32 fused pool), the copy
+fallback for rows that are not a multiple of 16 bytes, fp16 stages through TMA without the fused
+pool, input-channel splits up to 32 ways, the balanced schedule, more units than one persistent
+CTA per SM can hold in its table, and the fused pool.
 Outputs are compared with the float64 oracle (§4.1 Eq. 1 over the projection of §4.3-4.4) on
 two sampled images of the full batch; the bar is 1e-4 of sum|W_hat||x| for fp32 I/O and 2e-3 for
 fp16 I/O.  Inputs come from the seeded generators only."""
@@ -78,10 +79,21 @@ def test_linear_tile(pool):
 
 @pytest.mark.parametrize("pool", [False, True])
 def test_bank_group_lane_order(pool):
-    """56x56 maps at keep 0.3: rows of 14 (or 15 shifted) blocks, each warp's blocks dealt to
-    lanes by shared-memory bank group; shifted blocks without the pool, blocks at 4j with it."""
+    """56x56 maps at keep 0.3: rows of 15 shifted blocks, each warp's blocks dealt to lanes by
+    shared-memory bank group; blocks at 4j - 1 without the pool, at 4j - 2 with it."""
     plan, _ = _run(128, 128, 16, 56, 56, 0.3, "f32", pool=pool, seed=3)
-    assert plan["lane_sort"] == 1 and plan["shift"] == (0 if pool else 1)
+    assert plan["lane_sort"] == 1 and plan["shift"] == (2 if pool else 1)
+
+
+@pytest.mark.parametrize("split", [False, True])
+@pytest.mark.parametrize("h,w", [(14, 28), (14, 26), (13, 27), (12, 30), (9, 13)])
+def test_pool_blocks_at_4j_minus_2(h, w, split):
+    """fp32 fused pool with blocks at output columns 4j - 2: widths 0, 1, 2 and 3 (mod 4), so a
+    row's first block pools columns -2..1 (pooled column -1 is not stored) and its last one may
+    hang over the edge; rows through TMA (28 floats) and the copy fallback (26, 27, 30, 13);
+    without a workspace and with a 32-way split (pooled in the split's reduction)."""
+    plan, _ = _run(64, 64, 8, h, w, 0.3, "f32", pool=True, seed=20 + w, ws_cap=None if split else 0)
+    assert plan["shift"] == 2 and (plan["splits"] > 1) == split
 
 
 def test_multi_image_rectangles_with_split():
