@@ -39,6 +39,7 @@
 #include <cstring>
 #include <map>
 #include <mutex>
+#include <numeric>
 #include <tuple>
 #include <vector>
 
@@ -1350,6 +1351,415 @@ __global__ void __launch_bounds__(kDwThreads) pconv_depthwise_staged(const __gri
     asm volatile("cp.async.wait_all;" ::: "memory");
 }
 
+// ------------------------------------------------------------------------------ streamed depthwise
+
+// Streamed depthwise kernel (16-byte aligned tensors).  Every warp of a persistent CTA is its own
+// copy/compute pipeline with a private ring of shared-memory stages and one mbarrier per stage, so
+// no CTA barrier separates copying from computing and each SM keeps many copies in flight.  A
+// chunk is
+//   * rows mode (MODE 0; rows of a multiple of 16 bytes, at most 256 elements): R output rows of
+//     one plane.  One tensor copy brings its (R - 1) S + 3 whole input rows, the rows above and
+//     below the image zero-filled by the copy.  Lane (h, g) computes output columns 4g .. 4g + 3
+//     of rows h RPL .. (h + 1) RPL - 1 and rolls three input rows through registers; the channel
+//     is the same for the whole warp, so pruned taps are skipped by uniform branches;
+//   * planes mode (MODE 1: one output column per lane; MODE 2: two, as packed FMAs): P
+//     consecutive whole planes, which are contiguous in NCHW, by one bulk copy.  A lane owns
+//     columns of one plane and walks down its rows, taking the neighbouring input columns from the
+//     adjacent lanes by shuffle; a pass of the warp covers NPW planes, so the lanes of a warp meet
+//     several channels and apply all nine taps (zeros at the pruned ones).  Outputs go to a
+//     shared-memory buffer that one bulk copy writes back.
+// Warp w of the grid takes chunks w, w + nw, w + 2 nw, ... (nw warps in the grid).  Each CTA holds
+// the nine taps, the bias and the tap mask of every channel in a table (kDwsTab words a channel).
+constexpr int kDwsWarps = 16;
+constexpr int kDwsThreads = 32 * kDwsWarps;
+constexpr int kDwsMaxStages = 4;
+constexpr int kDwsCW = 4;     // rows mode: output columns per lane
+constexpr int kDwsTab = 12;   // table words per channel: taps 0-8, bias, mask, unused
+
+struct DwsParams {
+    const void* x;
+    void* y;
+    const float* bias;
+    const uint32_t* perm;
+    const uint64_t* desc;
+    const uint32_t* kofs;
+    const float4* vals;
+    unsigned* status;
+    int N, C, H, W, Ho, Wo, relu, NS;
+    int nst;                              // stages per warp
+    long long n_chunks;
+    int R, RIN, n_bands, NCG, NHL, RPL;   // rows mode
+    int P, LPP, NPW;                      // planes mode: planes per chunk, lanes per plane, planes per pass
+    long long n_planes;                   // N * C
+    unsigned in_b;                        // bytes of one input stage
+    unsigned off_tab, off_area, area_b;   // shared memory: mbarriers | table | one area per warp
+    int vec_out;                          // rows mode: 4-output vector stores
+    uint16_t masks[kMaxPatterns];
+};
+
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, int x, int y, int z,
+                                            uint32_t mbar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];"
+        ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(mbar) : "memory");
+}
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t mbar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 ::"r"(dst), "l"(src), "r"(bytes), "r"(mbar) : "memory");
+}
+__device__ __forceinline__ void bulk_store(void* dst, uint32_t src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst), "r"(src), "r"(bytes)
+                 : "memory");
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+
+template <typename T>
+__device__ __forceinline__ float2 ld_pair(const T* q);
+template <>
+__device__ __forceinline__ float2 ld_pair<float>(const float* q) { return *reinterpret_cast<const float2*>(q); }
+template <>
+__device__ __forceinline__ float2 ld_pair<__half>(const __half* q) {
+    return __half22float2(*reinterpret_cast<const __half2*>(q));
+}
+template <typename T>
+__device__ __forceinline__ void st_pair(T* q, float a, float b);
+template <>
+__device__ __forceinline__ void st_pair<float>(float* q, float a, float b) { *reinterpret_cast<float2*>(q) = make_float2(a, b); }
+template <>
+__device__ __forceinline__ void st_pair<__half>(__half* q, float a, float b) {
+    *reinterpret_cast<__half2*>(q) = __floats2half2_rn(a, b);
+}
+
+// rows mode: the window columns of one staged row for output columns c0 .. c0 + 3: input columns
+// c0 - 1 .. c0 + 4 (stride 1) or 2 c0 - 1 .. 2 c0 + 7 (stride 2), zeros outside the image
+template <int S, typename T>
+__device__ __forceinline__ void dws_row(const T* row, int c0, int W, float (&v)[(kDwsCW - 1) * S + 3]) {
+    constexpr int NM = kDwsCW * S;     // columns c0 S .. c0 S + NM - 1: one or two 16-byte loads, or 8 bytes
+    const T* m = row + c0 * S;
+    if constexpr (sizeof(T) == 4) {
+#pragma unroll
+        for (int i = 0; i < NM; i += 4) {
+            const float4 q = *reinterpret_cast<const float4*>(m + i);
+            v[1 + i] = q.x;
+            v[2 + i] = q.y;
+            v[3 + i] = q.z;
+            v[4 + i] = q.w;
+        }
+    } else if constexpr (NM == 4) {
+        const uint2 u = *reinterpret_cast<const uint2*>(m);
+        const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&u.x));
+        const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&u.y));
+        v[1] = a.x;
+        v[2] = a.y;
+        v[3] = b.x;
+        v[4] = b.y;
+    } else {
+        const uint4 u = *reinterpret_cast<const uint4*>(m);
+        const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&w4[k]));
+            v[1 + 2 * k] = f.x;
+            v[2 + 2 * k] = f.y;
+        }
+    }
+    v[0] = c0 > 0 ? to_f32<T>(m[-1]) : 0.0f;
+    if constexpr (S == 1) v[NM + 1] = c0 + NM < W ? to_f32<T>(m[NM]) : 0.0f;
+}
+
+template <int S, typename T, int MODE>
+__global__ void __launch_bounds__(kDwsThreads, 1)
+    pconv_dw_stream(const __grid_constant__ DwsParams p, const __grid_constant__ CUtensorMap tmap) {
+    static_assert(MODE != 2 || S == 1, "two columns per lane is a stride-1 layout");
+    pdl_trigger();
+    extern __shared__ __align__(128) unsigned char smem[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t bar0 = smem_u32(smem) + 8u * kDwsMaxStages * warp;
+    float* tab = reinterpret_cast<float*>(smem + p.off_tab);
+    unsigned char* area = smem + p.off_area + (size_t)warp * p.area_b;
+    T* ob = reinterpret_cast<T*>(area + (size_t)p.nst * p.in_b);   // planes mode: output buffer
+    const T* x = static_cast<const T*>(p.x);
+    T* y = static_cast<T*>(p.y);
+    const long long wid = (long long)blockIdx.x * kDwsWarps + warp, nw = (long long)gridDim.x * kDwsWarps;
+    const int n_mine = p.n_chunks > wid ? (int)((p.n_chunks - 1 - wid) / nw + 1) : 0;
+    if (lane == 0) {
+        for (int s = 0; s < p.nst; ++s) mbar_init(bar0 + 8u * s, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    // taps and mask of every channel (slot s holds channel perm[s]; a pruned kernel has no entry:
+    // mask 0, all taps zero).  The packed layer is immutable once bound, so this runs while the
+    // previous kernel of the stream finishes.
+    for (int s = threadIdx.x; s < p.NS; s += kDwsThreads) {
+        const uint32_t co = p.perm[s];
+        if (co == kPadSlot) continue;
+        const int g = s >> 3, f = s & 7;
+        const uint64_t d = p.desc[g];
+        const int cnt = (int)(d & 15u);
+        int pat = -1;
+        uint32_t k0 = p.kofs[g];
+        for (int j = 0; j < cnt; ++j) {
+            const int code = (int)((d >> (4 + 6 * j)) & 63u);
+            if ((code >> 3) == f) {
+                pat = code & 7;
+                k0 += j;
+            }
+        }
+        const float4 v = pat >= 0 ? p.vals[k0] : make_float4(0.f, 0.f, 0.f, 0.f);
+        const unsigned m = pat >= 0 ? p.masks[pat] : 0u;
+        float* w = tab + (size_t)co * kDwsTab;
+        int k = 0;
+#pragma unroll
+        for (int t = 0; t < 9; ++t) {
+            const bool on = (m >> t) & 1u;
+            const float vk = k == 0 ? v.x : k == 1 ? v.y : k == 2 ? v.z : v.w;
+            w[t] = on ? vk : 0.0f;
+            k += on ? 1 : 0;
+        }
+        w[10] = __uint_as_float(m);
+        w[11] = 0.0f;
+    }
+    pdl_wait();   // activations and the bias from here on
+    for (int c = threadIdx.x; c < p.C; c += kDwsThreads) tab[(size_t)c * kDwsTab + 9] = p.bias ? p.bias[c] : 0.0f;
+
+    const size_t pb = (size_t)p.H * p.W * sizeof(T), opb = (size_t)p.Ho * p.Wo * sizeof(T);
+    auto issue = [&](int j) {   // lane 0: the copy of this warp's j-th chunk into stage j % nst
+        const long long ch = wid + (long long)j * nw;
+        const uint32_t bar = bar0 + 8u * (j % p.nst);
+        const uint32_t dst = smem_u32(area + (size_t)(j % p.nst) * p.in_b);
+        if constexpr (MODE == 0) {
+            const int q = (int)(ch / p.n_bands), b = (int)(ch - (long long)q * p.n_bands);
+            mbar_arrive_expect_tx(bar, (uint32_t)((size_t)p.W * p.RIN * sizeof(T)));
+            tma_load_3d(dst, &tmap, 0, b * p.R * S - 1, q, bar);
+        } else {
+            const long long q0 = ch * p.P;
+            const long long np = min((long long)p.P, p.n_planes - q0);
+            const uint32_t bytes = (uint32_t)((size_t)np * pb) & ~15u;   // the rest (end of x) by plain loads
+            mbar_arrive_expect_tx(bar, bytes);
+            if (bytes) bulk_load(dst, reinterpret_cast<const unsigned char*>(p.x) + (size_t)q0 * pb, bytes, bar);
+        }
+    };
+    const int first = min(p.nst, n_mine);
+    if (lane == 0)
+        for (int j = 0; j < first; ++j) issue(j);
+    int issued = first;
+    __syncthreads();   // the table is complete
+
+    // rows mode: rows h RPL .. of the chunk's band, output columns 4g .. 4g + 3
+    auto rows_chunk = [&](long long ch, const T* st) {
+        const int q = (int)(ch / p.n_bands), b = (int)(ch - (long long)q * p.n_bands);
+        const float* tw = tab + (size_t)(q % p.C) * kDwsTab;
+        float w[9];
+#pragma unroll
+        for (int t = 0; t < 9; ++t) w[t] = tw[t];
+        const float bv = tw[9];
+        const unsigned m = __float_as_uint(tw[10]);
+        const int oy0 = b * p.R, nro = min(p.R, p.Ho - oy0);
+        const int h = lane / p.NCG, g = lane - h * p.NCG;
+        const int r0 = h * p.RPL, r1 = min(r0 + p.RPL, nro);
+        if (h >= p.NHL || r0 >= r1) return;
+        const int c0 = g * kDwsCW;
+        constexpr int NI = (kDwsCW - 1) * S + 3;
+        float va[NI], vb[NI], vc[NI];   // staged rows r S, r S + 1, r S + 2 (input rows (oy0 + r) S - 1 ..)
+        dws_row<S, T>(st + (size_t)(r0 * S) * p.W, c0, p.W, va);
+        if constexpr (S == 1) dws_row<S, T>(st + (size_t)(r0 + 1) * p.W, c0, p.W, vb);
+        T* yq = y + ((size_t)q * p.Ho + oy0) * p.Wo + c0;
+        for (int r = r0; r < r1; ++r) {
+            if constexpr (S == 2) dws_row<S, T>(st + (size_t)(2 * r + 1) * p.W, c0, p.W, vb);
+            dws_row<S, T>(st + (size_t)(r * S + 2) * p.W, c0, p.W, vc);
+            float acc[kDwsCW];
+#pragma unroll
+            for (int j = 0; j < kDwsCW; ++j) acc[j] = bv;
+#pragma unroll
+            for (int dx = 0; dx < 3; ++dx) {
+                if ((m >> dx) & 1u) {
+#pragma unroll
+                    for (int j = 0; j < kDwsCW; ++j) acc[j] = fmaf(w[dx], va[j * S + dx], acc[j]);
+                }
+                if ((m >> (3 + dx)) & 1u) {
+#pragma unroll
+                    for (int j = 0; j < kDwsCW; ++j) acc[j] = fmaf(w[3 + dx], vb[j * S + dx], acc[j]);
+                }
+                if ((m >> (6 + dx)) & 1u) {
+#pragma unroll
+                    for (int j = 0; j < kDwsCW; ++j) acc[j] = fmaf(w[6 + dx], vc[j * S + dx], acc[j]);
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < kDwsCW; ++j) acc[j] = p.relu ? fmaxf(acc[j], 0.0f) : acc[j];
+            T* out = yq + (size_t)r * p.Wo;
+            if (p.vec_out) {
+                if constexpr (sizeof(T) == 4) {
+                    *reinterpret_cast<float4*>(out) = make_float4(acc[0], acc[1], acc[2], acc[3]);
+                } else {
+                    __half2 h0 = __floats2half2_rn(acc[0], acc[1]), h1 = __floats2half2_rn(acc[2], acc[3]);
+                    uint2 u;
+                    u.x = *reinterpret_cast<unsigned*>(&h0);
+                    u.y = *reinterpret_cast<unsigned*>(&h1);
+                    *reinterpret_cast<uint2*>(out) = u;
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < kDwsCW; ++j) out[j] = from_f32<T>(acc[j]);
+            }
+#pragma unroll
+            for (int i = 0; i < NI; ++i) {
+                if constexpr (S == 1) {
+                    va[i] = vb[i];
+                    vb[i] = vc[i];
+                } else {
+                    va[i] = vc[i];
+                }
+            }
+        }
+    };
+
+    // planes mode: the warp's passes over the chunk's planes; lane l owns columns of plane
+    // l / LPP of the pass; every lane runs the same loop (shuffles), idle lanes on zeros
+    auto planes_chunk = [&](long long ch, const T* st) {
+        const long long q0 = ch * p.P;
+        const int np = (int)min((long long)p.P, p.n_planes - q0);
+        const int pl_l = lane / p.LPP, gc = lane - pl_l * p.LPP;
+        const int c_first = (int)(q0 % p.C);
+        constexpr int CPL = MODE == 2 ? 2 : 1;
+        const bool has_l = gc > 0;
+        const bool has_r = (S == 1) && (gc + 1) * CPL < p.W;
+        for (int k = 0; k < np; k += p.NPW) {
+            const int pl = k + pl_l;
+            const bool act = pl_l < p.NPW && pl < np;
+            int c = act ? c_first + pl : 0;
+            while (c >= p.C) c -= p.C;
+            const float* tw = tab + (size_t)c * kDwsTab;
+            float w[9];
+#pragma unroll
+            for (int t = 0; t < 9; ++t) w[t] = tw[t];
+            const float bv = tw[9];
+            const T* xp = st + (size_t)(act ? pl : 0) * p.H * p.W + gc * CPL * S;
+            T* op = ob + (size_t)(act ? pl : 0) * p.Ho * p.Wo + gc * CPL;
+            // one input row: (left, a, b, right) = input columns c S - 1 .. of this lane's outputs,
+            // zeros outside the image (and on idle lanes)
+            auto fetch = [&](int iy, float (&v)[4]) {
+                const bool in = act && iy >= 0 && iy < p.H;
+                float a = 0.0f, b = 0.0f;
+                if constexpr (CPL == 2 || S == 2) {
+                    if (in) {
+                        const float2 f = ld_pair<T>(xp + (size_t)iy * p.W);
+                        a = f.x;
+                        b = f.y;
+                    }
+                } else {
+                    if (in) a = to_f32<T>(xp[(size_t)iy * p.W]);
+                }
+                const float hi = (CPL == 2 || S == 2) ? b : a;
+                const float l = __shfl_up_sync(0xffffffffu, hi, 1);
+                const float r = __shfl_down_sync(0xffffffffu, a, 1);
+                v[0] = has_l ? l : 0.0f;
+                v[1] = a;
+                v[2] = b;
+                v[3] = has_r ? r : 0.0f;
+            };
+            float v0[4], v1[4], v2[4];
+            v0[0] = v0[1] = v0[2] = v0[3] = 0.0f;   // input row -1
+            if constexpr (S == 1) fetch(0, v1);
+            for (int oy = 0; oy < p.Ho; ++oy) {
+                if constexpr (S == 1) {
+                    fetch(oy + 1, v2);
+                } else {
+                    fetch(2 * oy, v1);
+                    fetch(2 * oy + 1, v2);
+                }
+                if constexpr (CPL == 2) {   // outputs (a, b): taps on (left, a), (a, b), (b, right)
+                    auto row2 = [&](const float (&v)[4], int t0, float2 o) {
+                        o = __ffma2_rn(make_float2(w[t0], w[t0]), make_float2(v[0], v[1]), o);
+                        o = __ffma2_rn(make_float2(w[t0 + 1], w[t0 + 1]), make_float2(v[1], v[2]), o);
+                        return __ffma2_rn(make_float2(w[t0 + 2], w[t0 + 2]), make_float2(v[2], v[3]), o);
+                    };
+                    float2 o = make_float2(bv, bv);
+                    o = row2(v0, 0, o);
+                    o = row2(v1, 3, o);
+                    o = row2(v2, 6, o);
+                    if (p.relu) {
+                        o.x = fmaxf(o.x, 0.0f);
+                        o.y = fmaxf(o.y, 0.0f);
+                    }
+                    if (act) st_pair<T>(op + (size_t)oy * p.Wo, o.x, o.y);
+                } else {
+                    // stride 1: columns (left, a, right); stride 2: (left, a, b)
+                    const int i2 = S == 1 ? 3 : 2;
+                    float o = bv;
+                    o = fmaf(w[0], v0[0], o);
+                    o = fmaf(w[1], v0[1], o);
+                    o = fmaf(w[2], v0[i2], o);
+                    o = fmaf(w[3], v1[0], o);
+                    o = fmaf(w[4], v1[1], o);
+                    o = fmaf(w[5], v1[i2], o);
+                    o = fmaf(w[6], v2[0], o);
+                    o = fmaf(w[7], v2[1], o);
+                    o = fmaf(w[8], v2[i2], o);
+                    if (p.relu) o = fmaxf(o, 0.0f);
+                    if (act) op[(size_t)oy * p.Wo] = from_f32<T>(o);
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    if constexpr (S == 1) {
+                        v0[i] = v1[i];
+                        v1[i] = v2[i];
+                    } else {
+                        v0[i] = v2[i];
+                    }
+                }
+            }
+        }
+    };
+
+    bool ok = true;
+    int j = 0;
+    for (; j < n_mine; ++j) {
+        const int s = j % p.nst;
+        if (!mbar_wait_warp(bar0 + 8u * s, (uint32_t)((j / p.nst) & 1), p.status, kStatusFullTimeout, kTimeoutCycles)) {
+            ok = false;
+            break;
+        }
+        const long long ch = wid + (long long)j * nw;
+        T* st = reinterpret_cast<T*>(area + (size_t)s * p.in_b);
+        if constexpr (MODE == 0) {
+            rows_chunk(ch, st);
+        } else {
+            const long long q0 = ch * p.P;
+            const long long np = min((long long)p.P, p.n_planes - q0);
+            const size_t in_e = (size_t)np * pb / sizeof(T), full_e = (((size_t)np * pb) & ~(size_t)15) / sizeof(T);
+            if (full_e < in_e) {   // the end of x: the last few elements by plain loads
+                for (size_t i = full_e + lane; i < in_e; i += 32) st[i] = x[(size_t)q0 * (pb / sizeof(T)) + i];
+                __syncwarp();
+            }
+            if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");   // ob free again
+            __syncwarp();
+            planes_chunk(ch, st);
+            const size_t out_e = (size_t)np * opb / sizeof(T), fo_e = (((size_t)np * opb) & ~(size_t)15) / sizeof(T);
+            T* yc = y + (size_t)q0 * (opb / sizeof(T));
+            for (size_t i = fo_e + lane; i < out_e; i += 32) yc[i] = ob[i];   // the end of y by plain stores
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");      // ob visible to the bulk copy
+            __syncwarp();
+            if (lane == 0 && fo_e) bulk_store(yc, smem_u32(ob), (uint32_t)(fo_e * sizeof(T)));
+        }
+        __syncwarp();
+        if (j + p.nst < n_mine) {
+            if (lane == 0) {
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                issue(j + p.nst);
+            }
+            ++issued;
+        }
+    }
+    if (lane == 0) {
+        // after a timeout no copy of this warp may still be landing when the CTA exits
+        if (!ok)
+            for (int k = j; k < issued; ++k)
+                mbar_wait(bar0 + 8u * (k % p.nst), (uint32_t)((k / p.nst) & 1), p.status, kStatusDrainTimeout);
+        asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+    }
+    __syncwarp();
+}
+
 // ------------------------------------------------------------------------------ generic path
 
 struct TapTable {
@@ -2234,9 +2644,165 @@ bool dw_staged_plan(const pp_layer* L, const void* x, int N, int H, int W, int H
     return true;
 }
 
+// Streamed depthwise kernel: chunking for one call shape.  Rows mode needs rows of a multiple of
+// 16 bytes and at most 256 elements and output rows of a multiple of 4 columns (at most 128);
+// planes mode needs whole output rows of at most 32 lanes (one or two columns each).  The tensor
+// pointers (16-byte aligned x and y) are the launcher's to check.  Returns false where the
+// kernel does not apply (the earlier depthwise kernels run then).
+constexpr size_t kDwsRowsStage = 4096;     // target bytes of one input stage, rows mode
+constexpr size_t kDwsPlanesStage = 3200;   // planes mode
+constexpr int kDwsChunksPerWarp = 3;       // planes mode: smaller chunks until every warp has this many
+
+int dws_smem_optin() {
+    static std::atomic<int> cached[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 232448;   // no device: a GB300
+    int v = cached[dev].load();
+    if (v > 0) return v;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess || v <= 0) return 232448;
+    cached[dev].store(v);
+    return v;
+}
+
+bool dws_enabled() {
+    static const bool on = [] {
+        const char* e = std::getenv("PATCONV_DW_STREAM");
+        return !(e && e[0] == '0');
+    }();
+    return on;
+}
+
+bool dws_plan(const pp_layer* L, int N, int H, int W, int Ho, int Wo, size_t es, DwsParams* p, int* mode,
+              size_t* smem) {
+    const int S = L->stride, C = L->cout;
+    const long long n_planes = (long long)N * C;
+    if (n_planes > INT_MAX) return false;
+    const size_t optin = (size_t)dws_smem_optin();
+    p->off_tab = 8 * kDwsMaxStages * kDwsWarps;
+    p->off_area = (unsigned)align_up(p->off_tab + (size_t)C * kDwsTab * 4, 128);
+    if ((size_t)p->off_area + (size_t)kDwsWarps * 4096 > optin) return false;   // the table leaves too little room
+    const size_t per_warp = (optin - p->off_area) / kDwsWarps / 128 * 128;
+    const long long warps = (long long)sm_count() * kDwsWarps;
+    size_t out_b = 0;
+    const bool rows = ((size_t)W * es) % 16 == 0 && W <= 256 && Wo % kDwsCW == 0 && Wo / kDwsCW <= 32 &&
+                      (S == 1 ? W == Wo : W == 2 * Wo);
+    if (rows) {
+        p->NCG = Wo / kDwsCW;
+        p->NHL = 32 / p->NCG;
+        const int rin_max = std::max(3, (int)(kDwsRowsStage / ((size_t)W * es)));
+        int R = std::min(Ho, (rin_max - 3) / S + 1);
+        if (R >= p->NHL) R -= R % p->NHL;
+        p->R = R;
+        p->RIN = (R - 1) * S + 3;
+        p->RPL = (R + p->NHL - 1) / p->NHL;
+        p->n_bands = (Ho + R - 1) / R;
+        p->in_b = (unsigned)align_up((size_t)W * p->RIN * es, 128);
+        p->n_chunks = n_planes * p->n_bands;
+        *mode = 0;
+    } else {
+        if (S == 1 ? W != Wo : W != 2 * Wo) return false;
+        const int cpl = (S == 1 && W % 2 == 0) ? 2 : 1;
+        p->LPP = (Wo + cpl - 1) / cpl;
+        if (p->LPP > 32) return false;
+        p->NPW = 32 / p->LPP;
+        const size_t pb = (size_t)H * W * es, opb = (size_t)Ho * Wo * es;
+        // chunk starts 16-byte aligned in x and y; whole passes of the warp where that allows
+        auto al = [](size_t b) { return (long long)(16 / std::gcd(b, (size_t)16)); };
+        const long long A = std::lcm(std::lcm(al(pb), al(opb)), (long long)p->NPW);
+        long long P = std::max<long long>(A, (long long)(kDwsPlanesStage / pb) / A * A);
+        while (P > A && (n_planes + P - 1) / P < kDwsChunksPerWarp * warps) P -= A;
+        if ((size_t)P * pb > ((size_t)1 << 30)) return false;
+        p->P = (int)P;
+        p->in_b = (unsigned)align_up((size_t)P * pb, 128);
+        out_b = align_up((size_t)P * opb, 128);
+        p->n_chunks = (n_planes + P - 1) / P;
+        *mode = cpl;
+    }
+    if (out_b + 2 * (size_t)p->in_b > per_warp) return false;
+    p->nst = (int)std::min<size_t>(kDwsMaxStages, (per_warp - out_b) / p->in_b);
+    p->area_b = (unsigned)((size_t)p->nst * p->in_b + out_b);
+    p->n_planes = n_planes;
+    *smem = p->off_area + (size_t)kDwsWarps * p->area_b;
+    return true;
+}
+
+template <int S, typename T, int MODE>
+int launch_dws(const DwsParams& p, const CUtensorMap& tmap, size_t smem, cudaStream_t st) {
+    static std::atomic<int> done[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return PP_ERR_CUDA;
+    if (!done[dev].load(std::memory_order_acquire)) {
+        if (cudaFuncSetAttribute(pconv_dw_stream<S, T, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 dws_smem_optin()) != cudaSuccess)
+            return PP_ERR_CUDA;
+        done[dev].store(1, std::memory_order_release);
+    }
+    const long long grid = std::min<long long>(sm_count(), (p.n_chunks + kDwsWarps - 1) / kDwsWarps);
+    return launch(pconv_dw_stream<S, T, MODE>, (unsigned)std::max<long long>(grid, 1), kDwsThreads, smem, st, p, tmap) ==
+                   cudaSuccess ? PP_OK : PP_ERR_CUDA;
+}
+
+// The streamed depthwise kernel where it applies (PP_OK or an error), else 1.
+template <typename T>
+int try_dws(const pp_layer* L, const void* x, void* y, const float* bias, int relu, int N, int H, int W, int Ho,
+            int Wo, cudaStream_t st) {
+    if (!dws_enabled() || reinterpret_cast<uintptr_t>(x) % 16 != 0 || reinterpret_cast<uintptr_t>(y) % 16 != 0) return 1;
+    DwsParams p{};
+    int mode = 0;
+    size_t smem = 0;
+    if (!dws_plan(L, N, H, W, Ho, Wo, sizeof(T), &p, &mode, &smem)) return 1;
+    const unsigned char* img = static_cast<const unsigned char*>(L->dev);
+    p.x = x;
+    p.y = y;
+    p.bias = bias;
+    p.perm = reinterpret_cast<const uint32_t*>(img + L->off_perm);
+    p.desc = reinterpret_cast<const uint64_t*>(img + L->off_desc);
+    p.kofs = reinterpret_cast<const uint32_t*>(img + L->off_kofs);
+    p.vals = reinterpret_cast<const float4*>(img + L->off_vals);
+    p.status = status_word();
+    if (!p.status) return PP_ERR_CUDA;
+    p.N = N;
+    p.C = L->cout;
+    p.H = H;
+    p.W = W;
+    p.Ho = Ho;
+    p.Wo = Wo;
+    p.relu = relu;
+    p.NS = L->G * kF;
+    p.vec_out = 1;   // rows mode: Wo a multiple of 4 and y 16-byte aligned
+    for (int i = 0; i < kMaxPatterns; ++i) p.masks[i] = i < L->n_patterns ? L->masks[i] : 0;
+    CUtensorMap tmap;
+    std::memset(&tmap, 0, sizeof(tmap));
+    const size_t es = sizeof(T);
+    if (mode == 0) {   // planes x rows x columns, one box = RIN whole rows of one plane
+        if (!encode_tiled()) return 1;
+        const cuuint64_t dims[3] = {(cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)p.n_planes};
+        const cuuint64_t strides[2] = {(cuuint64_t)W * es, (cuuint64_t)H * W * es};
+        const cuuint32_t box[3] = {(cuuint32_t)W, (cuuint32_t)p.RIN, 1};
+        const cuuint32_t estr[3] = {1, 1, 1};
+        if (encode_tiled()(&tmap, es == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3,
+                           const_cast<void*>(x), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                           CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return 1;
+    }
+    const int S = L->stride;
+    if (S == 1) {
+        if (mode == 0) return launch_dws<1, T, 0>(p, tmap, smem, st);
+        if (mode == 1) return launch_dws<1, T, 1>(p, tmap, smem, st);
+        return launch_dws<1, T, 2>(p, tmap, smem, st);
+    }
+    if (mode == 0) return launch_dws<2, T, 0>(p, tmap, smem, st);
+    return launch_dws<2, T, 1>(p, tmap, smem, st);
+}
+
 template <typename T>
 int launch_depthwise(const pp_layer* L, const void* x, void* y, const float* bias, int relu, int N, int H, int W,
                      int Ho, int Wo, cudaStream_t st) {
+    {
+        const int rc = try_dws<T>(L, x, y, bias, relu, N, H, W, Ho, Wo, st);
+        if (rc != 1) return rc;
+    }
     {
         const unsigned char* img = static_cast<const unsigned char*>(L->dev);
         DwStagedParams q{};
@@ -2452,8 +3018,22 @@ int conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t*
     if (!h || !info) return PP_ERR_NULL;
     if (N < 1 || H < 1 || W < 1 || n_info < 1) return PP_ERR_SHAPE;
     int64_t v[16] = {0};
-    if (!h->fast || h->depthwise) {
-        v[0] = h->depthwise ? 2 : 3;   // depthwise kernel / generic kernel: no plan, no workspace
+    if (h->depthwise) {
+        v[0] = 2;   // depthwise kernels: no workspace
+        DwsParams q{};
+        int mode = 0;
+        size_t smem = 0;
+        const int Ho = (H - 1) / h->stride + 1, Wo = (W - 1) / h->stride + 1;
+        if (dws_enabled() && dws_plan(h, N, H, W, Ho, Wo, (size_t)es, &q, &mode, &smem)) {
+            v[1] = 1 + mode;
+            v[3] = q.n_chunks;
+            v[4] = mode == 0 ? q.R : q.P;
+            v[5] = q.nst;
+            v[10] = (int64_t)smem;
+            v[12] = std::min<long long>(sm_count(), (q.n_chunks + kDwsWarps - 1) / kDwsWarps);
+        }
+    } else if (!h->fast) {
+        v[0] = 3;   // generic kernel: no plan, no workspace
     } else {
         Plan pl;
         const int rc = make_plan(h, N, H, W, workspace_bytes, &pl, pool, true, es);

@@ -251,6 +251,32 @@ def test_depthwise_unaligned_input(dtype):
     assert OC.max_norm_err(y.double().cpu().numpy(), ref, den) <= TOL[dtype]
 
 
+@pytest.mark.parametrize("shape,stride,dtype,kernel", [
+    ((3, 21, 13, 12), 1, torch.float32, 1),    # rows mode, one band
+    ((2, 10, 37, 64), 1, torch.float16, 1),    # rows mode: two lane row-sets, a short last band
+    ((2, 12, 33, 64), 2, torch.float16, 1),    # rows mode, stride 2, odd height (zero rows below)
+    ((2, 8, 40, 48), 2, torch.float32, 1),     # rows mode, stride 2, five lane row-sets
+    ((3, 21, 13, 12), 1, torch.float16, 3),    # planes, two columns a lane; x ends inside a 16-byte block
+    ((3, 21, 13, 12), 2, torch.float32, 2),    # planes, stride 2; y ends inside a 16-byte block
+    ((2, 24, 9, 9), 1, torch.float16, 2),      # planes, odd width
+    ((1, 13, 7, 7), 1, torch.float16, 2),      # 13 planes: a short last chunk
+    ((5, 40, 14, 14), 2, torch.float16, 2),    # planes, stride 2 to 7x7
+])
+def test_streamed_depthwise(shape, stride, dtype, kernel):
+    """The streamed depthwise kernel in each of its modes (asserted through the plan), with the
+    chunk tails its bulk copies leave to plain loads and stores, against the oracle; NaN guard
+    regions around y catch stray writes."""
+    N, C, H, W = shape
+    rng = np.random.default_rng(C * 3 + H + stride)
+    Wd = (rng.standard_normal((C, 1, 3, 3)) * np.sqrt(2 / 9)).astype(np.float32)
+    x = rnd(shape, 7 * H + W, dtype=_np_dt(dtype))
+    b = (rng.standard_normal(C) * 0.1).astype(np.float32)
+    lay = api.pp_pack(Wd, None, 1.0, C, stride)
+    assert lay.plan(shape, 0, dtype=dtype)["dw_kernel"] == kernel
+    check(Wd, x, b, 1.0, stride, depthwise=True, dtype=dtype, guard=64)
+    check(Wd, x, b, 0.6, stride, relu=False, depthwise=True, dtype=dtype, guard=64)
+
+
 @pytest.mark.parametrize("m", [6, 8])
 def test_designed_library_end_to_end(m):
     """A library designed from the layer's own kernels (§4.2 heuristic) packs and runs through

@@ -300,3 +300,53 @@ def test_one_handle_planned_from_many_threads():
         t.join()
     assert not errors
     assert all(o == out[0] for o in out) and len(out[0]) == len(shapes)
+
+
+# --------------------------------------------------------------------------- streamed depthwise
+
+SMEM_OPTIN = 232448   # shared memory one CTA may opt into on a GB300
+
+
+def _dw_layer(C, stride=1, seed=5):
+    rng = np.random.default_rng(seed)
+    return api.pp_pack(rng.standard_normal((C, 1, 3, 3)).astype(np.float32), None, 1.0, C, stride)
+
+
+@pytest.mark.parametrize("idx,kernel", [(0, 1), (1, 1), (2, 1), (3, 1),      # 112 / 56-wide rows
+                                        (4, 3), (6, 2), (7, 3), (13, 2),     # 28 / 14-wide planes
+                                        (14, 2)])                            # 7-wide planes
+def test_streamed_depthwise_mode_per_mobilenet_layer(idx, kernel):
+    """MobileNet-V2's fp16 layers at batch 128: 112- and 56-wide maps stream bands of whole rows
+    through tensor copies (rows of 224 or 112 bytes); 28-, 14- and 7-wide maps stream runs of whole
+    planes (two output columns per lane where the width is even at stride 1)."""
+    L = WL.mobilenet_v2_dw()[idx]
+    lay = _dw_layer(L.cout, L.stride)
+    pl = lay.plan((128, L.cin, L.h, L.w), 0, dtype=torch.float16)
+    assert pl["path"] == 2 and pl["dw_kernel"] == kernel, pl
+    assert 2 <= pl["stages"] <= 4 and pl["smem_bytes"] <= SMEM_OPTIN
+    es, ho, wo = 2, L.ho, L.wo
+    n_planes = 128 * L.cout
+    if kernel == 1:   # rows mode: bands of R output rows, every band's input rows in one stage
+        R = pl["rows_or_planes"]
+        assert 1 <= R <= ho and ((R - 1) * L.stride + 3) * L.w * es <= 4096
+        assert pl["chunks"] == n_planes * -(-ho // R)
+    else:             # planes mode: chunk starts 16-byte aligned in x and y
+        P = pl["rows_or_planes"]
+        assert (P * L.h * L.w * es) % 16 == 0 and (P * ho * wo * es) % 16 == 0
+        assert pl["chunks"] == -(-n_planes // P)
+        lpp = -(-wo // (2 if kernel == 3 else 1))
+        assert lpp <= 32 and P % (32 // lpp) == 0      # whole passes of the warp
+    assert pl["ctas"] == min(152, -(-pl["chunks"] // 16))
+
+
+@pytest.mark.parametrize("shape,stride,dtype,kernel", [
+    ((3, 21, 13, 12), 1, torch.float32, 1),     # 48-byte rows
+    ((3, 21, 13, 12), 2, torch.float32, 2),     # 6 output columns: planes
+    ((3, 21, 13, 12), 1, torch.float16, 3),     # 24-byte rows: planes, two columns a lane
+    ((2, 24, 9, 9), 1, torch.float32, 2),       # odd width
+    ((1, 4, 9, 2100), 1, torch.float16, 0),     # rows too wide for either mode
+    ((2, 16, 20, 100), 1, torch.float16, 0),    # 200-byte rows, 100 columns: neither mode
+])
+def test_streamed_depthwise_applicability(shape, stride, dtype, kernel):
+    lay = _dw_layer(shape[1], stride)
+    assert lay.plan(shape, 0, dtype=dtype)["dw_kernel"] == kernel
