@@ -203,10 +203,13 @@ int pp_conv_workspace_size(pp_handle h, int N, int H, int W, size_t* bytes);
  * launch is cooperative and resets the flags with a small memset first; the input must go
  * through TMA, else the launch takes whole units), else 0.  For path 2 (depthwise), assuming
  * x and y 16-byte aligned (else the row-item kernels run): info[1] = 1 streamed kernel in rows
- * mode (bands of whole rows of one plane per tensor copy), 2 streamed kernel in planes mode with
- * one output column per lane, 3 the same with two columns per lane, 0 the row-item kernels;
- * [3] chunks, [4] output rows per chunk (rows mode) or planes per chunk, [5] shared-memory
- * stages per warp, [10] shared-memory bytes, [12] CTAs.  Writes min(n_info, 16) values.
+ * mode (bands of whole rows of one plane per tensor copy), 2 streamed kernel in planes mode at
+ * stride 2 (one output column per lane), 3 planes mode at stride 1 with rows of even width (two
+ * columns per lane), 4 the same for rows of odd width, 5 / 6 tiles mode at stride 1 (each lane a
+ * band of 7 output rows by 7 / 14 columns of one plane), 7 tiles mode at stride 2 (a lane a 7x7
+ * output plane), 0 the row-item kernels; [3] chunks, [4] output rows per chunk (rows mode) or
+ * planes per chunk, [5] shared-memory stages per warp, [6] warps per CTA, [10] shared-memory
+ * bytes, [12] CTAs.  Writes min(n_info, 16) values.
  * Host-only. */
 int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info);
 

@@ -108,8 +108,9 @@ class Layer:
              dtype=torch.float32) -> dict:
         """Launch plan pp_conv_ws (or, with pool2x2, pp_conv_pool_ws) would use for an input of
         shape [N, C, H, W] and dtype (pp_conv_plan_dt).  Depthwise layers report ``dw_kernel``:
-        1 streamed rows, 2 streamed planes (one column per lane), 3 streamed planes (two columns
-        per lane), 0 the row-item kernels (for 16-byte aligned x and y)."""
+        1 streamed rows, 2 streamed planes at stride 2, 3 / 4 streamed planes at stride 1 (rows of
+        even / odd width), 5 / 6 streamed tiles of 7 / 14 columns at stride 1, 7 streamed tiles at
+        stride 2, 0 the row-item kernels (for 16-byte aligned x and y)."""
         N, _, H, W = x_shape
         n = len(self.PLAN_KEYS)
         info = (ctypes.c_int64 * n)()
@@ -119,7 +120,7 @@ class Layer:
         if d["path"] == 2:   # depthwise: info[1] names the kernel, there is no split
             d = {"path": 2, "splits": 0, "workspace_bytes": 0, "dw_kernel": int(info[1]),
                  "chunks": int(info[3]), "rows_or_planes": int(info[4]), "stages": int(info[5]),
-                 "smem_bytes": int(info[10]), "ctas": int(info[12])}
+                 "warps": int(info[6]), "smem_bytes": int(info[10]), "ctas": int(info[12])}
         return d
 
     def workspace_bytes(self, x_shape, pool2x2: bool = False, dtype=torch.float32) -> int:

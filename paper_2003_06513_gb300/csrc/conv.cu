@@ -1362,12 +1362,13 @@ __global__ void __launch_bounds__(kDwThreads) pconv_depthwise_staged(const __gri
 //     below the image zero-filled by the copy.  Lane (h, g) computes output columns 4g .. 4g + 3
 //     of rows h RPL .. (h + 1) RPL - 1 and rolls three input rows through registers; the channel
 //     is the same for the whole warp, so pruned taps are skipped by uniform branches;
-//   * planes mode (MODE 1: one output column per lane; MODE 2: two, as packed FMAs): P
-//     consecutive whole planes, which are contiguous in NCHW, by one bulk copy.  A lane owns
-//     columns of one plane and walks down its rows, taking the neighbouring input columns from the
-//     adjacent lanes by shuffle; a pass of the warp covers NPW planes, so the lanes of a warp meet
-//     several channels and apply all nine taps (zeros at the pruned ones).  Outputs go to a
-//     shared-memory buffer that one bulk copy writes back.
+//   * planes mode (MODE 1: stride 2, one output column per lane; MODE 2 / 3: stride 1, two
+//     output columns per lane as packed FMAs, rows of even / odd width): P consecutive whole
+//     planes, which are contiguous in NCHW, by one bulk copy.  A lane owns columns of one plane
+//     and walks down its rows, taking the neighbouring input columns from the adjacent lanes by
+//     shuffle; a pass of the warp covers NPW planes, so the lanes of a warp meet several channels
+//     and apply all nine taps (zeros at the pruned ones).  Outputs go to a shared-memory buffer
+//     that one bulk copy writes back.
 // Warp w of the grid takes chunks w, w + nw, w + 2 nw, ... (nw warps in the grid).  Each CTA holds
 // the nine taps, the bias and the tap mask of every channel in a table (kDwsTab words a channel).
 constexpr int kDwsWarps = 16;
@@ -1390,9 +1391,12 @@ struct DwsParams {
     long long n_chunks;
     int R, RIN, n_bands, NCG, NHL, RPL;   // rows mode
     int P, LPP, NPW;                      // planes mode: planes per chunk, lanes per plane, planes per pass
+    int ipp, npc;                         // tiles mode: lane items per plane, row pieces per output row
     long long n_planes;                   // N * C
     unsigned in_b;                        // bytes of one input stage
     unsigned off_tab, off_area, area_b;   // shared memory: mbarriers | table | one area per warp
+    unsigned zoff;                        // tiles mode: a zero row within each warp's area
+    int nwarps;                           // warps per CTA (the launch's block is 32 nwarps threads)
     int vec_out;                          // rows mode: 4-output vector stores
     uint16_t masks[kMaxPatterns];
 };
@@ -1467,10 +1471,201 @@ __device__ __forceinline__ void dws_row(const T* row, int c0, int W, float (&v)[
     if constexpr (S == 1) v[NM + 1] = c0 + NM < W ? to_f32<T>(m[NM]) : 0.0f;
 }
 
+// Rows mode, one lane: output rows r0 .. r0 + nrows - 1 of a chunk's band at output columns c0 ..
+// c0 + 3, from staged rows r S, r S + 1, r S + 2 (`off`: element offset of staged row r0 S,
+// column c0 S; `W`: elements per staged row).  The taps are those of mask M, known at compile
+// time (one of the pattern library's masks, so each output takes exactly its kept taps; 0x1FF:
+// all nine, zeros at the pruned ones), applied in ascending raster order.  Input rows rotate
+// through a register ring unrolled by its length, so no row is copied.
+template <int S, typename T, unsigned M>
+__device__ __forceinline__ void dws_rows(const T* st, int off, int W, T* yr, int Wo, int nrows, bool has_l,
+                                         bool has_r, bool relu, const float (&w)[9], float bv) {
+    constexpr int NI = (kDwsCW - 1) * S + 3;
+    constexpr bool kL = (M & 0x49u) != 0;              // a tap in column dx = 0 (taps 0, 3, 6)
+    constexpr bool kR = S == 1 && (M & 0x124u) != 0;   // stride 1: a tap in column dx = 2 (2, 5, 8)
+    struct Row { float e[NI]; };
+    auto fetch = [&](Row& v) {
+        const T* m = st + off;
+        if constexpr (sizeof(T) == 4) {
+#pragma unroll
+            for (int i = 0; i < kDwsCW * S; i += 4) {
+                const float4 f = *reinterpret_cast<const float4*>(m + i);
+                v.e[1 + i] = f.x;
+                v.e[2 + i] = f.y;
+                v.e[3 + i] = f.z;
+                v.e[4 + i] = f.w;
+            }
+        } else if constexpr (S == 1) {
+            const uint2 u = *reinterpret_cast<const uint2*>(m);
+            const float2 f0 = __half22float2(*reinterpret_cast<const __half2*>(&u.x));
+            const float2 f1 = __half22float2(*reinterpret_cast<const __half2*>(&u.y));
+            v.e[1] = f0.x;
+            v.e[2] = f0.y;
+            v.e[3] = f1.x;
+            v.e[4] = f1.y;
+        } else {
+            const uint4 u = *reinterpret_cast<const uint4*>(m);
+            const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&w4[i]));
+                v.e[1 + 2 * i] = f.x;
+                v.e[2 + 2 * i] = f.y;
+            }
+        }
+        v.e[0] = 0.0f;
+        if constexpr (kL) {   // column c0 S - 1, read inside the stage and zeroed at the image's edge
+            const float l = to_f32<T>(m[has_l ? -1 : 0]);
+            v.e[0] = has_l ? l : 0.0f;
+        }
+        if constexpr (S == 1) {
+            v.e[5] = 0.0f;
+            if constexpr (kR) {
+                const float r = to_f32<T>(m[has_r ? 4 : 3]);
+                v.e[5] = has_r ? r : 0.0f;
+            }
+        }
+        off += W;
+    };
+    auto out = [&](const Row& u, const Row& v, const Row& x3) {
+        float a[kDwsCW];
+#pragma unroll
+        for (int j = 0; j < kDwsCW; ++j) {
+            float o = bv;
+#pragma unroll
+            for (int t = 0; t < 9; ++t) {
+                if ((M >> t) & 1u) {
+                    const Row& rr = t < 3 ? u : (t < 6 ? v : x3);
+                    o = fmaf(w[t], rr.e[j * S + t % 3], o);
+                }
+            }
+            a[j] = relu ? fmaxf(o, 0.0f) : o;
+        }
+        if constexpr (sizeof(T) == 4) {
+            *reinterpret_cast<float4*>(yr) = make_float4(a[0], a[1], a[2], a[3]);
+        } else {
+            __half2 h0 = __floats2half2_rn(a[0], a[1]), h1 = __floats2half2_rn(a[2], a[3]);
+            uint2 q;
+            q.x = *reinterpret_cast<unsigned*>(&h0);
+            q.y = *reinterpret_cast<unsigned*>(&h1);
+            *reinterpret_cast<uint2*>(yr) = q;
+        }
+        yr += Wo;
+    };
+    Row A, B, C;
+    if constexpr (S == 1) {
+        fetch(A);
+        fetch(B);
+        for (int r = 0; r < nrows; r += 3) {
+            fetch(C);
+            out(A, B, C);
+            if (r + 1 >= nrows) break;
+            fetch(A);
+            out(B, C, A);
+            if (r + 2 >= nrows) break;
+            fetch(B);
+            out(C, A, B);
+        }
+    } else {
+        fetch(A);
+        for (int r = 0; r < nrows; r += 2) {
+            fetch(B);
+            fetch(C);
+            out(A, B, C);
+            if (r + 1 >= nrows) break;
+            fetch(B);
+            fetch(A);
+            out(C, B, A);
+        }
+    }
+}
+
+// Tiles mode, one lane: output rows oy0 .. oy0 + BR - 1 and columns c0 .. c0 + PW - 1 of one plane,
+// computed in straight-line code: every input row of the tile is read once into a register ring
+// (rows above and below the image from a zero row), all offsets are compile-time constants, and
+// all nine taps are applied (zeros at the pruned ones), in ascending raster order.  `xp` / `op`:
+// the plane's first element in the stage / in the output buffer.  PAIRS: rows of even width with
+// c0 S even, so the staged row segments are read and the outputs written as element pairs.
+template <int S, typename T, int PW, int BR, bool PAIRS>
+__device__ __forceinline__ void dws_tile(const T* xp, T* op, const T* zrow, int W, int H, int Wo, int oy0, int c0,
+                                         bool relu, const float (&w)[9], float bv) {
+    constexpr int NM = PW * S;       // columns c0 S .. c0 S + NM - 1 (stride 2: through 2 (c0 + PW) - 1)
+    constexpr int NIN = NM + 2;      // with column c0 S - 1 in front and c0 S + NM behind
+    const bool has_l = c0 > 0;
+    const bool has_r = S == 1 && c0 + PW < W;   // stride 2 never reads column 2 (c0 + PW)
+    float v[3][NIN];
+    auto fetch = [&](int k, float (&r)[NIN]) {   // input row oy0 S - 1 + k
+        const int iy = oy0 * S - 1 + k;
+        const T* row = (iy >= 0 && iy < H) ? xp + iy * W + c0 * S : zrow;
+        if constexpr (PAIRS) {
+#pragma unroll
+            for (int i = 0; i < NM; i += 2) {
+                const float2 f = ld_pair<T>(row + i);
+                r[1 + i] = f.x;
+                r[2 + i] = f.y;
+            }
+        } else {
+#pragma unroll
+            for (int i = 0; i < NM; ++i) r[1 + i] = to_f32<T>(row[i]);
+        }
+        const float l = to_f32<T>(row[-1]);   // inside the stage (or the zero row); zeroed at the edge
+        r[0] = has_l ? l : 0.0f;
+        if constexpr (S == 1) {
+            const float rr = to_f32<T>(row[NM]);
+            r[NIN - 1] = has_r ? rr : 0.0f;
+        } else {
+            r[NIN - 1] = 0.0f;
+        }
+    };
+    auto out = [&](int orow, const float (&a)[NIN], const float (&b)[NIN], const float (&c)[NIN]) {
+        float o[PW];
+#pragma unroll
+        for (int j = 0; j < PW; ++j) {
+            float q = bv;
+            q = fmaf(w[0], a[j * S], q);
+            q = fmaf(w[1], a[j * S + 1], q);
+            q = fmaf(w[2], a[j * S + 2], q);
+            q = fmaf(w[3], b[j * S], q);
+            q = fmaf(w[4], b[j * S + 1], q);
+            q = fmaf(w[5], b[j * S + 2], q);
+            q = fmaf(w[6], c[j * S], q);
+            q = fmaf(w[7], c[j * S + 1], q);
+            q = fmaf(w[8], c[j * S + 2], q);
+            o[j] = relu ? fmaxf(q, 0.0f) : q;
+        }
+        T* d = op + (oy0 + orow) * Wo + c0;
+        if constexpr (PAIRS && PW % 2 == 0) {
+#pragma unroll
+            for (int j = 0; j < PW; j += 2) st_pair<T>(d + j, o[j], o[j + 1]);
+        } else {
+#pragma unroll
+            for (int j = 0; j < PW; ++j) d[j] = from_f32<T>(o[j]);
+        }
+    };
+    if constexpr (S == 1) {
+        fetch(0, v[0]);
+        fetch(1, v[1]);
+#pragma unroll
+        for (int r = 0; r < BR; ++r) {
+            fetch(r + 2, v[(r + 2) % 3]);
+            out(r, v[r % 3], v[(r + 1) % 3], v[(r + 2) % 3]);
+        }
+    } else {
+        fetch(0, v[0]);
+#pragma unroll
+        for (int r = 0; r < BR; ++r) {
+            fetch(2 * r + 1, v[(2 * r + 1) % 3]);
+            fetch(2 * r + 2, v[(2 * r + 2) % 3]);
+            out(r, v[(2 * r) % 3], v[(2 * r + 1) % 3], v[(2 * r + 2) % 3]);
+        }
+    }
+}
+
 template <int S, typename T, int MODE>
 __global__ void __launch_bounds__(kDwsThreads, 1)
     pconv_dw_stream(const __grid_constant__ DwsParams p, const __grid_constant__ CUtensorMap tmap) {
-    static_assert(MODE != 2 || S == 1, "two columns per lane is a stride-1 layout");
+    static_assert(MODE != 2 && MODE != 3 && MODE != 4 && MODE != 5 || S == 1, "a stride-1 layout");
+    static_assert(MODE != 6 || S == 2, "a stride-2 layout");
     pdl_trigger();
     extern __shared__ __align__(128) unsigned char smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1480,50 +1675,20 @@ __global__ void __launch_bounds__(kDwsThreads, 1)
     T* ob = reinterpret_cast<T*>(area + (size_t)p.nst * p.in_b);   // planes mode: output buffer
     const T* x = static_cast<const T*>(p.x);
     T* y = static_cast<T*>(p.y);
-    const long long wid = (long long)blockIdx.x * kDwsWarps + warp, nw = (long long)gridDim.x * kDwsWarps;
-    const int n_mine = p.n_chunks > wid ? (int)((p.n_chunks - 1 - wid) / nw + 1) : 0;
+    const int nwarps = (int)(blockDim.x >> 5), nthr = (int)blockDim.x;
+    const int wid = (int)blockIdx.x * nwarps + warp, nw = (int)gridDim.x * nwarps;   // chunks < 2^31
+    const int n_mine = (int)p.n_chunks > wid ? ((int)p.n_chunks - 1 - wid) / nw + 1 : 0;
     if (lane == 0) {
         for (int s = 0; s < p.nst; ++s) mbar_init(bar0 + 8u * s, 1);
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // the barriers, for the copies
     }
-    // taps and mask of every channel (slot s holds channel perm[s]; a pruned kernel has no entry:
-    // mask 0, all taps zero).  The packed layer is immutable once bound, so this runs while the
-    // previous kernel of the stream finishes.
-    for (int s = threadIdx.x; s < p.NS; s += kDwsThreads) {
-        const uint32_t co = p.perm[s];
-        if (co == kPadSlot) continue;
-        const int g = s >> 3, f = s & 7;
-        const uint64_t d = p.desc[g];
-        const int cnt = (int)(d & 15u);
-        int pat = -1;
-        uint32_t k0 = p.kofs[g];
-        for (int j = 0; j < cnt; ++j) {
-            const int code = (int)((d >> (4 + 6 * j)) & 63u);
-            if ((code >> 3) == f) {
-                pat = code & 7;
-                k0 += j;
-            }
-        }
-        const float4 v = pat >= 0 ? p.vals[k0] : make_float4(0.f, 0.f, 0.f, 0.f);
-        const unsigned m = pat >= 0 ? p.masks[pat] : 0u;
-        float* w = tab + (size_t)co * kDwsTab;
-        int k = 0;
-#pragma unroll
-        for (int t = 0; t < 9; ++t) {
-            const bool on = (m >> t) & 1u;
-            const float vk = k == 0 ? v.x : k == 1 ? v.y : k == 2 ? v.z : v.w;
-            w[t] = on ? vk : 0.0f;
-            k += on ? 1 : 0;
-        }
-        w[10] = __uint_as_float(m);
-        w[11] = 0.0f;
+    if constexpr (MODE >= 4) {   // this warp's zero row (tiles mode: rows above and below the image)
+        if (lane < 32) reinterpret_cast<uint32_t*>(area + p.zoff)[lane] = 0u;
     }
     pdl_wait();   // activations and the bias from here on
-    for (int c = threadIdx.x; c < p.C; c += kDwsThreads) tab[(size_t)c * kDwsTab + 9] = p.bias ? p.bias[c] : 0.0f;
-
     const size_t pb = (size_t)p.H * p.W * sizeof(T), opb = (size_t)p.Ho * p.Wo * sizeof(T);
     auto issue = [&](int j) {   // lane 0: the copy of this warp's j-th chunk into stage j % nst
-        const long long ch = wid + (long long)j * nw;
+        const long long ch = (long long)wid + (long long)j * nw;
         const uint32_t bar = bar0 + 8u * (j % p.nst);
         const uint32_t dst = smem_u32(area + (size_t)(j % p.nst) * p.in_b);
         if constexpr (MODE == 0) {
@@ -1542,172 +1707,241 @@ __global__ void __launch_bounds__(kDwsThreads, 1)
     if (lane == 0)
         for (int j = 0; j < first; ++j) issue(j);
     int issued = first;
+    // taps, bias and mask of every channel (slot s holds channel perm[s]; a pruned kernel has no
+    // entry: mask 0, all taps zero), decoded while the first copies are in flight: up to four
+    // slots a thread, their independent loads issued together (two rounds of L2 latency)
+    for (int s0 = threadIdx.x; s0 < p.NS; s0 += 4 * nthr) {
+        uint32_t co[4], ko[4];
+        uint64_t d[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int s = s0 + u * nthr;
+            const bool in = s < p.NS;
+            co[u] = in ? p.perm[s] : kPadSlot;
+            d[u] = in ? p.desc[s >> 3] : 0ull;
+            ko[u] = in ? p.kofs[s >> 3] : 0u;
+        }
+        float4 v[4];
+        float bi[4];
+        unsigned msk[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int f = (s0 + u * nthr) & 7;
+            const int cnt = (int)(d[u] & 15u);
+            int pat = -1, jj = 0;
+            for (int j2 = 0; j2 < cnt; ++j2) {
+                const int code = (int)((d[u] >> (4 + 6 * j2)) & 63u);
+                if ((code >> 3) == f) {
+                    pat = code & 7;
+                    jj = j2;
+                }
+            }
+            const bool live = co[u] != kPadSlot;
+            v[u] = live && pat >= 0 ? p.vals[ko[u] + jj] : make_float4(0.f, 0.f, 0.f, 0.f);
+            bi[u] = live && p.bias ? p.bias[co[u]] : 0.0f;
+            msk[u] = live && pat >= 0 ? p.masks[pat] : 0u;
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            if (co[u] == kPadSlot) continue;
+            float* w = tab + (size_t)co[u] * kDwsTab;
+            int k = 0;
+#pragma unroll
+            for (int t = 0; t < 9; ++t) {
+                const bool on = (msk[u] >> t) & 1u;
+                const float vk = k == 0 ? v[u].x : k == 1 ? v[u].y : k == 2 ? v[u].z : v[u].w;
+                w[t] = on ? vk : 0.0f;
+                k += on ? 1 : 0;
+            }
+            w[9] = bi[u];
+            w[10] = __uint_as_float(msk[u]);
+            w[11] = 0.0f;
+        }
+    }
     __syncthreads();   // the table is complete
 
-    // rows mode: rows h RPL .. of the chunk's band, output columns 4g .. 4g + 3
+    // rows mode: rows h RPL .. of the chunk's band, output columns 4g .. 4g + 3.  The channel is
+    // the same for the whole warp, so its tap mask selects once per chunk a row loop compiled for
+    // that pattern (the library's eight) or, for any other mask, for all nine taps.
+    const int W = p.W, H = p.H, Wo = p.Wo, Ho = p.Ho, C = p.C;
+    const bool relu = p.relu != 0;
     auto rows_chunk = [&](long long ch, const T* st) {
         const int q = (int)(ch / p.n_bands), b = (int)(ch - (long long)q * p.n_bands);
-        const float* tw = tab + (size_t)(q % p.C) * kDwsTab;
-        float w[9];
-#pragma unroll
-        for (int t = 0; t < 9; ++t) w[t] = tw[t];
-        const float bv = tw[9];
-        const unsigned m = __float_as_uint(tw[10]);
-        const int oy0 = b * p.R, nro = min(p.R, p.Ho - oy0);
+        const float4* tw = reinterpret_cast<const float4*>(tab + (size_t)(q % C) * kDwsTab);
+        const float4 t0 = tw[0], t1 = tw[1], t2 = tw[2];
+        const float w[9] = {t0.x, t0.y, t0.z, t0.w, t1.x, t1.y, t1.z, t1.w, t2.x};
+        const float bv = t2.y;
+        const unsigned m = __float_as_uint(t2.z);
+        const int oy0 = b * p.R, nro = min(p.R, Ho - oy0);
         const int h = lane / p.NCG, g = lane - h * p.NCG;
         const int r0 = h * p.RPL, r1 = min(r0 + p.RPL, nro);
         if (h >= p.NHL || r0 >= r1) return;
         const int c0 = g * kDwsCW;
-        constexpr int NI = (kDwsCW - 1) * S + 3;
-        float va[NI], vb[NI], vc[NI];   // staged rows r S, r S + 1, r S + 2 (input rows (oy0 + r) S - 1 ..)
-        dws_row<S, T>(st + (size_t)(r0 * S) * p.W, c0, p.W, va);
-        if constexpr (S == 1) dws_row<S, T>(st + (size_t)(r0 + 1) * p.W, c0, p.W, vb);
-        T* yq = y + ((size_t)q * p.Ho + oy0) * p.Wo + c0;
-        for (int r = r0; r < r1; ++r) {
-            if constexpr (S == 2) dws_row<S, T>(st + (size_t)(2 * r + 1) * p.W, c0, p.W, vb);
-            dws_row<S, T>(st + (size_t)(r * S + 2) * p.W, c0, p.W, vc);
-            float acc[kDwsCW];
+        const bool has_l = c0 > 0, has_r = c0 + kDwsCW * S < W;
+        const int off = r0 * S * W + c0 * S;
+        T* yr = y + ((size_t)q * Ho + oy0 + r0) * Wo + c0;
+        const int n = r1 - r0;
+        switch (m) {
+            case kDefaultMasks[0]: dws_rows<S, T, kDefaultMasks[0]>(st, off, W, yr, Wo, n, has_l, has_r, relu, w, bv); break;
+            case kDefaultMasks[1]: dws_rows<S, T, kDefaultMasks[1]>(st, off, W, yr, Wo, n, has_l, has_r, relu, w, bv); break;
+            case kDefaultMasks[2]: dws_rows<S, T, kDefaultMasks[2]>(st, off, W, yr, Wo, n, has_l, has_r, relu, w, bv); break;
+            case kDefaultMasks[3]: dws_rows<S, T, kDefaultMasks[3]>(st, off, W, yr, Wo, n, has_l, has_r, relu, w, bv); break;
+            case kDefaultMasks[4]: dws_rows<S, T, kDefaultMasks[4]>(st, off, W, yr, Wo, n, has_l, has_r, relu, w, bv); break;
+            case kDefaultMasks[5]: dws_rows<S, T, kDefaultMasks[5]>(st, off, W, yr, Wo, n, has_l, has_r, relu, w, bv); break;
+            case kDefaultMasks[6]: dws_rows<S, T, kDefaultMasks[6]>(st, off, W, yr, Wo, n, has_l, has_r, relu, w, bv); break;
+            case kDefaultMasks[7]: dws_rows<S, T, kDefaultMasks[7]>(st, off, W, yr, Wo, n, has_l, has_r, relu, w, bv); break;
+            default: dws_rows<S, T, 0x1FFu>(st, off, W, yr, Wo, n, has_l, has_r, relu, w, bv); break;
+        }
+    };
+
+    // planes mode: the warp's passes over the chunk's planes; lane l owns columns of plane
+    // l / LPP of the pass.  Every lane runs the same code with no branch of its own: an idle lane
+    // reads plane 0 of the stage and writes its results to a junk word of the warp's output buffer,
+    // as does a lane's second output beyond an odd-width row; columns outside the image are read
+    // inside the stage and zeroed by select.  Stride 1 (MODE 2, rows of even width; MODE 3, odd):
+    // output columns 2j, 2j + 1 as packed FMAs, the neighbouring input columns from the adjacent
+    // lanes; stride 2 (MODE 1): output column j from input columns 2j - 1 .. 2j + 1, scalar FMAs.
+    // All nine taps are applied (the lanes of a pass meet several channels), zeros at the pruned ones.
+    auto planes_chunk = [&](long long ch, const T* st) {
+        const long long q0 = ch * p.P;
+        const int np = (int)min((long long)p.P, p.n_planes - q0);
+        const int pl_l = lane / p.LPP, j = lane - pl_l * p.LPP;
+        const int npw = p.NPW;
+        const int c_first = (int)(q0 % C);
+        constexpr int CPL = MODE == 1 ? 1 : 2;
+        const bool has_l = j > 0;
+        const bool has_b = S == 1 && 2 * j + 1 < W;    // stride 1: the lane's second column exists
+        const bool has_r = S == 1 && 2 * j + 2 < W;
+        const int boff = has_b ? 1 : 0;
+        T* junk = ob + (size_t)p.P * Ho * Wo;          // past the chunk's outputs (the buffer has room)
+        for (int k = 0; k < np; k += npw) {
+            const int pl = k + pl_l;
+            const bool act = pl_l < npw && pl < np;
+            const int plx = act ? pl : 0;
+            int c = c_first + plx;
+            while (c >= C) c -= C;
+            const float4* tw = reinterpret_cast<const float4*>(tab + (size_t)c * kDwsTab);
+            const float4 t0 = tw[0], t1 = tw[1], t2 = tw[2];
+            const float w[9] = {t0.x, t0.y, t0.z, t0.w, t1.x, t1.y, t1.z, t1.w, t2.x};
+            const float bv = t2.y;
+            int xo = plx * H * W + j * 2;                          // input column 2j of row 0
+            T* o0 = act ? ob + (size_t)pl * Ho * Wo + j * CPL : junk;
+            T* o1 = act && has_b ? o0 + 1 : junk;
+            const int ostep = act ? Wo : 0, ostep1 = act && has_b ? Wo : 0;
+            if constexpr (S == 1) {
+                struct Row { float2 q[3]; };   // (left, a), (a, b), (b, right)
+                auto fetch = [&](Row& v) {
+                    float a, b;
+                    if constexpr (MODE == 2) {
+                        const float2 f = ld_pair<T>(st + xo);
+                        a = f.x;
+                        b = f.y;
+                    } else {
+                        a = to_f32<T>(st[xo]);
+                        const float bb = to_f32<T>(st[xo + boff]);
+                        b = has_b ? bb : 0.0f;
+                    }
+                    xo += W;
+                    const float l = __shfl_up_sync(0xffffffffu, b, 1);
+                    const float r = __shfl_down_sync(0xffffffffu, a, 1);
+                    v.q[0] = make_float2(has_l ? l : 0.0f, a);
+                    v.q[1] = make_float2(a, b);
+                    v.q[2] = make_float2(b, has_r ? r : 0.0f);
+                };
+                float2 w2[9];
 #pragma unroll
-            for (int j = 0; j < kDwsCW; ++j) acc[j] = bv;
+                for (int t = 0; t < 9; ++t) w2[t] = make_float2(w[t], w[t]);
+                auto out = [&](const Row& u, const Row& v, const Row& x3) {
+                    float2 o = make_float2(bv, bv);
 #pragma unroll
-            for (int dx = 0; dx < 3; ++dx) {
-                if ((m >> dx) & 1u) {
-#pragma unroll
-                    for (int j = 0; j < kDwsCW; ++j) acc[j] = fmaf(w[dx], va[j * S + dx], acc[j]);
-                }
-                if ((m >> (3 + dx)) & 1u) {
-#pragma unroll
-                    for (int j = 0; j < kDwsCW; ++j) acc[j] = fmaf(w[3 + dx], vb[j * S + dx], acc[j]);
-                }
-                if ((m >> (6 + dx)) & 1u) {
-#pragma unroll
-                    for (int j = 0; j < kDwsCW; ++j) acc[j] = fmaf(w[6 + dx], vc[j * S + dx], acc[j]);
-                }
-            }
-#pragma unroll
-            for (int j = 0; j < kDwsCW; ++j) acc[j] = p.relu ? fmaxf(acc[j], 0.0f) : acc[j];
-            T* out = yq + (size_t)r * p.Wo;
-            if (p.vec_out) {
-                if constexpr (sizeof(T) == 4) {
-                    *reinterpret_cast<float4*>(out) = make_float4(acc[0], acc[1], acc[2], acc[3]);
-                } else {
-                    __half2 h0 = __floats2half2_rn(acc[0], acc[1]), h1 = __floats2half2_rn(acc[2], acc[3]);
-                    uint2 u;
-                    u.x = *reinterpret_cast<unsigned*>(&h0);
-                    u.y = *reinterpret_cast<unsigned*>(&h1);
-                    *reinterpret_cast<uint2*>(out) = u;
+                    for (int dx = 0; dx < 3; ++dx) {
+                        o = __ffma2_rn(w2[dx], u.q[dx], o);
+                        o = __ffma2_rn(w2[3 + dx], v.q[dx], o);
+                        o = __ffma2_rn(w2[6 + dx], x3.q[dx], o);
+                    }
+                    if (relu) {
+                        o.x = fmaxf(o.x, 0.0f);
+                        o.y = fmaxf(o.y, 0.0f);
+                    }
+                    if constexpr (MODE == 2) {
+                        st_pair<T>(o0, o.x, o.y);
+                    } else {
+                        *o0 = from_f32<T>(o.x);
+                        *o1 = from_f32<T>(o.y);
+                        o1 += ostep1;
+                    }
+                    o0 += ostep;
+                };
+                Row A, B, Cr;
+                A.q[0] = A.q[1] = A.q[2] = make_float2(0.0f, 0.0f);   // input row -1
+                fetch(B);
+                for (int oy = 0; oy < Ho; oy += 3) {
+                    if (oy + 1 < H) fetch(Cr); else Cr.q[0] = Cr.q[1] = Cr.q[2] = make_float2(0.0f, 0.0f);
+                    out(A, B, Cr);
+                    if (oy + 1 >= Ho) break;
+                    if (oy + 2 < H) fetch(A); else A.q[0] = A.q[1] = A.q[2] = make_float2(0.0f, 0.0f);
+                    out(B, Cr, A);
+                    if (oy + 2 >= Ho) break;
+                    if (oy + 3 < H) fetch(B); else B.q[0] = B.q[1] = B.q[2] = make_float2(0.0f, 0.0f);
+                    out(Cr, A, B);
                 }
             } else {
+                struct Row { float e[3]; };   // input columns 2j - 1, 2j, 2j + 1
+                auto fetch = [&](Row& v) {
+                    const float2 f = ld_pair<T>(st + xo);
+                    xo += W;
+                    const float l = __shfl_up_sync(0xffffffffu, f.y, 1);
+                    v.e[0] = has_l ? l : 0.0f;
+                    v.e[1] = f.x;
+                    v.e[2] = f.y;
+                };
+                auto out = [&](const Row& u, const Row& v, const Row& x3) {
+                    float o = bv;
 #pragma unroll
-                for (int j = 0; j < kDwsCW; ++j) out[j] = from_f32<T>(acc[j]);
-            }
-#pragma unroll
-            for (int i = 0; i < NI; ++i) {
-                if constexpr (S == 1) {
-                    va[i] = vb[i];
-                    vb[i] = vc[i];
-                } else {
-                    va[i] = vc[i];
+                    for (int dx = 0; dx < 3; ++dx) {
+                        o = fmaf(w[dx], u.e[dx], o);
+                        o = fmaf(w[3 + dx], v.e[dx], o);
+                        o = fmaf(w[6 + dx], x3.e[dx], o);
+                    }
+                    if (relu) o = fmaxf(o, 0.0f);
+                    *o0 = from_f32<T>(o);
+                    o0 += ostep;
+                };
+                Row A, B, Cr;
+                A.e[0] = A.e[1] = A.e[2] = 0.0f;   // input row -1
+                for (int oy = 0; oy < Ho; oy += 2) {
+                    fetch(B);
+                    if (2 * oy + 1 < H) fetch(Cr); else Cr.e[0] = Cr.e[1] = Cr.e[2] = 0.0f;
+                    out(A, B, Cr);
+                    if (oy + 1 >= Ho) break;
+                    fetch(B);
+                    if (2 * oy + 3 < H) fetch(A); else A.e[0] = A.e[1] = A.e[2] = 0.0f;
+                    out(Cr, B, A);
                 }
             }
         }
     };
 
-    // planes mode: the warp's passes over the chunk's planes; lane l owns columns of plane
-    // l / LPP of the pass; every lane runs the same loop (shuffles), idle lanes on zeros
-    auto planes_chunk = [&](long long ch, const T* st) {
+    // tiles mode: lane items (plane, band of BR output rows, piece of PW output columns), 32 a pass;
+    // a lane past the chunk's items repeats item 0 (the same values to the same place)
+    auto tiles_chunk = [&](long long ch, const T* st) {
+        constexpr int PW = MODE == 5 ? 14 : 7, BR = 7;
         const long long q0 = ch * p.P;
         const int np = (int)min((long long)p.P, p.n_planes - q0);
-        const int pl_l = lane / p.LPP, gc = lane - pl_l * p.LPP;
-        const int c_first = (int)(q0 % p.C);
-        constexpr int CPL = MODE == 2 ? 2 : 1;
-        const bool has_l = gc > 0;
-        const bool has_r = (S == 1) && (gc + 1) * CPL < p.W;
-        for (int k = 0; k < np; k += p.NPW) {
-            const int pl = k + pl_l;
-            const bool act = pl_l < p.NPW && pl < np;
-            int c = act ? c_first + pl : 0;
-            while (c >= p.C) c -= p.C;
-            const float* tw = tab + (size_t)c * kDwsTab;
-            float w[9];
-#pragma unroll
-            for (int t = 0; t < 9; ++t) w[t] = tw[t];
-            const float bv = tw[9];
-            const T* xp = st + (size_t)(act ? pl : 0) * p.H * p.W + gc * CPL * S;
-            T* op = ob + (size_t)(act ? pl : 0) * p.Ho * p.Wo + gc * CPL;
-            // one input row: (left, a, b, right) = input columns c S - 1 .. of this lane's outputs,
-            // zeros outside the image (and on idle lanes)
-            auto fetch = [&](int iy, float (&v)[4]) {
-                const bool in = act && iy >= 0 && iy < p.H;
-                float a = 0.0f, b = 0.0f;
-                if constexpr (CPL == 2 || S == 2) {
-                    if (in) {
-                        const float2 f = ld_pair<T>(xp + (size_t)iy * p.W);
-                        a = f.x;
-                        b = f.y;
-                    }
-                } else {
-                    if (in) a = to_f32<T>(xp[(size_t)iy * p.W]);
-                }
-                const float hi = (CPL == 2 || S == 2) ? b : a;
-                const float l = __shfl_up_sync(0xffffffffu, hi, 1);
-                const float r = __shfl_down_sync(0xffffffffu, a, 1);
-                v[0] = has_l ? l : 0.0f;
-                v[1] = a;
-                v[2] = b;
-                v[3] = has_r ? r : 0.0f;
-            };
-            float v0[4], v1[4], v2[4];
-            v0[0] = v0[1] = v0[2] = v0[3] = 0.0f;   // input row -1
-            if constexpr (S == 1) fetch(0, v1);
-            for (int oy = 0; oy < p.Ho; ++oy) {
-                if constexpr (S == 1) {
-                    fetch(oy + 1, v2);
-                } else {
-                    fetch(2 * oy, v1);
-                    fetch(2 * oy + 1, v2);
-                }
-                if constexpr (CPL == 2) {   // outputs (a, b): taps on (left, a), (a, b), (b, right)
-                    auto row2 = [&](const float (&v)[4], int t0, float2 o) {
-                        o = __ffma2_rn(make_float2(w[t0], w[t0]), make_float2(v[0], v[1]), o);
-                        o = __ffma2_rn(make_float2(w[t0 + 1], w[t0 + 1]), make_float2(v[1], v[2]), o);
-                        return __ffma2_rn(make_float2(w[t0 + 2], w[t0 + 2]), make_float2(v[2], v[3]), o);
-                    };
-                    float2 o = make_float2(bv, bv);
-                    o = row2(v0, 0, o);
-                    o = row2(v1, 3, o);
-                    o = row2(v2, 6, o);
-                    if (p.relu) {
-                        o.x = fmaxf(o.x, 0.0f);
-                        o.y = fmaxf(o.y, 0.0f);
-                    }
-                    if (act) st_pair<T>(op + (size_t)oy * p.Wo, o.x, o.y);
-                } else {
-                    // stride 1: columns (left, a, right); stride 2: (left, a, b)
-                    const int i2 = S == 1 ? 3 : 2;
-                    float o = bv;
-                    o = fmaf(w[0], v0[0], o);
-                    o = fmaf(w[1], v0[1], o);
-                    o = fmaf(w[2], v0[i2], o);
-                    o = fmaf(w[3], v1[0], o);
-                    o = fmaf(w[4], v1[1], o);
-                    o = fmaf(w[5], v1[i2], o);
-                    o = fmaf(w[6], v2[0], o);
-                    o = fmaf(w[7], v2[1], o);
-                    o = fmaf(w[8], v2[i2], o);
-                    if (p.relu) o = fmaxf(o, 0.0f);
-                    if (act) op[(size_t)oy * p.Wo] = from_f32<T>(o);
-                }
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    if constexpr (S == 1) {
-                        v0[i] = v1[i];
-                        v1[i] = v2[i];
-                    } else {
-                        v0[i] = v2[i];
-                    }
-                }
-            }
+        const int items = np * p.ipp;
+        const int c_first = (int)(q0 % C);
+        const T* zrow = reinterpret_cast<const T*>(area + p.zoff) + 2;
+        for (int i0 = 0; i0 < items; i0 += 32) {
+            const int it = i0 + lane < items ? i0 + lane : 0;
+            const int pl = it / p.ipp, rem = it - pl * p.ipp;
+            const int band = rem / p.npc, piece = rem - band * p.npc;
+            int c = c_first + pl;
+            while (c >= C) c -= C;
+            const float4* tw = reinterpret_cast<const float4*>(tab + (size_t)c * kDwsTab);
+            const float4 t0 = tw[0], t1 = tw[1], t2 = tw[2];
+            const float w[9] = {t0.x, t0.y, t0.z, t0.w, t1.x, t1.y, t1.z, t1.w, t2.x};
+            dws_tile<S, T, PW, BR, MODE != 4>(st + pl * H * W, ob + pl * Ho * Wo, zrow, W, H, Wo, band * BR,
+                                               piece * PW, relu, w, t2.y);
         }
     };
 
@@ -1719,7 +1953,7 @@ __global__ void __launch_bounds__(kDwsThreads, 1)
             ok = false;
             break;
         }
-        const long long ch = wid + (long long)j * nw;
+        const long long ch = (long long)wid + (long long)j * nw;
         T* st = reinterpret_cast<T*>(area + (size_t)s * p.in_b);
         if constexpr (MODE == 0) {
             rows_chunk(ch, st);
@@ -1733,7 +1967,8 @@ __global__ void __launch_bounds__(kDwsThreads, 1)
             }
             if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");   // ob free again
             __syncwarp();
-            planes_chunk(ch, st);
+            if constexpr (MODE >= 4) tiles_chunk(ch, st);
+            else planes_chunk(ch, st);
             const size_t out_e = (size_t)np * opb / sizeof(T), fo_e = (((size_t)np * opb) & ~(size_t)15) / sizeof(T);
             T* yc = y + (size_t)q0 * (opb / sizeof(T));
             for (size_t i = fo_e + lane; i < out_e; i += 32) yc[i] = ob[i];   // the end of y by plain stores
@@ -2681,11 +2916,23 @@ bool dws_plan(const pp_layer* L, int N, int H, int W, int Ho, int Wo, size_t es,
     p->off_tab = 8 * kDwsMaxStages * kDwsWarps;
     p->off_area = (unsigned)align_up(p->off_tab + (size_t)C * kDwsTab * 4, 128);
     if ((size_t)p->off_area + (size_t)kDwsWarps * 4096 > optin) return false;   // the table leaves too little room
-    const size_t per_warp = (optin - p->off_area) / kDwsWarps / 128 * 128;
-    const long long warps = (long long)sm_count() * kDwsWarps;
-    size_t out_b = 0;
+    const size_t avail = optin - p->off_area;
+    const long long sms = sm_count();
+    size_t out_b = 0, extra = 0;
+    auto al = [](size_t b) { return (long long)(16 / std::gcd(b, (size_t)16)); };   // planes per 16 bytes
+    const size_t pb = (size_t)H * W * es, opb = (size_t)Ho * Wo * es;
     const bool rows = ((size_t)W * es) % 16 == 0 && W <= 256 && Wo % kDwsCW == 0 && Wo / kDwsCW <= 32 &&
                       (S == 1 ? W == Wo : W == 2 * Wo);
+    // tiles mode: each lane a band of 7 output rows by 7 or 14 columns of a plane
+    int tile = 0;
+    long long tP = 0;
+    if (S == 1 && W == Wo && H == Ho && H % 7 == 0) tile = W == 7 ? 4 : (W == 14 || W == 28) ? 5 : 0;
+    if (S == 2 && W == 14 && H == 2 * Ho && Ho % 7 == 0) tile = 6;
+    if (tile) {   // planes per chunk: 16-byte aligned chunk starts in x and y, lane items a multiple of 32
+        const int ipp = (Wo / (tile == 5 ? 14 : 7)) * (Ho / 7);
+        tP = std::lcm(std::lcm(al(pb), al(opb)), (long long)(32 / std::gcd(ipp, 32)));
+        if ((size_t)tP * pb > 16384) tile = 0;   // stages too large: planes mode
+    }
     if (rows) {
         p->NCG = Wo / kDwsCW;
         p->NHL = 32 / p->NCG;
@@ -2699,31 +2946,47 @@ bool dws_plan(const pp_layer* L, int N, int H, int W, int Ho, int Wo, size_t es,
         p->in_b = (unsigned)align_up((size_t)W * p->RIN * es, 128);
         p->n_chunks = n_planes * p->n_bands;
         *mode = 0;
-    } else {
-        if (S == 1 ? W != Wo : W != 2 * Wo) return false;
-        const int cpl = (S == 1 && W % 2 == 0) ? 2 : 1;
-        p->LPP = (Wo + cpl - 1) / cpl;
-        if (p->LPP > 32) return false;
-        p->NPW = 32 / p->LPP;
-        const size_t pb = (size_t)H * W * es, opb = (size_t)Ho * Wo * es;
-        // chunk starts 16-byte aligned in x and y; whole passes of the warp where that allows
-        auto al = [](size_t b) { return (long long)(16 / std::gcd(b, (size_t)16)); };
-        const long long A = std::lcm(std::lcm(al(pb), al(opb)), (long long)p->NPW);
-        long long P = std::max<long long>(A, (long long)(kDwsPlanesStage / pb) / A * A);
-        while (P > A && (n_planes + P - 1) / P < kDwsChunksPerWarp * warps) P -= A;
-        if ((size_t)P * pb > ((size_t)1 << 30)) return false;
+    } else if (tile) {
+        const int pw = tile == 5 ? 14 : 7;
+        p->npc = Wo / pw;
+        p->ipp = p->npc * (Ho / 7);
+        const long long P = tP;
         p->P = (int)P;
         p->in_b = (unsigned)align_up((size_t)P * pb, 128);
         out_b = align_up((size_t)P * opb, 128);
+        extra = 128;                     // the zero row
         p->n_chunks = (n_planes + P - 1) / P;
-        *mode = cpl;
+        *mode = tile;
+    } else {
+        if (S == 1 ? W != Wo : W != 2 * Wo) return false;
+        const int cpl = S == 1 ? 2 : 1;
+        p->LPP = (Wo + cpl - 1) / cpl;
+        if (p->LPP > 32) return false;
+        p->NPW = 32 / p->LPP;
+        // chunk starts 16-byte aligned in x and y; whole passes of the warp where that allows
+        const long long A = std::lcm(std::lcm(al(pb), al(opb)), (long long)p->NPW);
+        long long P = std::max<long long>(A, (long long)(kDwsPlanesStage / pb) / A * A);
+        while (P > A && (n_planes + P - 1) / P < kDwsChunksPerWarp * sms * kDwsWarps) P -= A;
+        if ((size_t)P * pb > ((size_t)1 << 30)) return false;
+        p->P = (int)P;
+        p->in_b = (unsigned)align_up((size_t)P * pb, 128);
+        out_b = align_up((size_t)P * opb + 16, 128);   // + a junk word for idle lanes' results
+        p->n_chunks = (n_planes + P - 1) / P;
+        *mode = S == 2 ? 1 : (W % 2 == 0 ? 2 : 3);
     }
-    if (out_b + 2 * (size_t)p->in_b > per_warp) return false;
-    p->nst = (int)std::min<size_t>(kDwsMaxStages, (per_warp - out_b) / p->in_b);
-    p->area_b = (unsigned)((size_t)p->nst * p->in_b + out_b);
+    if (p->n_chunks > INT_MAX) return false;
+    // warps per CTA: as many as hold two stages each (at most 16); then stages per warp
+    const size_t two = 2 * (size_t)p->in_b + out_b + extra;
+    const int nwarps = (int)std::min<size_t>(kDwsWarps, avail / two);
+    if (nwarps < 4) return false;
+    const size_t per_warp = avail / nwarps / 128 * 128;
+    p->nwarps = nwarps;
+    p->nst = (int)std::min<size_t>(kDwsMaxStages, (per_warp - out_b - extra) / p->in_b);
+    p->zoff = (unsigned)((size_t)p->nst * p->in_b + out_b);
+    p->area_b = (unsigned)align_up((size_t)p->nst * p->in_b + out_b + extra, 128);
     p->n_planes = n_planes;
-    *smem = p->off_area + (size_t)kDwsWarps * p->area_b;
-    return true;
+    *smem = p->off_area + (size_t)nwarps * p->area_b;
+    return *smem <= optin;
 }
 
 template <int S, typename T, int MODE>
@@ -2737,8 +3000,8 @@ int launch_dws(const DwsParams& p, const CUtensorMap& tmap, size_t smem, cudaStr
             return PP_ERR_CUDA;
         done[dev].store(1, std::memory_order_release);
     }
-    const long long grid = std::min<long long>(sm_count(), (p.n_chunks + kDwsWarps - 1) / kDwsWarps);
-    return launch(pconv_dw_stream<S, T, MODE>, (unsigned)std::max<long long>(grid, 1), kDwsThreads, smem, st, p, tmap) ==
+    const long long grid = std::min<long long>(sm_count(), (p.n_chunks + p.nwarps - 1) / p.nwarps);
+    return launch(pconv_dw_stream<S, T, MODE>, (unsigned)std::max<long long>(grid, 1), 32u * p.nwarps, smem, st, p, tmap) ==
                    cudaSuccess ? PP_OK : PP_ERR_CUDA;
 }
 
@@ -2789,10 +3052,13 @@ int try_dws(const pp_layer* L, const void* x, void* y, const float* bias, int re
     const int S = L->stride;
     if (S == 1) {
         if (mode == 0) return launch_dws<1, T, 0>(p, tmap, smem, st);
-        if (mode == 1) return launch_dws<1, T, 1>(p, tmap, smem, st);
-        return launch_dws<1, T, 2>(p, tmap, smem, st);
+        if (mode == 2) return launch_dws<1, T, 2>(p, tmap, smem, st);
+        if (mode == 3) return launch_dws<1, T, 3>(p, tmap, smem, st);
+        if (mode == 4) return launch_dws<1, T, 4>(p, tmap, smem, st);
+        return launch_dws<1, T, 5>(p, tmap, smem, st);
     }
     if (mode == 0) return launch_dws<2, T, 0>(p, tmap, smem, st);
+    if (mode == 6) return launch_dws<2, T, 6>(p, tmap, smem, st);
     return launch_dws<2, T, 1>(p, tmap, smem, st);
 }
 
@@ -3030,7 +3296,8 @@ int conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t*
             v[4] = mode == 0 ? q.R : q.P;
             v[5] = q.nst;
             v[10] = (int64_t)smem;
-            v[12] = std::min<long long>(sm_count(), (q.n_chunks + kDwsWarps - 1) / kDwsWarps);
+            v[12] = std::min<long long>(sm_count(), (q.n_chunks + q.nwarps - 1) / q.nwarps);
+            v[6] = q.nwarps;
         }
     } else if (!h->fast) {
         v[0] = 3;   // generic kernel: no plan, no workspace

@@ -258,9 +258,14 @@ def test_depthwise_unaligned_input(dtype):
     ((2, 8, 40, 48), 2, torch.float32, 1),     # rows mode, stride 2, five lane row-sets
     ((3, 21, 13, 12), 1, torch.float16, 3),    # planes, two columns a lane; x ends inside a 16-byte block
     ((3, 21, 13, 12), 2, torch.float32, 2),    # planes, stride 2; y ends inside a 16-byte block
-    ((2, 24, 9, 9), 1, torch.float16, 2),      # planes, odd width
-    ((1, 13, 7, 7), 1, torch.float16, 2),      # 13 planes: a short last chunk
-    ((5, 40, 14, 14), 2, torch.float16, 2),    # planes, stride 2 to 7x7
+    ((2, 24, 9, 9), 1, torch.float16, 4),      # planes, odd width
+    ((1, 13, 7, 7), 1, torch.float16, 5),      # tiles of 7x7: 13 planes, a short last chunk
+    ((3, 40, 7, 7), 1, torch.float32, 5),      # tiles of 7x7, fp32
+    ((5, 40, 14, 14), 2, torch.float16, 7),    # tiles at stride 2, 14x14 to 7x7
+    ((3, 21, 14, 14), 1, torch.float16, 6),    # tiles of 7 rows x 14 columns, two bands a plane
+    ((2, 11, 28, 28), 1, torch.float16, 6),    # tiles: two column pieces x four bands a plane
+    ((2, 11, 28, 28), 1, torch.float32, 1),    # fp32: 112-byte rows, rows mode
+    ((2, 24, 28, 28), 2, torch.float16, 2),    # 28 -> 14 at stride 2: column lanes
 ])
 def test_streamed_depthwise(shape, stride, dtype, kernel):
     """The streamed depthwise kernel in each of its modes (asserted through the plan), with the
@@ -275,6 +280,23 @@ def test_streamed_depthwise(shape, stride, dtype, kernel):
     assert lay.plan(shape, 0, dtype=dtype)["dw_kernel"] == kernel
     check(Wd, x, b, 1.0, stride, depthwise=True, dtype=dtype, guard=64)
     check(Wd, x, b, 0.6, stride, relu=False, depthwise=True, dtype=dtype, guard=64)
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.float16])
+@pytest.mark.parametrize("stride", [1, 2])
+def test_streamed_depthwise_rows_other_library(dtype, stride):
+    """Rows mode with a library other than the compiled one: its masks match none of the row
+    loops compiled per pattern, so every channel takes the nine-tap loop."""
+    rng = np.random.default_rng(77 + stride)
+    C, H, W = 12, 18, 64
+    masks = [OP.mask_of(t) for t in ([0, 4, 5, 8], [1, 4, 6, 7], [2, 3, 4, 8])]
+    Wd = (rng.standard_normal((C, 1, 3, 3)) * np.sqrt(2 / 9)).astype(np.float32)
+    x = rnd((2, C, H, W), 60 + stride, dtype=_np_dt(dtype))
+    b = (rng.standard_normal(C) * 0.1).astype(np.float32)
+    lay = api.pp_pack(Wd, masks, 1.0, C, stride)
+    assert lay.plan((2, C, H, W), 0, dtype=dtype)["dw_kernel"] == 1
+    check(Wd, x, b, 1.0, stride, depthwise=True, dtype=dtype, masks=masks)
+    check(Wd, x, b, 0.6, stride, depthwise=True, dtype=dtype, masks=masks)
 
 
 @pytest.mark.parametrize("m", [6, 8])

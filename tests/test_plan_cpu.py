@@ -313,12 +313,14 @@ def _dw_layer(C, stride=1, seed=5):
 
 
 @pytest.mark.parametrize("idx,kernel", [(0, 1), (1, 1), (2, 1), (3, 1),      # 112 / 56-wide rows
-                                        (4, 3), (6, 2), (7, 3), (13, 2),     # 28 / 14-wide planes
-                                        (14, 2)])                            # 7-wide planes
+                                        (4, 6), (7, 6), (11, 6),             # 28 / 14-wide tiles
+                                        (13, 7), (14, 5),                    # 14 -> 7, 7-wide tiles
+                                        (6, 2)])                             # 28 -> 14: column lanes
 def test_streamed_depthwise_mode_per_mobilenet_layer(idx, kernel):
     """MobileNet-V2's fp16 layers at batch 128: 112- and 56-wide maps stream bands of whole rows
     through tensor copies (rows of 224 or 112 bytes); 28-, 14- and 7-wide maps stream runs of whole
-    planes (two output columns per lane where the width is even at stride 1)."""
+    planes, each lane a band of 7 output rows by 7 or 14 columns (the 28 -> 14 stride-2 layer:
+    one output column per lane)."""
     L = WL.mobilenet_v2_dw()[idx]
     lay = _dw_layer(L.cout, L.stride)
     pl = lay.plan((128, L.cin, L.h, L.w), 0, dtype=torch.float16)
@@ -330,20 +332,25 @@ def test_streamed_depthwise_mode_per_mobilenet_layer(idx, kernel):
         R = pl["rows_or_planes"]
         assert 1 <= R <= ho and ((R - 1) * L.stride + 3) * L.w * es <= 4096
         assert pl["chunks"] == n_planes * -(-ho // R)
-    else:             # planes mode: chunk starts 16-byte aligned in x and y
+    else:             # planes and tiles modes: chunk starts 16-byte aligned in x and y
         P = pl["rows_or_planes"]
         assert (P * L.h * L.w * es) % 16 == 0 and (P * ho * wo * es) % 16 == 0
         assert pl["chunks"] == -(-n_planes // P)
-        lpp = -(-wo // (2 if kernel == 3 else 1))
-        assert lpp <= 32 and P % (32 // lpp) == 0      # whole passes of the warp
-    assert pl["ctas"] == min(152, -(-pl["chunks"] // 16))
+        if kernel >= 5:   # tiles: lane items (plane, 7 output rows, 7 or 14 columns), 32 a pass
+            items = P * (ho // 7) * (wo // (14 if kernel == 6 else 7))
+            assert items % 32 == 0
+        else:
+            lpp = -(-wo // (1 if kernel == 2 else 2))
+            assert lpp <= 32 and P % (32 // lpp) == 0      # whole passes of the warp
+    assert 4 <= pl["warps"] <= 16
+    assert pl["ctas"] == min(152, -(-pl["chunks"] // pl["warps"]))
 
 
 @pytest.mark.parametrize("shape,stride,dtype,kernel", [
     ((3, 21, 13, 12), 1, torch.float32, 1),     # 48-byte rows
     ((3, 21, 13, 12), 2, torch.float32, 2),     # 6 output columns: planes
     ((3, 21, 13, 12), 1, torch.float16, 3),     # 24-byte rows: planes, two columns a lane
-    ((2, 24, 9, 9), 1, torch.float32, 2),       # odd width
+    ((2, 24, 9, 9), 1, torch.float32, 4),       # odd width
     ((1, 4, 9, 2100), 1, torch.float16, 0),     # rows too wide for either mode
     ((2, 16, 20, 100), 1, torch.float16, 0),    # 200-byte rows, 100 columns: neither mode
 ])
