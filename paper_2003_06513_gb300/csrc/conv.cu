@@ -2927,7 +2927,7 @@ bool dws_plan(const pp_layer* L, int N, int H, int W, int Ho, int Wo, size_t es,
     int tile = 0;
     long long tP = 0;
     if (S == 1 && W == Wo && H == Ho && H % 7 == 0) tile = W == 7 ? 4 : (W == 14 || W == 28) ? 5 : 0;
-    if (S == 2 && W == 14 && H == 2 * Ho && Ho % 7 == 0) tile = 6;
+    if (S == 2 && (W == 14 || W == 28) && H == 2 * Ho && Ho % 7 == 0) tile = 6;
     if (tile) {   // planes per chunk: 16-byte aligned chunk starts in x and y, lane items a multiple of 32
         const int ipp = (Wo / (tile == 5 ? 14 : 7)) * (Ho / 7);
         tP = std::lcm(std::lcm(al(pb), al(opb)), (long long)(32 / std::gcd(ipp, 32)));

@@ -265,7 +265,8 @@ def test_depthwise_unaligned_input(dtype):
     ((3, 21, 14, 14), 1, torch.float16, 6),    # tiles of 7 rows x 14 columns, two bands a plane
     ((2, 11, 28, 28), 1, torch.float16, 6),    # tiles: two column pieces x four bands a plane
     ((2, 11, 28, 28), 1, torch.float32, 1),    # fp32: 112-byte rows, rows mode
-    ((2, 24, 28, 28), 2, torch.float16, 2),    # 28 -> 14 at stride 2: column lanes
+    ((2, 24, 28, 28), 2, torch.float16, 7),    # tiles at stride 2: two column pieces x two bands
+    ((3, 21, 13, 12), 2, torch.float16, 2),    # 6 output columns at stride 2: column lanes
 ])
 def test_streamed_depthwise(shape, stride, dtype, kernel):
     """The streamed depthwise kernel in each of its modes (asserted through the plan), with the

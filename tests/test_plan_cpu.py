@@ -314,13 +314,11 @@ def _dw_layer(C, stride=1, seed=5):
 
 @pytest.mark.parametrize("idx,kernel", [(0, 1), (1, 1), (2, 1), (3, 1),      # 112 / 56-wide rows
                                         (4, 6), (7, 6), (11, 6),             # 28 / 14-wide tiles
-                                        (13, 7), (14, 5),                    # 14 -> 7, 7-wide tiles
-                                        (6, 2)])                             # 28 -> 14: column lanes
+                                        (13, 7), (14, 5), (6, 7)])           # 14 -> 7, 28 -> 14, 7-wide
 def test_streamed_depthwise_mode_per_mobilenet_layer(idx, kernel):
     """MobileNet-V2's fp16 layers at batch 128: 112- and 56-wide maps stream bands of whole rows
     through tensor copies (rows of 224 or 112 bytes); 28-, 14- and 7-wide maps stream runs of whole
-    planes, each lane a band of 7 output rows by 7 or 14 columns (the 28 -> 14 stride-2 layer:
-    one output column per lane)."""
+    planes, each lane a band of 7 output rows by 7 or 14 columns."""
     L = WL.mobilenet_v2_dw()[idx]
     lay = _dw_layer(L.cout, L.stride)
     pl = lay.plan((128, L.cin, L.h, L.w), 0, dtype=torch.float16)
