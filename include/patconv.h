@@ -21,10 +21,11 @@
  *     a 9-bit mask with bit t set for each kept tap;
  *   - tensors are contiguous NCHW; weights are host fp32 [Cout][Cin/groups][3][3];
  *   - kernels are launched with programmatic dependent launch on a stream that is not being
- *     captured into a CUDA graph: a convolution may start its set-up while the kernel before it
- *     on the stream finishes, and reads or writes no activation before that kernel has completed,
- *     so stream order holds as for a plain launch.  The environment variable PATCONV_PDL=0
- *     (read once) makes every launch a plain one.
+ *     captured into a CUDA graph (the streamed depthwise kernel also under capture): a
+ *     convolution may start its set-up (reading the layer's bound device image) while the kernel
+ *     before it on the stream finishes, and reads or writes no activation and reads no bias
+ *     before that kernel has completed, so stream order holds as for a plain launch.  The
+ *     environment variable PATCONV_PDL=0 (read once) makes every launch a plain one.
  *
  * Thread safety: a handle is immutable after pp_pack/pp_bind_device, so pp_conv on one handle
  * may be called from several host threads and streams at once.

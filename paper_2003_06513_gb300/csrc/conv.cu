@@ -1685,6 +1685,55 @@ __global__ void __launch_bounds__(kDwsThreads, 1)
     if constexpr (MODE >= 4) {   // this warp's zero row (tiles mode: rows above and below the image)
         if (lane < 32) reinterpret_cast<uint32_t*>(area + p.zoff)[lane] = 0u;
     }
+    // taps and mask of every channel (slot s holds channel perm[s]; a pruned kernel has no entry:
+    // mask 0, all taps zero): up to four slots a thread, their independent loads issued together
+    // (two rounds of L2 latency).  The packed layer is immutable once bound, so this runs before
+    // the previous kernel of the stream has completed (programmatic launch)
+    for (int s0 = threadIdx.x; s0 < p.NS; s0 += 4 * nthr) {
+        uint32_t co[4], ko[4];
+        uint64_t d[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int s = s0 + u * nthr;
+            const bool in = s < p.NS;
+            co[u] = in ? p.perm[s] : kPadSlot;
+            d[u] = in ? p.desc[s >> 3] : 0ull;
+            ko[u] = in ? p.kofs[s >> 3] : 0u;
+        }
+        float4 v[4];
+        unsigned msk[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int f = (s0 + u * nthr) & 7;
+            const int cnt = (int)(d[u] & 15u);
+            int pat = -1, jj = 0;
+            for (int j2 = 0; j2 < cnt; ++j2) {
+                const int code = (int)((d[u] >> (4 + 6 * j2)) & 63u);
+                if ((code >> 3) == f) {
+                    pat = code & 7;
+                    jj = j2;
+                }
+            }
+            const bool live = co[u] != kPadSlot;
+            v[u] = live && pat >= 0 ? p.vals[ko[u] + jj] : make_float4(0.f, 0.f, 0.f, 0.f);
+            msk[u] = live && pat >= 0 ? p.masks[pat] : 0u;
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            if (co[u] == kPadSlot) continue;
+            float* w = tab + (size_t)co[u] * kDwsTab;
+            int k = 0;
+#pragma unroll
+            for (int t = 0; t < 9; ++t) {
+                const bool on = (msk[u] >> t) & 1u;
+                const float vk = k == 0 ? v[u].x : k == 1 ? v[u].y : k == 2 ? v[u].z : v[u].w;
+                w[t] = on ? vk : 0.0f;
+                k += on ? 1 : 0;
+            }
+            w[10] = __uint_as_float(msk[u]);
+            w[11] = 0.0f;
+        }
+    }
     pdl_wait();   // activations and the bias from here on
     const size_t pb = (size_t)p.H * p.W * sizeof(T), opb = (size_t)p.Ho * p.Wo * sizeof(T);
     auto issue = [&](int j) {   // lane 0: the copy of this warp's j-th chunk into stage j % nst
@@ -1707,57 +1756,7 @@ __global__ void __launch_bounds__(kDwsThreads, 1)
     if (lane == 0)
         for (int j = 0; j < first; ++j) issue(j);
     int issued = first;
-    // taps, bias and mask of every channel (slot s holds channel perm[s]; a pruned kernel has no
-    // entry: mask 0, all taps zero), decoded while the first copies are in flight: up to four
-    // slots a thread, their independent loads issued together (two rounds of L2 latency)
-    for (int s0 = threadIdx.x; s0 < p.NS; s0 += 4 * nthr) {
-        uint32_t co[4], ko[4];
-        uint64_t d[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const int s = s0 + u * nthr;
-            const bool in = s < p.NS;
-            co[u] = in ? p.perm[s] : kPadSlot;
-            d[u] = in ? p.desc[s >> 3] : 0ull;
-            ko[u] = in ? p.kofs[s >> 3] : 0u;
-        }
-        float4 v[4];
-        float bi[4];
-        unsigned msk[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const int f = (s0 + u * nthr) & 7;
-            const int cnt = (int)(d[u] & 15u);
-            int pat = -1, jj = 0;
-            for (int j2 = 0; j2 < cnt; ++j2) {
-                const int code = (int)((d[u] >> (4 + 6 * j2)) & 63u);
-                if ((code >> 3) == f) {
-                    pat = code & 7;
-                    jj = j2;
-                }
-            }
-            const bool live = co[u] != kPadSlot;
-            v[u] = live && pat >= 0 ? p.vals[ko[u] + jj] : make_float4(0.f, 0.f, 0.f, 0.f);
-            bi[u] = live && p.bias ? p.bias[co[u]] : 0.0f;
-            msk[u] = live && pat >= 0 ? p.masks[pat] : 0u;
-        }
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            if (co[u] == kPadSlot) continue;
-            float* w = tab + (size_t)co[u] * kDwsTab;
-            int k = 0;
-#pragma unroll
-            for (int t = 0; t < 9; ++t) {
-                const bool on = (msk[u] >> t) & 1u;
-                const float vk = k == 0 ? v[u].x : k == 1 ? v[u].y : k == 2 ? v[u].z : v[u].w;
-                w[t] = on ? vk : 0.0f;
-                k += on ? 1 : 0;
-            }
-            w[9] = bi[u];
-            w[10] = __uint_as_float(msk[u]);
-            w[11] = 0.0f;
-        }
-    }
+    for (int c = threadIdx.x; c < p.C; c += nthr) tab[(size_t)c * kDwsTab + 9] = p.bias ? p.bias[c] : 0.0f;
     __syncthreads();   // the table is complete
 
     // rows mode: rows h RPL .. of the chunk's band, output columns 4g .. 4g + 3.  The channel is
@@ -2114,8 +2113,10 @@ int sm_count() {
 // Kernel launch with programmatic stream serialisation (pdl_wait / pdl_trigger) on a stream that
 // is not being captured, unless the environment sets PATCONV_PDL=0; returns the launch's error,
 // which it also clears.  In a CUDA graph the kernel nodes already follow each other without host
-// work, and programmatic edges there measured slower (VGG-16 at batch 1: 0.477 against 0.464 ms
-// per image), so a captured launch is a plain one.
+// work, and programmatic edges there measured slower for the dense kernels (VGG-16 at batch 1:
+// 0.477 against 0.464 ms per image; equal at batch 32), so their captured launches are plain
+// ones; the streamed depthwise kernel keeps the edge (pdl_captured), whose set-up (the tap table)
+// then overlaps the previous kernel.
 bool pdl_enabled() {
     static const bool on = [] {
         const char* e = std::getenv("PATCONV_PDL");
@@ -2135,7 +2136,7 @@ bool balanced_enabled() {
 
 template <typename... KArgs, typename... Args>
 cudaError_t launch_ex(bool cooperative, void (*kern)(KArgs...), unsigned grid, unsigned block, size_t smem,
-                      cudaStream_t st, const Args&... args) {
+                      cudaStream_t st, bool pdl_captured, const Args&... args) {
     cudaLaunchAttribute attr[1];
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
@@ -2152,7 +2153,7 @@ cudaError_t launch_ex(bool cooperative, void (*kern)(KArgs...), unsigned grid, u
     } else {
         attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
         attr[0].val.programmaticStreamSerializationAllowed = 1;
-        cfg.numAttrs = pdl_enabled() && !captured ? 1 : 0;
+        cfg.numAttrs = pdl_enabled() && (!captured || pdl_captured) ? 1 : 0;
     }
     const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, args...);
     const cudaError_t l = cudaGetLastError();
@@ -2162,7 +2163,7 @@ cudaError_t launch_ex(bool cooperative, void (*kern)(KArgs...), unsigned grid, u
 template <typename... KArgs, typename... Args>
 cudaError_t launch(void (*kern)(KArgs...), unsigned grid, unsigned block, size_t smem, cudaStream_t st,
                    const Args&... args) {
-    return launch_ex(false, kern, grid, block, smem, st, args...);
+    return launch_ex(false, kern, grid, block, smem, st, false, args...);
 }
 
 using EncodeTiledFn = PFN_cuTensorMapEncodeTiled_v12000;
@@ -2764,7 +2765,7 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
                                                  align_up((size_t)P * kSlotFloats * sizeof(float), 256));
         if (cudaMemsetAsync(p.sk_flags, 0, (size_t)P * kCompute * sizeof(unsigned), st) != cudaSuccess)
             return PP_ERR_CUDA;
-        if (launch_ex(true, kern, (unsigned)P, kThreadsTM, smem, st, p, tmap) != cudaSuccess) return PP_ERR_CUDA;
+        if (launch_ex(true, kern, (unsigned)P, kThreadsTM, smem, st, false, p, tmap) != cudaSuccess) return PP_ERR_CUDA;
         return PP_OK;
     }
     // TMA path: one persistent CTA per SM walks its units as one chunk stream (the halo is zero
@@ -3001,8 +3002,10 @@ int launch_dws(const DwsParams& p, const CUtensorMap& tmap, size_t smem, cudaStr
         done[dev].store(1, std::memory_order_release);
     }
     const long long grid = std::min<long long>(sm_count(), (p.n_chunks + p.nwarps - 1) / p.nwarps);
-    return launch(pconv_dw_stream<S, T, MODE>, (unsigned)std::max<long long>(grid, 1), 32u * p.nwarps, smem, st, p, tmap) ==
-                   cudaSuccess ? PP_OK : PP_ERR_CUDA;
+    // programmatic launch also under stream capture: the tap table's decode then overlaps the
+    // previous kernel in a graph as on a stream (MobileNet-V2 b128: 0.390 -> 0.359 ms graphed)
+    return launch_ex(false, pconv_dw_stream<S, T, MODE>, (unsigned)std::max<long long>(grid, 1), 32u * p.nwarps, smem, st,
+                     true, p, tmap) == cudaSuccess ? PP_OK : PP_ERR_CUDA;
 }
 
 // The streamed depthwise kernel where it applies (PP_OK or an error), else 1.
