@@ -202,7 +202,9 @@ int pp_conv_workspace_size(pp_handle h, int N, int H, int W, size_t* bytes);
  * between two CTAs is finished by the CTA holding its first chunks, which adds the later ones'
  * raw sums from their workspace slots (workspace: 256 KiB per SM + flags, reported in [2]; the
  * launch is cooperative and resets the flags with a small memset first; the input must go
- * through TMA, else the launch takes whole units), else 0.  For path 2 (depthwise), assuming
+ * through TMA, else the launch takes whole units), else 0; [16] filter groups per warp (2 for
+ * stride-2 layers: 8 warps of 16 filter slots, each input window serving both groups' kept
+ * kernels; else 1).  For path 2 (depthwise), assuming
  * x and y 16-byte aligned (else the row-item kernels run): info[1] = 1 streamed kernel in rows
  * mode (bands of whole rows of one plane per tensor copy), 2 streamed kernel in planes mode at
  * stride 2 (one output column per lane), 3 planes mode at stride 1 with rows of even width (two
@@ -210,7 +212,7 @@ int pp_conv_workspace_size(pp_handle h, int N, int H, int W, size_t* bytes);
  * band of 7 output rows by 7 / 14 columns of one plane), 7 tiles mode at stride 2 (a lane a 7x7
  * output plane), 0 the row-item kernels; [3] chunks, [4] output rows per chunk (rows mode) or
  * planes per chunk, [5] shared-memory stages per warp, [6] warps per CTA, [10] shared-memory
- * bytes, [12] CTAs.  Writes min(n_info, 16) values.
+ * bytes, [12] CTAs.  Writes min(n_info, 17) values.
  * Host-only. */
 int pp_conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t* info, int n_info);
 

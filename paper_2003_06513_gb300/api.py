@@ -102,7 +102,7 @@ class Layer:
 
     PLAN_KEYS = ("path", "splits", "workspace_bytes", "units", "tile_by", "tile_bx", "tile_nb",
                  "channels_per_stage", "filter_groups", "spatial_warps", "smem_bytes",
-                 "chunks_per_unit", "ctas", "lane_sort", "shift", "streamk")
+                 "chunks_per_unit", "ctas", "lane_sort", "shift", "streamk", "groups_per_warp")
 
     def plan(self, x_shape, workspace_bytes: int = 0, pool2x2: bool = False,
              dtype=torch.float32) -> dict:

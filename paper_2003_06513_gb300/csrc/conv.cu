@@ -207,7 +207,7 @@ __device__ __forceinline__ void tmem_zero16(uint32_t ta) {
 // Fallback input staging when no TMA descriptor applies (row pitch not a multiple of 16 bytes,
 // the stage holds the input's own type): thread tid copies elements tid, tid + 512, ... of the
 // in-image part of the tile; everything else in the stage keeps the zero written at kernel start.
-template <typename TIn>
+template <typename TIn, int NT = kThreadsTM>
 __device__ __forceinline__ void stage_input_share(const TmParams& p, TIn* s_in, int c0, int ckv, int n0,
                                                   int iy0, int ix0, int tid) {
     const TIn* x = static_cast<const TIn*>(p.x);
@@ -229,8 +229,8 @@ __device__ __forceinline__ void stage_input_share(const TmParams& p, TIn* s_in, 
     int r = q % nr;
     q /= nr;
     int cl = q % ckv, img = q / ckv;
-    q = kThreadsTM / units;
-    const int su = kThreadsTM - q * units, sr = q % nr;
+    q = NT / units;
+    const int su = NT - q * units, sr = q % nr;
     q /= nr;
     const int scl = q % ckv, simg = q / ckv;
     const size_t HW = (size_t)p.H * p.W;
@@ -297,13 +297,13 @@ __device__ __forceinline__ Unit unit_of(const TmParams& p, int u) {
 
 // This thread's share of filling pipeline stage q % kStages with input channel chunk k of unit U
 // (non-blocking): warp 0 lane 0 issues the input tile's TMA, or every thread copies its share of
-// the tile; the warps of filter group wg copy that group's descriptors and its kept weights
-// vals[beg, end).  The stage's full barrier completes when all 512 threads have arrived and
-// every byte has landed.
-template <typename TIn>
+// the tile; the warps of filter group wg (DG groups per warp: wg DG .. wg DG + DG - 1) copy those
+// groups' descriptors and kept weights vals[beg[d], end[d]).  The stage's full barrier completes
+// when all threads of the CTA (kThreadsTM / DG) have arrived and every byte has landed.
+template <typename TIn, int DG = 1>
 __device__ __forceinline__ void fill_share(const TmParams& p, const CUtensorMap* tmap, unsigned char* smem,
-                                           uint32_t full0, int q, const Unit& U, int k, uint32_t beg,
-                                           uint32_t end, int warp, int lane) {
+                                           uint32_t full0, int q, const Unit& U, int k, const uint32_t (&beg)[DG],
+                                           const uint32_t (&end)[DG], int warp, int lane) {
     const int s = q % kStages;
     unsigned char* st = smem + p.stage_off + (size_t)s * p.stage_bytes;
     const uint32_t fb = full0 + 8 * s;
@@ -316,14 +316,19 @@ __device__ __forceinline__ void fill_share(const TmParams& p, const CUtensorMap*
         }
     }
     if (!p.use_tma)
-        stage_input_share<TIn>(p, reinterpret_cast<TIn*>(st), c0, ckv, U.n0, U.iy0, U.ix0, warp * 32 + lane);
-    const int wg = warp / p.WS, ws = warp - wg * p.WS, g = U.g0 + wg;
-    if (g < p.G) {
-        uint64_t* sd = reinterpret_cast<uint64_t*>(st + p.desc_off) + wg * p.CK;
-        for (int cl = ws * 32 + lane; cl < ckv; cl += p.WS * 32)
-            cp_async8(sd + cl, p.desc + (size_t)g * p.C + c0 + cl);
-        float4* sv = reinterpret_cast<float4*>(st + p.vals_off) + wg * p.maxk;
-        for (uint32_t i = beg + ws * 32 + lane; i < end; i += p.WS * 32) cp_async16(sv + (i - beg), p.vals + i);
+        stage_input_share<TIn, kThreadsTM / DG>(p, reinterpret_cast<TIn*>(st), c0, ckv, U.n0, U.iy0, U.ix0,
+                                                warp * 32 + lane);
+    const int wg = warp / p.WS, ws = warp - wg * p.WS;
+#pragma unroll
+    for (int d = 0; d < DG; ++d) {
+        const int gl = wg * DG + d, g = U.g0 + gl;   // the group's index within the unit, and in the layer
+        if (g < p.G) {
+            uint64_t* sd = reinterpret_cast<uint64_t*>(st + p.desc_off) + gl * p.CK;
+            for (int cl = ws * 32 + lane; cl < ckv; cl += p.WS * 32)
+                cp_async8(sd + cl, p.desc + (size_t)g * p.C + c0 + cl);
+            float4* sv = reinterpret_cast<float4*>(st + p.vals_off) + gl * p.maxk;
+            for (uint32_t i = beg[d] + ws * 32 + lane; i < end[d]; i += p.WS * 32) cp_async16(sv + (i - beg[d]), p.vals + i);
+        }
     }
     __threadfence_block();   // orders the fp16 path's plain shared stores before the arrival
     cp_async_arrive(fb);
@@ -343,10 +348,11 @@ __device__ __forceinline__ void tmem_st16(uint32_t ta, const float (&a)[16]) {
 // Balanced schedule, a part segment's end: the warp's raw accumulators (8 slots x 16 per lane) go
 // to this CTA's workspace slot ([warp][slot][16][lane]: coalesced), tensor memory is zeroed
 // behind, then the warp's flag is released once every lane's stores are visible.
+template <int DG>
 __device__ __noinline__ void sk_store_part(const TmParams& p, uint32_t tw, int warp, int lane) {
-    float* sl = p.sk_slots + (size_t)blockIdx.x * kSlotFloats + (size_t)warp * kF * 16 * 32 + lane;
+    float* sl = p.sk_slots + (size_t)blockIdx.x * kSlotFloats + (size_t)warp * kF * DG * 16 * 32 + lane;
 #pragma unroll 1
-    for (int f = 0; f < kF; ++f) {
+    for (int f = 0; f < kF * DG; ++f) {
         float a[16];
         __syncwarp();
         tmem_ld16(tw + 16u * f, a);
@@ -365,6 +371,7 @@ __device__ __noinline__ void sk_store_part(const TmParams& p, uint32_t tw, int w
 // Balanced schedule, a head segment's end: wait (bounded) for the flags of the unit's parts, held
 // by CTAs [pb0, pb1), then add their sums to the warp's accumulators in chunk order (a fixed
 // summation order).  A flag that never comes records a status bit and the parts are left out.
+template <int DG>
 __device__ __noinline__ void sk_add_parts(const TmParams& p, uint32_t tw, int warp, int lane, int pb0, int pb1) {
     bool ok = true;
     for (int b = pb0; b < pb1; ++b) {
@@ -386,12 +393,12 @@ __device__ __noinline__ void sk_add_parts(const TmParams& p, uint32_t tw, int wa
     __syncwarp();   // the other lanes read the slots after lane 0's acquire
     if (!ok) return;
 #pragma unroll 1
-    for (int f = 0; f < kF; ++f) {
+    for (int f = 0; f < kF * DG; ++f) {
         float a[16];
         __syncwarp();
         tmem_ld16(tw + 16u * f, a);
         for (int b = pb0; b < pb1; ++b) {
-            const float* sl = p.sk_slots + (size_t)b * kSlotFloats + (size_t)warp * kF * 16 * 32 + lane + f * 16 * 32;
+            const float* sl = p.sk_slots + (size_t)b * kSlotFloats + (size_t)warp * kF * DG * 16 * 32 + lane + f * 16 * 32;
 #pragma unroll
             for (int i = 0; i < 16; ++i) a[i] += __ldcg(sl + 32 * i);
         }
@@ -406,10 +413,12 @@ __device__ __noinline__ void sk_add_parts(const TmParams& p, uint32_t tw, int wa
 // bank conflicted); its blocks split 2x2 pooling windows, so the fused pool never uses it.
 // SHIFT 2 (fp32): column 0 at 1 (mod 4), each row two 16-byte loads, and blocks start at even
 // columns, so the fused pool's windows stay inside a block.
-template <int S, typename TIn, bool SORT = false, int SHIFT = 0, bool SK = false>
-__global__ void __launch_bounds__(kThreadsTM, 1)
+template <int S, typename TIn, bool SORT = false, int SHIFT = 0, bool SK = false, int DG = 1>
+__global__ void __launch_bounds__(kThreadsTM / DG, 1)
     pconv_tm(const TmParams p, const __grid_constant__ CUtensorMap tmap) {
     constexpr int RY = 4, RX = 4;
+    constexpr int NT = kThreadsTM / DG, NWP = kCompute / DG;   // threads, warps of the CTA
+    static_assert(DG == 1 || (S == 2 && !SORT), "two filter groups per warp: the stride-2 kernel");
     static_assert(!SHIFT || S == 1, "shifted blocks are a stride-1 layout");
     static_assert(SHIFT != 2 || sizeof(TIn) == 4, "blocks at 4j - 2 are an fp32 layout");
     extern __shared__ __align__(128) unsigned char smem[];
@@ -453,13 +462,13 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     if (!p.use_tma) {   // the fallback writes only in-image elements: zero all stages once
         float* z = reinterpret_cast<float*>(smem + p.stage_off);
         const int nf = (int)(kStages * p.stage_bytes / 4);
-        for (int i = threadIdx.x; i < nf; i += kThreadsTM) z[i] = 0.0f;
+        for (int i = threadIdx.x; i < nf; i += NT) z[i] = 0.0f;
     }
     if (warp == 0) {
         if (lane == 0) {
             for (int s = 0; s < kStages; ++s) {
-                mbar_init(full0 + 8 * s, kThreadsTM + 1);   // 512 cp.async arrivals + the expect-tx one
-                mbar_init(empty0 + 8 * s, kCompute);        // one arrival per warp
+                mbar_init(full0 + 8 * s, NT + 1);   // a cp.async arrival per thread + the expect-tx one
+                mbar_init(empty0 + 8 * s, NWP);     // one arrival per warp
             }
             *s_issued = 0;
         }
@@ -480,17 +489,20 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     // that chunk (loaded one fill ahead, so its latency hides behind a chunk of compute)
     // (units are read from the table where needed: few registers live across the loop)
     int fi = 0, fk = 0;
-    uint32_t fbeg = 0, fend = 0;
+    uint32_t fbeg[DG], fend[DG];
     auto fetch_range = [&]() {
-        fbeg = fend = 0;
-        if (fi < n_my) {
-            const Unit FU = s_units[fi];
-            const int g = FU.g0 + wg;
-            if (g < p.G) {
-                const int c0 = FU.c_lo + fk * p.CK;
-                const size_t b = (size_t)g * p.C;
-                fbeg = p.kofs[b + c0];
-                fend = p.kofs[b + min(c0 + p.CK, FU.c_hi)];
+#pragma unroll
+        for (int d = 0; d < DG; ++d) {
+            fbeg[d] = fend[d] = 0;
+            if (fi < n_my) {
+                const Unit FU = s_units[fi];
+                const int g = FU.g0 + wg * DG + d;
+                if (g < p.G) {
+                    const int c0 = FU.c_lo + fk * p.CK;
+                    const size_t b = (size_t)g * p.C;
+                    fbeg[d] = p.kofs[b + c0];
+                    fend[d] = p.kofs[b + min(c0 + p.CK, FU.c_hi)];
+                }
             }
         }
     };
@@ -502,8 +514,7 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
         fetch_range();
     };
     auto fill = [&](int q) {
-        fill_share<TIn>(p, &tmap, smem, full0, q, s_units[fi], fk, fbeg, fend,
-                        warp, lane);
+        fill_share<TIn, DG>(p, &tmap, smem, full0, q, s_units[fi], fk, fbeg, fend, warp, lane);
         advance_fill();
     };
     fetch_range();
@@ -513,10 +524,10 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
         if (threadIdx.x == 0) *s_issued = first;
     }
 
-    // tensor memory: warp w owns lanes 32*(w%4).. and columns 128*(w/4) + 16*slot ..
-    const uint32_t tw = tbase + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)(128 * (warp >> 2));
+    // tensor memory: warp w owns lanes 32*(w%4).. and columns 128*DG*(w/4) + 16*slot .. (DG*8 slots)
+    const uint32_t tw = tbase + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)(128 * DG * (warp >> 2));
 #pragma unroll
-    for (int f = 0; f < kF; ++f) tmem_zero16(tw + 16u * f);
+    for (int f = 0; f < kF * DG; ++f) tmem_zero16(tw + 16u * f);
 
     const int blk = ws * 32 + lane;
     const int lanes_t = 32 * p.WS, bpi = p.BY * p.BX;
@@ -580,26 +591,26 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
     // accumulators of unit U out of tensor memory (zeroed behind) + bias, ReLU, optional pool, to
     // the original channel; with a split, raw partial sums to the workspace
     auto epilogue = [&](const Unit& U) {
-        const int g = U.g0 + wg;
         const int n = U.n0 + img;
         const int oyb = U.oy0 + by * RY, oxb = U.ox0 + bx * RX - SHIFT;
         // balanced schedule: a part only publishes its raw sums; a head first adds its unit's
         // parts into tensor memory (out of line: the common path keeps its registers)
         if constexpr (SK) {
             if ((U.sk & 3) == kRolePart) {
-                sk_store_part(p, tw, warp, lane);
+                sk_store_part<DG>(p, tw, warp, lane);
                 return;
             }
-            if ((U.sk & 3) == kRoleHead) sk_add_parts(p, tw, warp, lane, blockIdx.x + 1, U.sk >> 2);
+            if ((U.sk & 3) == kRoleHead) sk_add_parts<DG>(p, tw, warp, lane, blockIdx.x + 1, U.sk >> 2);
         }
 #pragma unroll 1
-        for (int f = 0; f < kF; ++f) {
+        for (int f = 0; f < kF * DG; ++f) {
             float a[16];
             __syncwarp();
             tmem_ld16(tw + 16u * f, a);
             tmem_zero16(tw + 16u * f);
+            const int g = U.g0 + wg * DG + f / kF;
             if (g >= p.G || !active || n >= p.N) continue;
-            const uint32_t co = p.perm[g * kF + f];
+            const uint32_t co = p.perm[g * kF + f % kF];
             if (co == kPadSlot) continue;
             if (p.KS > 1) {   // raw partial sums of this split; bias, ReLU and rounding come later
                 float* wc = p.ws + (size_t)U.ks * p.ws_stride + ((size_t)n * p.Cout + co) * p.Ho * p.Wo;
@@ -738,14 +749,24 @@ __global__ void __launch_bounds__(kThreadsTM, 1)
         const int s = q % kStages;
         if (!mbar_wait_warp(full0 + 8 * s, (q / kStages) & 1, p.status, kStatusFullTimeout, p.wait_limit)) break;
         const Unit CU = s_units[ci];
-        if (CU.g0 + wg < p.G) {
+        if (CU.g0 + wg * DG < p.G) {
             const unsigned char* st = smem + p.stage_off + (size_t)s * p.stage_bytes;
             const uint32_t win_addr = smem_u32(reinterpret_cast<const TIn*>(st) + in_off);
-            const uint32_t desc_addr = smem_u32(reinterpret_cast<const uint64_t*>(st + p.desc_off) + wg * p.CK);
-            const uint32_t vals_addr = smem_u32(reinterpret_cast<const float4*>(st + p.vals_off) + wg * p.maxk);
+            const uint32_t desc_addr = smem_u32(reinterpret_cast<const uint64_t*>(st + p.desc_off) + wg * DG * p.CK);
+            const uint32_t vals_addr = smem_u32(reinterpret_cast<const float4*>(st + p.vals_off) + wg * DG * p.maxk);
             const int ckv = min(p.CK, CU.c_hi - CU.c_lo - ck * p.CK);
             constexpr int es = (int)sizeof(TIn);
-            if constexpr (S == 1 && es == 4 && SHIFT == 2) {
+            if constexpr (DG == 2) {   // the warp's second group: descriptors and weights one group up
+                const uint32_t desc_b = desc_addr + 8u * p.CK, vals_b = vals_addr + 16u * p.maxk;
+                const uint32_t valid_b = CU.g0 + wg * DG + 1 < p.G ? 1u : 0u;
+                if constexpr (es == 4) {
+                    PP_STAGE_KERNELS_S2_G2(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw, edge,
+                                           desc_b, vals_b, valid_b);
+                } else {
+                    PP_STAGE_KERNELS_S2_H_G2(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw, edge,
+                                             desc_b, vals_b, valid_b);
+                }
+            } else if constexpr (S == 1 && es == 4 && SHIFT == 2) {
                 PP_STAGE_KERNELS_S1_B(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw, edge);
             } else if constexpr (S == 1 && es == 4 && SHIFT == 1) {
                 PP_STAGE_KERNELS_S1_A(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw, edge);
@@ -2125,6 +2146,15 @@ bool pdl_enabled() {
     return on;
 }
 
+// Stride-2 layers give each warp two filter groups (PATCONV_S2_GROUPS=1: one, as stride 1 does).
+bool s2_two_groups() {
+    static const bool on = [] {
+        const char* e = std::getenv("PATCONV_S2_GROUPS");
+        return !(e && e[0] == '1');
+    }();
+    return on;
+}
+
 // The balanced schedule can be switched off (PATCONV_BALANCED=0): plans then take whole units.
 bool balanced_enabled() {
     static const bool on = [] {
@@ -2215,6 +2245,7 @@ struct Plan {
     int lane_sort = 0;            // stride 1: pconv_tm deals blocks to lanes by bank group
     int shift = 0;                // stride 1: blocks start at output columns 4j - shift (SHIFT)
     int streamk = 0;              // balanced schedule over sm_count() CTAs (KS = 1)
+    int dg = 1;                   // stride 2: filter groups per warp (2: 8 warps of 16 slots)
     size_t ws_bytes = 0;          // workspace the chosen split or schedule needs (0: none)
 };
 
@@ -2443,12 +2474,13 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
         // SMs idle (busy share <= 0.88) and there are at least 0.75 units per CTA.  It costs the
         // slots' traffic (256 KiB per CTA out and in, about 14 us a launch measured on VGG-16)
         // and the launch overlap of the previous kernel (a cooperative launch), so it is taken
-        // only with a 5 % margin.  Only for stride 1 and where the input goes through TMA
-        // (persistent CTAs)
+        // only with a 5 % margin.  Only where the input goes through TMA (persistent CTAs), and at
+        // stride 2 with two filter groups per warp
         pl->streamk = 0;
         const long long U1 = pl->ctas;   // whole units without a split
         const double busy = (double)U1 / ((double)sms * ((U1 + sms - 1) / sms));
-        if (S == 1 && allow_sk && balanced_enabled() && tma_rows && busy <= 0.88 && 4 * U1 >= 3 * sms) {
+        if ((S == 1 || (wg >= 2 && s2_two_groups())) && allow_sk && balanced_enabled() && tma_rows && busy <= 0.88 &&
+            4 * U1 >= 3 * sms) {
             const long long T = U1 * nck_total;
             const size_t skb = streamk_bytes(sms);
             if (T >= 2 * sms && U1 <= (long long)(kMaxUnitsPerCta - 2) * sms && ws_avail >= skb) {
@@ -2552,6 +2584,9 @@ int make_plan(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out
     double cost = 0;
     const int rc = make_plan_uncached(L, N, H, W, ws_avail, 0, &pl, &cost, allow_sk, es);
     if (rc != PP_OK) return rc;
+    // stride 2: two filter groups per warp (8 warps of 16 slots), so that each input window a lane
+    // loads from shared memory serves twice the kept kernels (these layers are held by shared memory)
+    if (L->stride == 2 && pl.WG >= 2 && s2_two_groups()) pl.dg = 2;
     if (L->stride == 1 && (!pool || es == 4)) {   // shifted blocks where their estimate is lower:
         // at 4j - 1 without the fused pool, at 4j - 2 (fp32 only) with it
         Plan ps;
@@ -2616,7 +2651,7 @@ __global__ void splitk_reduce_pool(const float* __restrict__ ws, T* __restrict__
 // Raise the kernel's dynamic shared-memory limit to the device's opt-in maximum once per device
 // (a launch needs at most that), so that later calls, including ones under stream capture, make
 // no attribute call.
-template <int S, typename T, bool SORT, int SHIFT, bool SK>
+template <int S, typename T, bool SORT, int SHIFT, bool SK, int DG = 1>
 bool allow_max_smem(size_t need) {
     static std::atomic<int> done[64];
     int dev = 0;
@@ -2625,7 +2660,7 @@ bool allow_max_smem(size_t need) {
     int optin = 0;
     if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess) return false;
     if ((size_t)optin < need) return false;
-    if (cudaFuncSetAttribute(pconv_tm<S, T, SORT, SHIFT, SK>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin) != cudaSuccess)
+    if (cudaFuncSetAttribute(pconv_tm<S, T, SORT, SHIFT, SK, DG>, cudaFuncAttributeMaxDynamicSharedMemorySize, optin) != cudaSuccess)
         return false;
     done[dev].store(1, std::memory_order_release);
     return true;
@@ -2636,11 +2671,20 @@ using TmKernel = void (*)(const TmParams, const CUtensorMap);
 // The kernel variant for a plan: the balanced-schedule variants (SK) exist for stride 1 only,
 // where the planner takes that schedule.
 template <int S, typename T, bool SORT, int SHIFT>
-TmKernel pick_tm(bool sk, size_t smem, bool* ok) {
+TmKernel pick_tm(bool sk, size_t smem, bool* ok, int dg = 1) {
     if constexpr (S == 1) {
         if (sk) {
             *ok = allow_max_smem<S, T, SORT, SHIFT, true>(smem);
             return pconv_tm<S, T, SORT, SHIFT, true>;
+        }
+    } else {
+        if (dg == 2 && sk) {
+            *ok = allow_max_smem<S, T, SORT, SHIFT, true, 2>(smem);
+            return pconv_tm<S, T, SORT, SHIFT, true, 2>;
+        }
+        if (dg == 2) {
+            *ok = allow_max_smem<S, T, SORT, SHIFT, false, 2>(smem);
+            return pconv_tm<S, T, SORT, SHIFT, false, 2>;
         }
     }
     *ok = allow_max_smem<S, T, SORT, SHIFT, false>(smem);
@@ -2732,7 +2776,7 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
         p.tma_bytes = (unsigned)((size_t)p.BWb * p.IH * p.CK * p.NB * es);
     }
     // balanced schedule (TMA path only: the copy fallback keeps one CTA per unit)
-    p.streamk = S == 1 && pl.streamk && p.use_tma ? 1 : 0;
+    p.streamk = (S == 1 || pl.dg == 2) && pl.streamk && p.use_tma ? 1 : 0;
     const bool sk = p.streamk != 0;
     TmKernel kern;
     bool smem_ok = false;
@@ -2750,7 +2794,7 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
         if (pl.shift) kern = pick_tm<1, T, false, 1>(sk, smem, &smem_ok);
         else kern = pick_tm<1, T, false, 0>(sk, smem, &smem_ok);
     } else {
-        kern = pick_tm<S, T, false, 0>(false, smem, &smem_ok);
+        kern = pick_tm<S, T, false, 0>(sk && pl.dg == 2, smem, &smem_ok, pl.dg);
     }
     if (!smem_ok) return PP_ERR_CUDA;
     const long long units = pl.ctas * pl.KS;
@@ -2765,7 +2809,7 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
                                                  align_up((size_t)P * kSlotFloats * sizeof(float), 256));
         if (cudaMemsetAsync(p.sk_flags, 0, (size_t)P * kCompute * sizeof(unsigned), st) != cudaSuccess)
             return PP_ERR_CUDA;
-        if (launch_ex(true, kern, (unsigned)P, kThreadsTM, smem, st, false, p, tmap) != cudaSuccess) return PP_ERR_CUDA;
+        if (launch_ex(true, kern, (unsigned)P, kThreadsTM / pl.dg, smem, st, false, p, tmap) != cudaSuccess) return PP_ERR_CUDA;
         return PP_OK;
     }
     // TMA path: one persistent CTA per SM walks its units as one chunk stream (the halo is zero
@@ -2774,7 +2818,7 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
     const long long ctas = p.use_tma ? std::max<long long>(std::min<long long>(units, sm_count()),
                                                            (units + kMaxUnitsPerCta - 1) / kMaxUnitsPerCta)
                                      : units;
-    if (launch(kern, (unsigned)ctas, kThreadsTM, smem, st, p, tmap) != cudaSuccess) return PP_ERR_CUDA;
+    if (launch(kern, (unsigned)ctas, kThreadsTM / pl.dg, smem, st, p, tmap) != cudaSuccess) return PP_ERR_CUDA;
     if (pl.KS > 1) {
         const size_t total = p.ws_stride;
         const unsigned blocks = (unsigned)std::max<size_t>(1, std::min<size_t>((total + 255) / 256, (size_t)sm_count() * 16));
@@ -3286,7 +3330,7 @@ int conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t*
               int es) {
     if (!h || !info) return PP_ERR_NULL;
     if (N < 1 || H < 1 || W < 1 || n_info < 1) return PP_ERR_SHAPE;
-    int64_t v[16] = {0};
+    int64_t v[17] = {0};
     if (h->depthwise) {
         v[0] = 2;   // depthwise kernels: no workspace
         DwsParams q{};
@@ -3325,11 +3369,12 @@ int conv_plan(pp_handle h, int N, int H, int W, size_t workspace_bytes, int64_t*
         v[10] = (int64_t)pl.smem;
         v[11] = pl.n_chunks;
         v[13] = pl.lane_sort;
+        v[16] = pl.dg;
         v[14] = pl.shift;
         v[15] = pl.streamk;
         if (pl.streamk) v[12] = sm_count();
     }
-    for (int i = 0; i < n_info && i < 16; ++i) info[i] = v[i];
+    for (int i = 0; i < n_info && i < 17; ++i) info[i] = v[i];
     return PP_OK;
 }
 }  // namespace

@@ -38,6 +38,11 @@ and (3, 4); with blocks at 4j - 1 the side-column taps (0, 3, 6 and 2, 5, 8), wh
 stay scalar.
 Taps are applied in ascending raster order for every output.
 
+Two filter groups per warp (the "_G2" macros, stride 2): per input channel both groups'
+descriptors are read and the window is loaded once; the kept kernels of the first group, then
+those of the second (weights from its own list, accumulators 128 tensor-memory columns up), run
+as one visit stream through the same bodies.
+
 Every branch is warp-uniform (bra.uni), so no convergence code surrounds the loop.  The macros'
 operands are listed in macro().  The library masks are the eight defaults (centre + 3 of the 4
 edge neighbours; centre + one edge + its 2 flanking corners).
@@ -54,7 +59,7 @@ def taps(mask):
     return [t for t in range(9) if (mask >> t) & 1]
 
 
-def macro(S, half=False, shift=0):
+def macro(S, half=False, shift=0, groups=1):
     RY = RX = 4
     WY, WX = (RY - 1) * S + 3, (RX - 1) * S + 3
     R = RY * RX
@@ -63,7 +68,9 @@ def macro(S, half=False, shift=0):
     # operands: %0 channels, %1 descriptor address, %2 weights address, %3 window address of
     # channel 0 (of window column -1 for shift 2), %4 row pitch in bytes, %5 channel plane in
     # bytes, %6 tensor-memory base, %7 nonzero where the left neighbour lane does not hold the
-    # block to the left (stride 2)
+    # block to the left (stride 2); with two filter groups per warp also %8 / %9 the second
+    # group's descriptor / weights addresses and %10 nonzero where that group exists (its
+    # accumulators sit 128 tensor-memory columns above the first group's)
     packed = S == 1
     aligned = shift == 1
     pairs = (0, 2, 4) if aligned else (1, 3)      # window columns starting an aligned pair
@@ -86,6 +93,9 @@ def macro(S, half=False, shift=0):
          "mov.b32 va, %2;",
          "mov.b32 rb0, %3;",
          "setp.ne.u32 EL, %7, 0;"]
+    if groups == 2:
+        L[1:1] = [".reg .pred VB;", ".reg .b32 dab, vaa, vab, cb, tot, tb;", ".reg .b64 db;"]
+        L += ["mov.b32 dab, %8;", "mov.b32 vab, %9;", "mov.b32 vaa, %2;", "setp.ne.u32 VB, %10, 0;"]
     for r in range(1, WY):
         L.append(f"add.u32 rb{r}, rb{r - 1}, %4;")
     L += ["CL:",
@@ -94,9 +104,19 @@ def macro(S, half=False, shift=0):
           "ld.shared.u64 d, [da];",
           "add.u32 da, da, 8;",
           "cvt.u32.u64 cnt, d;",
-          "and.b32 cnt, cnt, 15;",
-          "setp.eq.u32 P, cnt, 0;",
-          "@P bra.uni CN;"]
+          "and.b32 cnt, cnt, 15;"]
+    if groups == 2:   # the second group's descriptor (none where the group does not exist)
+        L += ["ld.shared.u64 db, [dab];",
+              "add.u32 dab, dab, 8;",
+              "@!VB mov.b64 db, 0;",
+              "cvt.u32.u64 cb, db;",
+              "and.b32 cb, cb, 15;",
+              "add.u32 tot, cnt, cb;",
+              "setp.eq.u32 P, tot, 0;",
+              "@P bra.uni CN;"]
+    else:
+        L += ["setp.eq.u32 P, cnt, 0;",
+              "@P bra.uni CN;"]
 
     def cvt_pair(p, a):                   # two packed halves to x{a}, x{a+1}
         return [f"mov.b32 {{h0, h1}}, {p};", f"cvt.f32.f16 x{a}, h0;", f"cvt.f32.f16 x{a + 1}, h1;"]
@@ -140,8 +160,23 @@ def macro(S, half=False, shift=0):
             L.append(f"ld.shared.f32 x{base + 5}, [rb{r}+20];")
         for c0 in pairs:
             L.append(f"mov.b64 xq{5 * r + c0}, {{x{base + c0}, x{base + c0 + 1}}};")
-    L += ["shr.b64 dd, d, 4;",
-          "PL:",
+    if groups == 2:
+        # one visit stream: the first group's kept kernels (weights from vaa, accumulators at the
+        # base), then the second group's (weights from vab, accumulators 128 columns up)
+        L += ["shr.b64 dd, d, 4;",
+              "mov.b32 va, vaa;",
+              "mov.b32 tb, %6;",
+              "setp.ne.u32 P, cnt, 0;",
+              "@P bra.uni PL;",
+              "shr.b64 dd, db, 4;",
+              "mov.b32 va, vab;",
+              "add.u32 tb, %6, 128;",
+              "mov.b32 cnt, cb;"]
+        tbase = "tb"
+    else:
+        L += ["shr.b64 dd, d, 4;"]
+        tbase = "%6"
+    L += ["PL:",
           "ld.shared.v4.f32 {w0, w1, w2, w3}, [va];",
           "add.u32 va, va, 16;",
           "cvt.u32.u64 code, dd;",
@@ -149,7 +184,7 @@ def macro(S, half=False, shift=0):
           "and.b32 pat, code, 7;",
           "and.b32 t1, code, 56;",
           "shl.b32 t1, t1, 1;",
-          "add.u32 ta, %6, t1;",
+          f"add.u32 ta, {tbase}, t1;",
           f"tcgen05.ld.sync.aligned.32x32b.x{R}.b32 {{{acc}}}, [ta];",
           "tcgen05.wait::ld.sync.aligned;",
           "setp.lt.u32 P, pat, 4;", "@P bra.uni T03;",
@@ -191,8 +226,25 @@ def macro(S, half=False, shift=0):
           "tcgen05.wait::st.sync.aligned;",
           "sub.u32 cnt, cnt, 1;",
           "setp.ne.u32 P, cnt, 0;",
-          "@P bra.uni PL;",
-          "CN:"]
+          "@P bra.uni PL;"]
+    if groups == 2:   # first group done: the second group's kept kernels, if any remain
+        L += ["setp.ne.u32 P, tb, %6;",
+              "@P bra.uni CE;",
+              "setp.eq.u32 P, cb, 0;",
+              "@P bra.uni CE;",
+              "shr.b64 dd, db, 4;",
+              "mov.b32 va, vab;",
+              "add.u32 tb, %6, 128;",
+              "mov.b32 cnt, cb;",
+              "bra.uni PL;",
+              "CE:",
+              "cvt.u32.u64 t1, d;",          # both groups' weight pointers past this channel
+              "and.b32 t1, t1, 15;",
+              "shl.b32 t1, t1, 4;",
+              "add.u32 vaa, vaa, t1;",
+              "shl.b32 t1, cb, 4;",
+              "add.u32 vab, vab, t1;"]
+    L += ["CN:"]
     for r in range(WY):
         L.append(f"add.u32 rb{r}, rb{r}, %5;")
     L += ["sub.u32 cl, cl, 1;",
@@ -202,12 +254,19 @@ def macro(S, half=False, shift=0):
     body = "\\n\\t".join(L)
     tag = {0: "", 1: "A", 2: "B"}[shift]
     name = f"PP_STAGE_KERNELS_S{S}" + ("_H" if half else "") + ((tag if half else "_" + tag) if tag else "")
+    if groups == 2:
+        name += "_G2"
+        what_g = ", two filter groups per warp"
+    else:
+        what_g = ""
     where = {0: "", 1: ", window column 0 at 2 mod 4", 2: ", window column 0 at 1 mod 4"}[shift]
-    what = f"stride {S}{', fp16 stage' if half else ''}{where}"
+    what = f"stride {S}{', fp16 stage' if half else ''}{where}{what_g}"
+    extra_args = ", desc_b, vals_b, valid_b" if groups == 2 else ""
+    extra_ops = ', "r"(desc_b), "r"(vals_b), "r"(valid_b)' if groups == 2 else ""
     return (f"// {what}: 4x4 outputs per lane, {WY}x{WX} input window\n"
-            f"#define {name}(nch, desc_addr, vals_addr, win_addr, pitch_b, plane_b, tbase, edge) \\\n"
+            f"#define {name}(nch, desc_addr, vals_addr, win_addr, pitch_b, plane_b, tbase, edge{extra_args}) \\\n"
             f'    asm volatile("{body}" :: "r"(nch), "r"(desc_addr), "r"(vals_addr), "r"(win_addr), '
-            f'"r"(pitch_b), "r"(plane_b), "r"(tbase), "r"(edge) : "memory")\n')
+            f'"r"(pitch_b), "r"(plane_b), "r"(tbase), "r"(edge){extra_ops} : "memory")\n')
 
 
 def generate() -> str:
@@ -216,6 +275,8 @@ def generate() -> str:
     for S in STRIDES:
         for half in (False, True):
             text.append(macro(S, half))
+            if S == 2:
+                text.append(macro(S, half, groups=2))
             if S == 1:
                 text.append(macro(S, half, shift=1))
                 if not half:

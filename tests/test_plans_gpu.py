@@ -127,6 +127,27 @@ def test_no_balanced_schedule_without_tma_rows():
     assert plan["streamk"] == 0
 
 
+@pytest.mark.parametrize("cout,cin,n,h,io,groups", [
+    (128, 64, 16, 56, "f32", 2),    # ResNet-50's first stage head, at a smaller batch
+    (40, 24, 3, 30, "f32", 2),      # 5 filter groups: one warp's second group missing, one warp idle
+    (256, 128, 8, 28, "f16", 2),    # fp16 stages
+    (64, 32, 4, 29, "f32", 2),      # odd map: the copy fallback, a ragged last block row and column
+    (8, 16, 2, 20, "f32", 1),       # a single filter group: one group per warp
+])
+def test_stride2_two_groups_per_warp(cout, cin, n, h, io, groups):
+    """Stride-2 launches give each warp two filter groups (8 warps of 16 slots, one input window
+    per lane serving both groups' kept kernels) wherever a unit holds two groups or more."""
+    plan, _ = _run(cout, cin, n, h, h, 0.4, io, stride=2, seed=30 + h)
+    assert plan["groups_per_warp"] == groups
+
+
+def test_stride2_balanced_schedule():
+    """512 input channels, 128 whole units at stride 2: the balanced schedule over 152 CTAs with
+    two filter groups per warp (a part's 16 slots per warp go to its workspace slot)."""
+    plan, _ = _run(256, 512, 32, 56, 56, 0.4, "f32", stride=2, seed=41)
+    assert plan["streamk"] == 1 and plan["groups_per_warp"] == 2 and plan["ctas"] == _sms()
+
+
 def test_batch_one_split_32_ways():
     plan, _ = _run(256, 256, 1, 14, 14, 0.25, "f32", seed=5)
     assert plan["splits"] == 32 and plan["shift"] == 1
