@@ -33,6 +33,13 @@ def _no_pipeline_timeout():
     assert st.value == 0, f"a conv kernel recorded pipeline timeout bits {st.value:#x}"
 
 
+SPLIT_CAP = 32 << 20   # a workspace below the balanced schedule's (39 MB): the input-channel split
+
+
+def _sms():
+    return torch.cuda.get_device_properties(0).multi_processor_count
+
+
 def _np_dt(dt):
     return np.float32 if dt == torch.float32 else np.float16
 
@@ -418,7 +425,7 @@ def test_conv_pool_fused_with_split_equals_unfused_pool():
     x = torch.from_numpy(WL.layer_input(L, 16)).cuda()
     bt = torch.from_numpy(b).cuda()
     layer = api.pp_pack(W, None, L.keep).bind("cuda")
-    nb = max(layer.workspace_bytes(x.shape, pool2x2=True), layer.workspace_bytes(x.shape))
+    nb = min(max(layer.workspace_bytes(x.shape, pool2x2=True), layer.workspace_bytes(x.shape)), SPLIT_CAP)
     assert layer.plan(x.shape, nb, pool2x2=True)["splits"] > 1
     ws = torch.full((nb // 4,), float("nan"), device="cuda")
     fused = layer.conv(x, bt, True, workspace=ws, pool2x2=True)
@@ -519,13 +526,15 @@ def _split_case():
 
 
 def test_split_is_planned_for_small_images():
-    """14x14 maps leave SMs idle with whole units: with a workspace the input-channel split
-    (their 56-byte fp32 rows take the copy fallback, which keeps one CTA per unit, so not the
-    balanced schedule), without one a single pass."""
+    """14x14 maps leave SMs idle with whole units (64 units of two whole images on 152 SMs; their
+    56-byte fp32 rows take the copy fallback): with the full workspace the balanced schedule over
+    persistent CTAs, with less than it needs the input-channel split, without one a single pass."""
     L, W, b, x = _split_case()
     lay = api.pp_pack(W, None, L.keep)
     plan = lay.plan(x.shape, lay.workspace_bytes(x.shape))
-    assert plan["path"] == 1 and plan["splits"] > 1 and plan["streamk"] == 0
+    assert plan["path"] == 1 and plan["splits"] == 1 and plan["streamk"] == 1 and plan["ctas"] == _sms()
+    plan = lay.plan(x.shape, SPLIT_CAP)
+    assert plan["splits"] > 1 and plan["streamk"] == 0
     assert lay.plan(x.shape, 0)["splits"] == 1
     big = api.pp_pack(WL.weights(WL.vgg16()[1]), None, 0.3)
     assert big.plan((32, 64, 224, 224), 1 << 34)["splits"] == 1
@@ -533,14 +542,32 @@ def test_split_is_planned_for_small_images():
 
 def test_split_matches_oracle_single_pass_and_is_deterministic():
     L, W, b, x = _split_case()
-    y_split, lay = run_gpu(W, x, b, L.keep, ws=True)
-    y_split2, _ = run_gpu(W, x, b, L.keep, ws=True)
+    y_split, lay = run_gpu(W, x, b, L.keep, ws=True, ws_bytes=SPLIT_CAP)
+    y_split2, _ = run_gpu(W, x, b, L.keep, ws=True, ws_bytes=SPLIT_CAP)
     y_one, _ = run_gpu(W, x, b, L.keep, ws=False)
     assert np.array_equal(y_split, y_split2)
     ref, den = oracle(W, x[[0, 31]], b, L.keep)
     assert OC.max_norm_err(y_split[[0, 31]], ref, den) <= 1e-4
     d = np.abs(y_split - y_one) / np.maximum(np.abs(y_one), 1e-3)
     assert float(np.max(d)) < 1e-3                       # only fp32 summation order differs
+
+
+def test_balanced_schedule_copy_fallback_whole_images():
+    """The same 14x14 layer with the full workspace: persistent CTAs over the copy fallback's
+    stages (the zero halo of whole-image tiles is the same for every unit) and the balanced
+    schedule; deterministic, within the oracle's tolerance, and equal to the single pass up to
+    fp32 summation order."""
+    L, W, b, x = _split_case()
+    lay = api.pp_pack(W, None, L.keep)
+    assert lay.plan(x.shape, lay.workspace_bytes(x.shape))["streamk"] == 1
+    y1, _ = run_gpu(W, x, b, L.keep, ws=True)
+    y2, _ = run_gpu(W, x, b, L.keep, ws=True)
+    y0, _ = run_gpu(W, x, b, L.keep, ws=False)
+    assert np.array_equal(y1, y2)
+    ref, den = oracle(W, x[[0, 31]], b, L.keep)
+    assert OC.max_norm_err(y1[[0, 31]], ref, den) <= 1e-4
+    d = np.abs(y1 - y0) / np.maximum(np.abs(y0), 1e-3)
+    assert float(np.max(d)) < 1e-3
 
 
 def test_balanced_schedule_matches_oracle_and_is_deterministic():
