@@ -2263,7 +2263,8 @@ struct PlanCache : PlanCacheBase {
 // Candidate spatial tiles of at most 32*WS blocks (4x4 outputs each; with shift, block j of a row
 // starts at output column 4j - shift, so a row of Wo outputs takes (Wo + shift + 3) / 4 blocks).
 //   rectangles: BY x BX blocks of one image (several whole images when the rectangle is the
-//     whole image); stride-1 rows need 4*BX + 5 staged columns, stride-2 rows 8*BX + 4, rounded
+//     whole image; several images side by side when it is a band of full block rows, below);
+//     stride-1 rows need 4*BX + 5 staged columns, stride-2 rows 8*BX + 4, rounded
 //     to a 16-byte multiple and padded to 4 (mod 8) floats so that rows four apart fall in other
 //     banks;
 //   linear: 32*WS consecutive blocks of the (image, block row, block column) sequence, staged as
@@ -2288,6 +2289,21 @@ std::vector<TileChoice> tile_candidates(int N, int Ho, int Wo, int S, int lanes,
         }
     }
     const long long bpi = (long long)nby * nbx;
+    // bands: full-width rectangles of `by` block rows (a divisor of the image's block rows, so no
+    // row is computed past the image) of several images side by side in one stage, where a whole
+    // image is more than the lanes hold.  28x28 outputs are 7 block rows: rectangles of 4 block
+    // rows compute 8 of them, bands of 1 block row of 4 images exactly 7.  Listed after the
+    // rectangles, so they are taken only where they cover strictly fewer lanes.  Measured against
+    // the rectangles they replace: VGG-16's 28x28 layers 7-10 % faster (4.74 -> 4.60 ms a step),
+    // ResNet-50's 56x56 and 28x28 layers 9 and 6 %, its first stride-2 head 13 %
+    if (bpi > lanes) {
+        for (int by = 1; by < nby && by * nbx <= lanes / 2; ++by) {
+            if (nby % by) continue;
+            const int nb = std::min(N, lanes / (nbx * by));
+            const int ih = ih_of(by), bw = bw_of(nbx);
+            if (nb >= 2 && bw <= 256 && ih <= 256) out.push_back(TileChoice{by, nbx, nb, ih, bw, 0});
+        }
+    }
     if (bpi < lanes && lanes % bpi == 0) return out;    // the whole-image rectangle is this tile
     const int nb = (int)std::min<long long>(N, (lanes - 1) / bpi + 2);
     const int ih = ih_of(nby), bw = bw_of(nbx);
@@ -2480,19 +2496,23 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
         const long long U1 = pl->ctas;   // whole units without a split
         const double busy = (double)U1 / ((double)sms * ((U1 + sms - 1) / sms));
         // persistent CTAs: through TMA, or rectangles of whole images (the copy fallback's zero
-        // halo is then the same for every unit).  Copy-fallback rectangles of whole images take the
-        // schedule down to 0.2 units per CTA and whatever the estimate: measured faster than the
-        // channel split on 128 CTAs by 13 % on VGG-16's 14x14 layers (64 units, batch 32) and by
-        // 8-10 % on ResNet-50's 14x14 and 7x7 layers (64 and 32 units, batch 64)
+        // halo is then the same for every unit).  Two kinds of launch take the schedule down to 0.2
+        // units per CTA and whatever the estimate, as measured faster than whole units or the
+        // channel split on 128 CTAs: copy-fallback rectangles of whole images (VGG-16's 14x14 layers
+        // 13 %, 64 units at batch 32; ResNet-50's 14x14 and 7x7 layers 8-10 %, 64 and 32 units at
+        // batch 64), stride 2 with two filter groups per warp (ResNet-50's heads 5 and 12 %,
+        // 128 units of 128 input channels and 64 units of 256) and bands (the estimate puts them
+        // level with a 2-way channel split, whose partial sums and reduction pass it leaves out)
         const bool whole = tx == 1 && ty == 1 && !t.linear && !tma_rows;
+        const bool relax = whole || S == 2 || (t.NB > 1 && ty > 1);
         const bool persist = tma_rows || whole;
         if ((S == 1 || (wg >= 2 && s2_two_groups())) && allow_sk && balanced_enabled() && persist && busy <= 0.88 &&
-            (4 * U1 >= 3 * sms || whole)) {
+            (4 * U1 >= 3 * sms || relax)) {
             const long long T = U1 * nck_total;
             const size_t skb = streamk_bytes(sms);
             if (T >= 2 * sms && U1 <= (long long)(kMaxUnitsPerCta - 2) * sms && ws_avail >= skb) {
                 const double cost_sk = (double)U1 * (C + 2.0 * nck_total) / sms + 4.0 * ck + 42.0;
-                if (cost_sk < 0.95 * steps || whole) {
+                if (cost_sk < 0.95 * steps || relax) {
                     steps = cost_sk;
                     pl->streamk = 1;
                     pl->KS = 1;
@@ -2517,6 +2537,9 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
     bool have_rect = false, have_lin = false;
     for (const TileChoice& t : tile_candidates(N, Ho, Wo, S, lanes, shift)) {
         if ((long long)t.NB * t.IH * t.BWb * 4 * ck_min > 48 * 1024) continue;
+        // bands only through TMA: the copy fallback (one CTA per unit) stages their extra halo
+        // rows with the compute threads
+        if (t.NB > 1 && t.BY < nby && !t.linear && !tma_rows) continue;
         if (t.linear) {
             lin = t;
             have_lin = true;

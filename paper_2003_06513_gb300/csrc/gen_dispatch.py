@@ -185,9 +185,10 @@ def macro(S, half=False, shift=0, groups=1):
           "and.b32 t1, code, 56;",
           "shl.b32 t1, t1, 1;",
           f"add.u32 ta, {tbase}, t1;",
-          f"tcgen05.ld.sync.aligned.32x32b.x{R}.b32 {{{acc}}}, [ta];",
-          "tcgen05.wait::ld.sync.aligned;",
-          "setp.lt.u32 P, pat, 4;", "@P bra.uni T03;",
+          f"tcgen05.ld.sync.aligned.32x32b.x{R}.b32 {{{acc}}}, [ta];"]
+    if groups == 1:
+        L += ["tcgen05.wait::ld.sync.aligned;"]
+    L += ["setp.lt.u32 P, pat, 4;", "@P bra.uni T03;",
           "setp.lt.u32 P, pat, 6;", "@P bra.uni T45;",
           "setp.eq.u32 P, pat, 6;", "@P bra.uni B6;", "bra.uni B7;",
           "T45:", "setp.eq.u32 P, pat, 4;", "@P bra.uni B4;", "bra.uni B5;",
@@ -196,6 +197,8 @@ def macro(S, half=False, shift=0, groups=1):
           "T01:", "setp.eq.u32 P, pat, 0;", "@P bra.uni B0;", "bra.uni B1;"]
     for p, m in enumerate(MASKS):
         L.append(f"B{p}:")
+        if groups == 2:              # the accumulators' load flew during the pattern dispatch
+            L.append("tcgen05.wait::ld.sync.aligned;")
         tp = taps(m)
         if packed:
             L += [f"mov.b64 ap{i}, {{a{2 * i}, a{2 * i + 1}}};" for i in range(R // 2)]
@@ -222,9 +225,10 @@ def macro(S, half=False, shift=0, groups=1):
         if p != len(MASKS) - 1:
             L.append("bra.uni BS;")
     L += ["BS:",
-          f"tcgen05.st.sync.aligned.32x32b.x{R}.b32 [ta], {{{acc}}};",
-          "tcgen05.wait::st.sync.aligned;",
-          "sub.u32 cnt, cnt, 1;",
+          f"tcgen05.st.sync.aligned.32x32b.x{R}.b32 [ta], {{{acc}}};"]
+    if groups == 1:
+        L += ["tcgen05.wait::st.sync.aligned;"]
+    L += ["sub.u32 cnt, cnt, 1;",
           "setp.ne.u32 P, cnt, 0;",
           "@P bra.uni PL;"]
     if groups == 2:   # first group done: the second group's kept kernels, if any remain
@@ -245,6 +249,8 @@ def macro(S, half=False, shift=0, groups=1):
               "shl.b32 t1, cb, 4;",
               "add.u32 vab, vab, t1;"]
     L += ["CN:"]
+    if groups == 2:   # the channel's stores complete before a later channel loads the same slot
+        L += ["tcgen05.wait::st.sync.aligned;"]
     for r in range(WY):
         L.append(f"add.u32 rb{r}, rb{r}, %5;")
     L += ["sub.u32 cl, cl, 1;",

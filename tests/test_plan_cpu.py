@@ -202,10 +202,12 @@ def test_other_paths_report_no_plan():
 
 
 def test_linear_tile_weighed_by_density():
-    """28x28 maps with blocks at columns 4j (7 blocks a row, the fp16 fused-pool layout): at
-    VGG-16's keep 0.3 the planner takes 4x7 rectangles without a split; at keep 1.0 the linear
-    tile (every lane busy) pays for its per-channel cost.  With blocks at 4j - 1 (no pool) or
-    4j - 2 (fp32 pool) a row has 8 blocks, and 4x8 rectangles keep every lane busy."""
+    """28x28 maps with blocks at columns 4j (7 blocks a row, the fp16 fused-pool layout, rows
+    through the copy fallback): at VGG-16's keep 0.3 the planner takes 4x7 rectangles without a
+    split; at keep 1.0 the linear tile (every lane busy) pays for its per-channel cost.  With
+    blocks at 4j - 1 (no pool) or 4j - 2 (fp32 pool) a row has 8 blocks, and fp32 rows go through
+    TMA: bands of one block row of 4 images keep every lane busy and compute the 7 block rows of
+    an image exactly (rectangles of 4 block rows compute 8), on the balanced schedule."""
     f16 = torch.float16
     for L in WL.vgg16()[7:10]:
         layer = api.pp_pack(WL.weights(L), None, L.keep)
@@ -213,9 +215,11 @@ def test_linear_tile_weighed_by_density():
         pl = layer.plan(shape, layer.workspace_bytes(shape, True, f16), pool2x2=True, dtype=f16)
         assert (pl["tile_by"], pl["tile_bx"], pl["tile_nb"], pl["splits"], pl["shift"]) == (4, 7, 1, 1, 0), L.name
         pl = layer.plan(shape, layer.workspace_bytes(shape, True), pool2x2=True)
-        assert (pl["tile_by"], pl["tile_bx"], pl["tile_nb"], pl["splits"], pl["shift"]) == (4, 8, 1, 1, 2), L.name
+        assert (pl["tile_by"], pl["tile_bx"], pl["tile_nb"], pl["splits"], pl["shift"]) == (1, 8, 4, 1, 2), L.name
+        assert pl["streamk"] == 1, L.name
         pl = layer.plan(shape, layer.workspace_bytes(shape))
-        assert (pl["tile_by"], pl["tile_bx"], pl["tile_nb"], pl["splits"], pl["shift"]) == (4, 8, 1, 1, 1), L.name
+        assert (pl["tile_by"], pl["tile_bx"], pl["tile_nb"], pl["splits"], pl["shift"]) == (1, 8, 4, 1, 1), L.name
+        assert pl["streamk"] == 1, L.name
     rng = np.random.default_rng(7)
     W = (rng.standard_normal((256, 256, 3, 3)) * np.sqrt(2 / (9 * 256))).astype(np.float32)
     shape = (64, 256, 28, 28)

@@ -2,7 +2,8 @@
 full batch.
 
 Each case states the plan outcome it exercises and asserts it through layer.plan (the same plan
-the launch uses): linear tiles, rectangles of several whole images, the bank-group lane order,
+the launch uses): linear tiles, rectangles of several whole images, bands of block rows of
+several images, the bank-group lane order,
 blocks shifted to start at output columns 4j - 1 (4j - 2 under the fp32 fused pool), the copy
 fallback for rows that are not a multiple of 16 bytes, fp16 stages through TMA without the fused
 pool, input-channel splits up to 32 ways, the balanced schedule, more units than one persistent
@@ -71,10 +72,39 @@ def test_units_overflow_the_persistent_table():
 def test_linear_tile(pool):
     """28x28 maps at keep 1.0: lanes take consecutive blocks across image boundaries (whole
     images staged, several per tile), with a split."""
-    plan, _ = _run(256, 256, 64, 28, 28, 1.0, "f32", pool=pool, seed=2)
+    plan, _ = _run(128, 128, 64, 28, 28, 1.0, "f32", pool=pool, seed=2)
     nb_rect = max(1, 32 * plan["spatial_warps"] // (plan["tile_by"] * plan["tile_bx"]))
     assert (plan["tile_by"], plan["tile_bx"]) == (7, 7) and plan["tile_nb"] > nb_rect   # linear
     assert plan["shift"] == 0 and plan["splits"] > 1 and plan["streamk"] == 0
+
+
+@pytest.mark.parametrize("case", [
+    # cout, cin, n, h, keep, io, pool, stride, workspace cap (None: what the plan asks for)
+    (256, 256, 8, 28, 0.3, "f32", False, 1, None),     # bands and a channel split
+    (256, 256, 8, 28, 0.3, "f32", False, 1, 0),        # bands alone
+    (256, 256, 8, 28, 0.3, "f32", True, 1, None),      # fused pool, blocks at 4j - 2
+    (64, 64, 16, 56, 0.4, "f16", False, 1, None),      # fp16 stages (56 halves: TMA rows)
+    (256, 256, 32, 28, 0.3, "f32", False, 1, None),    # balanced schedule (VGG-16 28x28 shape)
+    (64, 64, 16, 56, 0.4, "f32", False, 1, None),      # two spatial warps, bank-group lane order
+    (128, 128, 8, 56, 0.4, "f32", False, 2, None),     # stride 2, two filter groups per warp
+    (128, 128, 8, 56, 0.4, "f16", False, 2, 0),
+])
+def test_band_tiles(case):
+    """Bands: full-width rectangles of whole block rows of several images side by side in one
+    stage (28x28 outputs: one block row of 4 images; 56x56: one block row of 4 images over two
+    spatial warps), so no output row is computed past the image."""
+    cout, cin, n, h, keep, io, pool, stride, cap = case
+    plan, _ = _run(cout, cin, n, h, h, keep, io, pool=pool, stride=stride, seed=40 + h + n, ws_cap=cap)
+    ho = (h - 1) // stride + 1
+    nby, nbx = -(-ho // 4), (ho + plan["shift"] + 3) // 4
+    assert plan["tile_bx"] == nbx and plan["tile_by"] < nby and nby % plan["tile_by"] == 0
+    assert plan["tile_nb"] > 1 and plan["tile_by"] * nbx * plan["tile_nb"] <= 32 * plan["spatial_warps"]
+    if n == 32:
+        assert plan["streamk"] == 1
+    if stride == 2:
+        assert plan["groups_per_warp"] == 2
+    if cap == 0:
+        assert plan["splits"] == 1 and plan["streamk"] == 0
 
 
 @pytest.mark.parametrize("pool", [False, True])
