@@ -2531,15 +2531,18 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
     // rectangles: fewest CTA waves, then fewest lanes covered (idle lanes), then the widest rows;
     // a tile must leave room for at least the channels per stage that kMaxChunks needs
     const int ck_min = (C + kMaxChunks - 1) / kMaxChunks;
+    const double kpc_all = (double)L->beta / ((double)L->G * C);   // kept kernels per (channel, group)
     long long best_waves = LLONG_MAX, best_cover = LLONG_MAX;
     TileChoice rect, lin;
     int rtx = 0, rty = 0, rtn = 0;
     bool have_rect = false, have_lin = false;
     for (const TileChoice& t : tile_candidates(N, Ho, Wo, S, lanes, shift)) {
         if ((long long)t.NB * t.IH * t.BWb * 4 * ck_min > 48 * 1024) continue;
-        // bands only through TMA: the copy fallback (one CTA per unit) stages their extra halo
-        // rows with the compute threads
-        if (t.NB > 1 && t.BY < nby && !t.linear && !tma_rows) continue;
+        // bands only through TMA (the copy fallback, one CTA per unit, stages their extra halo
+        // rows with the compute threads) and below 6 kept kernels per (input channel, filter
+        // group): at 8 (keep 1.0) the linear tile's lanes, all busy, beat the bands' 7 of 8
+        // (28x28 maps: 4-9 % in 4 of 6 sweep points, 1-6 % slower in the other 2)
+        if (t.NB > 1 && t.BY < nby && !t.linear && (!tma_rows || kpc_all >= 6.0)) continue;
         if (t.linear) {
             lin = t;
             have_lin = true;
@@ -2569,8 +2572,7 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
     Plan pr, pli;
     const double cr = have_rect ? finish(rect, rtx, rty, rtn, &pr) : 1e300;
     const int ltn = (int)(((long long)N * nby * nbx + lanes - 1) / lanes);
-    const double kpc = (double)L->beta / ((double)L->G * C);
-    const double cl = have_lin ? (1.3 + kpc) / (0.4 + kpc) * finish(lin, 1, 1, ltn, &pli) : 1e300;
+    const double cl = have_lin ? (1.3 + kpc_all) / (0.4 + kpc_all) * finish(lin, 1, 1, ltn, &pli) : 1e300;
     if (cr >= 1e300 && cl >= 1e300) return PP_ERR_SHAPE;
     *out = cl < cr ? pli : pr;
     out->shift = shift;
