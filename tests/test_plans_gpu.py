@@ -85,6 +85,7 @@ def test_linear_tile(pool):
     (256, 256, 8, 28, 0.3, "f32", True, 1, None),      # fused pool, blocks at 4j - 2
     (64, 64, 16, 56, 0.4, "f16", False, 1, None),      # fp16 stages (56 halves: TMA rows)
     (256, 256, 32, 28, 0.3, "f32", False, 1, None),    # balanced schedule (VGG-16 28x28 shape)
+    (256, 256, 30, 28, 0.3, "f32", False, 1, 0),       # a last band of 2 images (30 = 7 x 4 + 2)
     (64, 64, 16, 56, 0.4, "f32", False, 1, None),      # two spatial warps, bank-group lane order
     (128, 128, 8, 56, 0.4, "f32", False, 2, None),     # stride 2, two filter groups per warp
     (128, 128, 8, 56, 0.4, "f16", False, 2, 0),
