@@ -185,7 +185,9 @@ int pp_conv_workspace_size(pp_handle h, int N, int H, int W, size_t* bytes);
 /* Launch plan of pp_conv_ws for a call shape and workspace size, for tests and tuning:
  * info[0] = path (1 dense fast kernel, 2 depthwise kernel, 3 generic kernel); for path 1:
  * info[1] channel splits KS, [2] workspace bytes used, [3] work units (spatial tiles x filter
- * chunks x splits), [4..6] tile BY, BX, NB (4x4 output blocks, images), [7] channels per stage,
+ * chunks x splits), [4..6] tile BY, BX, NB (4x4 output blocks; NB > 1 images side by side in one
+ * stage: whole images, the linear tile's consecutive blocks across images, or bands of BY full
+ * block rows where a whole image exceeds the lanes), [7] channels per stage,
  * [8] filter groups and [9] spatial warps per CTA, [10] shared-memory bytes, [11] channel chunks
  * per unit, [12] CTAs launched when the input goes through TMA (fp32 with rows a multiple of 16
  * bytes: persistent CTAs, at most one per SM unless the units overflow a CTA's unit table; the
@@ -202,7 +204,7 @@ int pp_conv_workspace_size(pp_handle h, int N, int H, int W, size_t* bytes);
  * between two CTAs is finished by the CTA holding its first chunks, which adds the later ones'
  * raw sums from their workspace slots (workspace: 256 KiB per SM + flags, reported in [2]; the
  * launch is cooperative and resets the flags with a small memset first; the input must go
- * through TMA, else the launch takes whole units), else 0; [16] filter groups per warp (2 for
+ * through TMA, or the tile be whole images, else the launch takes whole units), else 0; [16] filter groups per warp (2 for
  * stride-2 layers: 8 warps of 16 filter slots, each input window serving both groups' kept
  * kernels; else 1).  For path 2 (depthwise), assuming
  * x and y 16-byte aligned (else the row-item kernels run): info[1] = 1 streamed kernel in rows

@@ -1,31 +1,37 @@
 // CUDA kernels and launchers of libpatconv (sm_103a): pattern-sparse 3x3 convolution.
 //
-// Dense layers, main kernel pconv_tm<S, T, SORT, SHIFT, SK>:
+// Dense layers, main kernel pconv_tm<S, T, SORT, SHIFT, SK, DG>:
 //   * a lane owns a 4x4 block of output pixels of one image; a warp owns one filter group (8
-//     filter slots, the "filter kernel reorder" of §3.4) for its 32 blocks; a CTA is 16 warps =
-//     WG filter groups x WS spatial warps over one spatial tile;
+//     filter slots, the "filter kernel reorder" of §3.4), or DG = 2 groups at stride 2, for its
+//     32 blocks; a CTA is 16 / DG warps = WG filter groups x WS spatial warps over one tile;
+//   * tiles: rectangles of blocks of one image, several whole images, bands of full block rows
+//     of several images side by side, or the linear tile (consecutive blocks across images);
 //   * accumulators live in tensor memory: 16 warps x 8 slots x 16 fp32 = all 512 columns; a kept
 //     kernel is applied by tcgen05.ld of its slot, 64 FMAs, tcgen05.st;
 //   * input channels stream through a 3-stage mbarrier pipeline: one TMA box per stage (the tile
 //     of CK channels with its zero halo, padding 1) or, where rows are not 16-byte multiples, a
-//     copy shared by all 512 threads; each group's descriptors and kept weights for those channels
+//     copy shared by all threads; each group's descriptors and kept weights for those channels
 //     arrive by cp.async beside it;
 //   * per input channel a lane loads its input window into registers once and applies it to every
-//     kept kernel of its group: the 6-bit (slot, pattern) code of each kept kernel selects one of
-//     8 compile-time pattern bodies (generated inline PTX, gen_dispatch.py) whose four tap
+//     kept kernel of its group(s): the 6-bit (slot, pattern) code of each kept kernel selects one
+//     of 8 compile-time pattern bodies (generated inline PTX, gen_dispatch.py) whose four tap
 //     operands are fixed registers (the 4 taps of §3.2), so no per-element index is decoded;
+//     SHIFT moves the blocks to output columns 4j - 1 or 4j - 2 (aligned window loads), SORT
+//     deals a warp's blocks to lanes by shared-memory bank group;
 //   * persistent CTAs (one per SM unless the units overflow a CTA's table) walk their units
 //     (tile, filter chunk, input-channel split) as one chunk stream;
-//   * SK (balanced schedule, stride 1): one CTA per SM takes an equal range of all units'
-//     channel chunks; a unit cut between CTAs is finished by the CTA holding its first chunks,
-//     which adds the later CTAs' raw sums (a cooperative launch: every CTA is resident);
+//   * SK (balanced schedule): one CTA per SM takes an equal range of all units' channel chunks;
+//     a unit cut between CTAs is finished by the CTA holding its first chunks, which adds the
+//     later CTAs' raw sums (a cooperative launch: every CTA is resident);
 //   * epilogue: + bias, ReLU, optionally the 2x2 max-pool, fp32 or fp16 (round to nearest even)
 //     stores to the original channel of each slot, or raw partial sums to the split workspace;
 //   * every pipeline wait is bounded; a wait that runs out records a bit in the status word and
 //     the kernel drains its copies, frees tensor memory and returns.
-// Depthwise layers: pconv_depthwise / pconv_depthwise_staged (HBM-bound).  Other pattern
-// libraries: pconv_generic.  The path is a gathered sparse contraction, so it runs on the
-// CUDA-core FFMA pipe.
+// Depthwise layers (one pattern per channel, HBM-bound): pconv_dw_stream, per-warp bulk-copy
+// pipelines of a persistent CTA per SM (rows, planes and tiles modes) for 16-byte aligned
+// tensors; pconv_depthwise / pconv_depthwise_staged for the rest.  Other pattern libraries:
+// pconv_generic.  The path is a gathered sparse contraction, so it runs on the CUDA-core FFMA
+// pipe.
 #include <cuda_fp16.h>
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -2490,8 +2496,8 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
         // SMs idle (busy share <= 0.88) and there are at least 0.75 units per CTA.  It costs the
         // slots' traffic (256 KiB per CTA out and in, about 14 us a launch measured on VGG-16)
         // and the launch overlap of the previous kernel (a cooperative launch), so it is taken
-        // only with a 5 % margin.  Only where the input goes through TMA (persistent CTAs), and at
-        // stride 2 with two filter groups per warp
+        // only with a 5 % margin.  Only on persistent CTAs (the input through TMA, or tiles of
+        // whole images), at stride 1 or at stride 2 with two filter groups per warp
         pl->streamk = 0;
         const long long U1 = pl->ctas;   // whole units without a split
         const double busy = (double)U1 / ((double)sms * ((U1 + sms - 1) / sms));
@@ -2700,8 +2706,8 @@ bool allow_max_smem(size_t need) {
 
 using TmKernel = void (*)(const TmParams, const CUtensorMap);
 
-// The kernel variant for a plan: the balanced-schedule variants (SK) exist for stride 1 only,
-// where the planner takes that schedule.
+// The kernel variant for a plan: the balanced-schedule variants (SK) exist where the planner
+// takes that schedule: stride 1, and stride 2 with two filter groups per warp.
 template <int S, typename T, bool SORT, int SHIFT>
 TmKernel pick_tm(bool sk, size_t smem, bool* ok, int dg = 1) {
     if constexpr (S == 1) {
