@@ -47,7 +47,21 @@ def _check(layer, shape, ws):
     assert pl["lane_sort"] in (0, 1) and (layer.stride == 1 or pl["lane_sort"] == 0)
     assert pl["shift"] in (0, 1, 2) and (layer.stride == 1 or pl["shift"] == 0)
     assert pl["streamk"] in (0, 1)
+    # bands (several images, fewer block rows than an image): full-width rows of block rows that
+    # divide the image's, within the lanes, only for inputs through TMA (fp32 rows of a multiple
+    # of 4) and below 6 kept kernels per (input channel, filter group)
+    ho, wo = (shape[2] - 1) // layer.stride + 1, (shape[3] - 1) // layer.stride + 1
+    nby = (ho + 3) // 4
+    if pl["tile_nb"] > 1 and pl["tile_by"] < nby:
+        BANDS_SEEN.append(shape)
+        assert pl["tile_bx"] == _nbx(pl, wo) and nby % pl["tile_by"] == 0
+        assert pl["tile_by"] * pl["tile_bx"] * pl["tile_nb"] <= 32 * pl["spatial_warps"]
+        assert shape[3] % 4 == 0
+        assert layer.beta / (-(-layer.cout // 8) * shape[1]) < 6
     return pl
+
+
+BANDS_SEEN = []
 
 
 def _nbx(pl, wo):
@@ -184,11 +198,13 @@ def test_random_shapes(seed):
 def test_workload_plans(which):
     layers = WL.vgg16() if which == "vgg16" else WL.resnet50_3x3()
     n = 32 if which == "vgg16" else 64
+    before = len(BANDS_SEEN)
     for L in layers:
         layer = api.pp_pack(WL.weights(L), None, L.keep, 1, L.stride)
         shape = (n, L.cin, L.h, L.w)
         for ws in (0, layer.workspace_bytes(shape), 1 << 20):
             _check(layer, shape, ws)
+    assert len(BANDS_SEEN) > before       # the 28x28 (and ResNet-50's 56x56) layers take bands
 
 
 def test_other_paths_report_no_plan():
