@@ -2463,8 +2463,11 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
         double steps = (double)waves * (std::min(pl->c_split, C) + 2.0 * per + 2.0 * ck);
         // tiny launches (the SMs stay idle even with 8 splits): fewer channels per stage and up to
         // 32 splits within one wave (more cost more in partial sums than they save: measured on the
-        // 64->64 32x32 N=1 layer and the sweep's N=1 points), chosen by estimated channel steps
-        if (pl->ctas * std::min(8, nck_total) < sms) {
+        // 64->64 32x32 N=1 layer and the sweep's N=1 points), chosen by estimated channel steps.
+        // Not below 16 input channels: there every split writes and reads back an output-sized
+        // plane of partial sums for a channel or two of work (VGG-16 layer 1 at batch 1, 3 input
+        // channels: 25.9 us split 3 ways, 14.0 us whole)
+        if (pl->ctas * std::min(8, nck_total) < sms && C >= 16) {
             for (int ck2 = ck;; ck2 = std::max(1, ck2 / 2)) {
                 const int nck2 = (C + ck2 - 1) / ck2;
                 if (nck2 > kMaxChunks) break;
@@ -2641,24 +2644,86 @@ int make_plan(const pp_layer* L, int N, int H, int W, size_t ws_avail, Plan* out
     return PP_OK;
 }
 
-// Sum the KS partial planes in split order, + bias, ReLU, round to the output type.
+// Sum the KS partial planes in split order, + bias, ReLU, round to the output type.  A thread
+// issues the loads of 8 splits before it adds them, so that many loads are in flight; with
+// `quads` (large outputs, a multiple of 4 elements, 16-byte aligned workspace) it takes 4
+// consecutive elements, one 16-byte load per split.  Each element is still summed in split order
+// (the result is that of a plain loop over the splits).
 template <typename T>
 __global__ void splitk_reduce(const float* __restrict__ ws, T* __restrict__ y, const float* __restrict__ bias,
-                              int KS, size_t stride, int Cout, int HoWo, int relu) {
+                              int KS, size_t stride, int Cout, int HoWo, int relu, int quads) {
     pdl_trigger();
     pdl_wait();
-    const size_t total = stride;
-    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total; i += (size_t)gridDim.x * blockDim.x) {
-        float a = ws[i];
-        for (int k = 1; k < KS; ++k) a += ws[(size_t)k * stride + i];
-        const int co = (int)((i / (size_t)HoWo) % (size_t)Cout);
-        a += bias ? bias[co] : 0.0f;
-        y[i] = from_f32<T>(relu ? fmaxf(a, 0.0f) : a);
+    const bool vec = quads != 0;
+    const size_t n = vec ? stride / 4 : stride;
+    for (size_t q = blockIdx.x * (size_t)blockDim.x + threadIdx.x; q < n; q += (size_t)gridDim.x * blockDim.x) {
+        float v[4];
+        int ne;
+        size_t i0;
+        if (vec) {
+            const float4* w4 = reinterpret_cast<const float4*>(ws) + q;
+            const size_t s4 = stride / 4;
+            float4 a = w4[0];
+            int k = 1;
+            for (; k + 8 <= KS; k += 8) {
+                float4 t[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) t[j] = w4[(size_t)(k + j) * s4];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    a.x += t[j].x;
+                    a.y += t[j].y;
+                    a.z += t[j].z;
+                    a.w += t[j].w;
+                }
+            }
+            for (; k < KS; ++k) {
+                const float4 t = w4[(size_t)k * s4];
+                a.x += t.x;
+                a.y += t.y;
+                a.z += t.z;
+                a.w += t.w;
+            }
+            v[0] = a.x;
+            v[1] = a.y;
+            v[2] = a.z;
+            v[3] = a.w;
+            ne = 4;
+            i0 = 4 * q;
+        } else {
+            float a = ws[q];
+            int k = 1;
+            for (; k + 8 <= KS; k += 8) {
+                float t[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) t[j] = ws[(size_t)(k + j) * stride + q];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) a += t[j];
+            }
+            for (; k < KS; ++k) a += ws[(size_t)k * stride + q];
+            v[0] = a;
+            ne = 1;
+            i0 = q;
+        }
+        // output channel of the first element; the next ones may cross into the next plane
+        int rem = (int)(i0 % (size_t)HoWo);
+        int co = (int)((i0 / (size_t)HoWo) % (size_t)Cout);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            if (e >= ne) break;
+            const float r = v[e] + (bias ? bias[co] : 0.0f);
+            y[i0 + e] = from_f32<T>(relu ? fmaxf(r, 0.0f) : r);
+            if (++rem == HoWo) {
+                rem = 0;
+                co = co + 1 == Cout ? 0 : co + 1;
+            }
+        }
     }
 }
 
 // Split-K reduction with the fused 2x2/2 max-pool: each pooled output sums the KS partial planes
-// at its four positions (split order), takes the maximum, adds the bias and applies ReLU.
+// at its four positions (split order), takes the maximum, adds the bias and applies ReLU.  The
+// loads of 4 splits (16 loads) are issued before they are added.
 template <typename T>
 __global__ void splitk_reduce_pool(const float* __restrict__ ws, T* __restrict__ y, const float* __restrict__ bias,
                                    int KS, size_t stride, int Cout, int Ho, int Wo, int relu) {
@@ -2672,13 +2737,25 @@ __global__ void splitk_reduce_pool(const float* __restrict__ ws, T* __restrict__
         const int py = (int)(r % Hp);
         const size_t plane = r / Hp;                       // n * Cout + co
         const size_t base = (plane * Ho + 2 * py) * Wo + 2 * px;
-        float q[4];
         const size_t off[4] = {0, 1, (size_t)Wo, (size_t)Wo + 1};
+        float q[4];
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            float a = ws[base + off[j]];
-            for (int k = 1; k < KS; ++k) a += ws[(size_t)k * stride + base + off[j]];
-            q[j] = a;
+        for (int j = 0; j < 4; ++j) q[j] = ws[base + off[j]];
+        int k = 1;
+        for (; k + 4 <= KS; k += 4) {
+            float t[4][4];
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) t[kk][j] = ws[(size_t)(k + kk) * stride + base + off[j]];
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) q[j] += t[kk][j];
+        }
+        for (; k < KS; ++k) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) q[j] += ws[(size_t)k * stride + base + off[j]];
         }
         const int co = (int)(plane % (size_t)Cout);
         float a = fmaxf(fmaxf(q[0], q[1]), fmaxf(q[2], q[3])) + (bias ? bias[co] : 0.0f);
@@ -2860,12 +2937,18 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
     if (launch(kern, (unsigned)ctas, kThreadsTM / pl.dg, smem, st, p, tmap) != cudaSuccess) return PP_ERR_CUDA;
     if (pl.KS > 1) {
         const size_t total = p.ws_stride;
-        const unsigned blocks = (unsigned)std::max<size_t>(1, std::min<size_t>((total + 255) / 256, (size_t)sm_count() * 16));
         const float* wsf = p.ws;
+        // threads: pooled outputs, or quads of outputs where the reduction loads 16 bytes a split
+        // and there are enough of them to give every SM 512 threads (smaller outputs take more
+        // threads, one element each: 64x64 32x32 N=1 16.1 us, in quads 16.8 us)
+        const int quads = total % 4 == 0 && reinterpret_cast<uintptr_t>(wsf) % 16 == 0 &&
+                          total / 4 >= (size_t)sm_count() * 512;
+        const size_t items = pool ? total / 4 : (quads ? total / 4 : total);
+        const unsigned blocks = (unsigned)std::max<size_t>(1, std::min<size_t>((items + 255) / 256, (size_t)sm_count() * 16));
         T* yt = static_cast<T*>(y);
         const int ks = pl.KS, cout = L->cout, hw = Ho * Wo;
         const cudaError_t e = pool ? launch(splitk_reduce_pool<T>, blocks, 256, 0, st, wsf, yt, bias, ks, total, cout, Ho, Wo, relu)
-                                   : launch(splitk_reduce<T>, blocks, 256, 0, st, wsf, yt, bias, ks, total, cout, hw, relu);
+                                   : launch(splitk_reduce<T>, blocks, 256, 0, st, wsf, yt, bias, ks, total, cout, hw, relu, quads);
         if (e != cudaSuccess) return PP_ERR_CUDA;
     }
     return PP_OK;

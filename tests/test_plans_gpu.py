@@ -179,6 +179,18 @@ def test_stride2_balanced_schedule():
     assert plan["streamk"] == 1 and plan["groups_per_warp"] == 2 and plan["ctas"] == _sms()
 
 
+@pytest.mark.parametrize("shape", [(5, 64, 1, 13, 13), (5, 64, 3, 13, 11), (24, 96, 1, 7, 7),
+                                   (64, 64, 1, 75, 75), (128, 64, 1, 55, 55)])
+def test_split_reduction_element_counts(shape):
+    """The split reduction takes 4 outputs per thread (16-byte loads of every split) where the
+    output count is a multiple of 4 and large (360 000 and 387 200 here, planes of 5625 and 3025
+    outputs, so quads cross from one output plane into the next and take each element's own
+    bias), else one output per thread (845, 2145 and 1176)."""
+    cout, cin, n, h, w = shape
+    plan, _ = _run(cout, cin, n, h, w, 0.5, "f32", seed=50 + h + n)
+    assert plan["splits"] > 8
+
+
 def test_batch_one_split_32_ways():
     plan, _ = _run(256, 256, 1, 14, 14, 0.25, "f32", seed=5)
     assert plan["splits"] == 32 and plan["shift"] == 1
