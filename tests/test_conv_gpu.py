@@ -571,13 +571,15 @@ def test_balanced_schedule_copy_fallback_whole_images():
 
 
 def test_balanced_schedule_matches_oracle_and_is_deterministic():
-    """VGG-16 layer 9 at batch 32 (the balanced schedule): the same result on every run (the
-    head of a cut unit adds its parts in chunk order), the oracle's within tolerance, and the
-    whole-unit schedule's up to fp32 summation order (the schedule off: no workspace)."""
+    """VGG-16 layer 9 at batch 32 (bands of one block row of 4 images on the balanced schedule):
+    the same result on every run (the head of a cut unit adds its parts in chunk order), the
+    oracle's within tolerance, and the whole-unit schedule's up to fp32 summation order (the
+    schedule off: no workspace)."""
     L = WL.vgg16()[8]
     W, b, x = WL.weights(L), WL.bias(L), WL.layer_input(L, 32)
     lay = api.pp_pack(W, None, L.keep)
-    assert lay.plan(x.shape, lay.workspace_bytes(x.shape))["streamk"] == 1
+    pl = lay.plan(x.shape, lay.workspace_bytes(x.shape))
+    assert pl["streamk"] == 1 and (pl["tile_by"], pl["tile_nb"]) == (1, 4)
     y1, _ = run_gpu(W, x, b, L.keep, ws=True)
     y2, _ = run_gpu(W, x, b, L.keep, ws=True)
     y0, _ = run_gpu(W, x, b, L.keep, ws=False)
