@@ -424,7 +424,8 @@ __global__ void __launch_bounds__(kThreadsTM / DG, 1)
     pconv_tm(const TmParams p, const __grid_constant__ CUtensorMap tmap) {
     constexpr int RY = 4, RX = 4;
     constexpr int NT = kThreadsTM / DG, NWP = kCompute / DG;   // threads, warps of the CTA
-    static_assert(DG == 1 || (S == 2 && !SORT), "two filter groups per warp: the stride-2 kernel");
+    static_assert(DG == 1 || S == 2, "two filter groups per warp: the stride-2 kernel");
+    static_assert(!SORT || (sizeof(TIn) == 4 && (S == 1 || DG == 2)), "lanes by bank group: fp32, stride 2 with two groups");
     static_assert(!SHIFT || S == 1, "shifted blocks are a stride-1 layout");
     static_assert(SHIFT != 2 || sizeof(TIn) == 4, "blocks at 4j - 2 are an fp32 layout");
     extern __shared__ __align__(128) unsigned char smem[];
@@ -542,6 +543,7 @@ __global__ void __launch_bounds__(kThreadsTM / DG, 1)
     int ci = 0, ck = 0;
     int img = 0, by = 0, bx = 0, in_off = 3;
     uint32_t edge = 1;
+    uint32_t srcl = 0;   // stride 2 with blocks dealt by bank group: the lane holding the left block
     bool active = false;
     auto place_lane = [&]() {
         const Unit CU = s_units[ci];
@@ -569,26 +571,33 @@ __global__ void __launch_bounds__(kThreadsTM / DG, 1)
             in_off = active ? img * p.CK * plane + by * RY * S * p.BWb + bx * RX * S + d : d;
         };
         locate(blk);
+        int src = lane;
         if constexpr (SORT) {
-            static_assert(S == 1 && sizeof(TIn) == 4, "bank groups are those of fp32 stride-1 windows");
             // The warp's 32 blocks are dealt to its lanes so that each 8-lane phase of the
             // 16-byte window loads (window columns 1-4 at in_off + 1, 2-5 at in_off + 2 with
-            // SHIFT 1, -1..2 and 3..6 at in_off and in_off + 4 with SHIFT 2) meets distinct bank
-            // groups where the blocks allow it: blocks are ordered by (rank among the blocks of
-            // their bank group, bank group) and lane i takes the i-th.  Rows of 7 or 14 blocks
-            // otherwise put two blocks of a phase on one bank group.  Idle lanes go last.  The
-            // planner picks this instance where it lowers the wavefronts (window_wavefronts).
+            // SHIFT 1, -1..2 and 3..6 at in_off and in_off + 4 with SHIFT 2; at stride 2 columns
+            // 1-4 at in_off + 1 and 5-8 one group further) meets distinct bank groups where the
+            // blocks allow it: blocks are ordered by (rank among the blocks of their bank group,
+            // bank group) and lane i takes the i-th.  Rows of 7 or 14 blocks (stride 1), or the
+            // blocks of one row 32 bytes apart (stride 2: every other group), otherwise put two
+            // blocks of a phase on one bank group.  Idle lanes go last.  The planner picks this
+            // instance where it lowers the wavefronts (window_wavefronts).
             const int grp = active ? ((in_off + (SHIFT == 0 ? 1 : SHIFT == 1 ? 2 : 0)) >> 2) & 7 : 8;
             const unsigned same = __match_any_sync(0xffffffffu, grp);
             const int key = active ? 16 * __popc(same & ((1u << lane) - 1u)) + grp : 1024 + lane;   // distinct
-            int pos = 0, src = 0;
+            int pos = 0;
+            src = 0;
             for (int i = 0; i < 32; ++i) pos += __shfl_sync(0xffffffffu, key, i) < key ? 1 : 0;
             for (int i = 0; i < 32; ++i) src = __shfl_sync(0xffffffffu, pos, i) == lane ? i : src;
             locate(ws * 32 + src);
+            if constexpr (S == 2) {   // the lane holding the block to the left (raster src - 1)
+                srcl = lane;
+                for (int i = 0; i < 32; ++i) srcl = __shfl_sync(0xffffffffu, src, i) == src - 1 ? i : srcl;
+            }
         }
-        // lanes whose left neighbour lane does not hold the block to their left (stride 2 takes
-        // window column 0 from that neighbour)
-        edge = (bx == 0 || lane == 0) ? 1u : 0u;
+        // lanes whose left block is not held by the lane they take window column 0 from (stride 2
+        // takes it by shuffle): the first block of a row or of the warp's range
+        edge = (bx == 0 || src == 0) ? 1u : 0u;
     };
     place_lane();
 
@@ -766,8 +775,13 @@ __global__ void __launch_bounds__(kThreadsTM / DG, 1)
                 const uint32_t desc_b = desc_addr + 8u * p.CK, vals_b = vals_addr + 16u * p.maxk;
                 const uint32_t valid_b = CU.g0 + wg * DG + 1 < p.G ? 1u : 0u;
                 if constexpr (es == 4) {
-                    PP_STAGE_KERNELS_S2_G2(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw, edge,
-                                           desc_b, vals_b, valid_b);
+                    if constexpr (SORT) {
+                        PP_STAGE_KERNELS_S2_G2D(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw,
+                                                edge, desc_b, vals_b, valid_b, srcl);
+                    } else {
+                        PP_STAGE_KERNELS_S2_G2(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw, edge,
+                                               desc_b, vals_b, valid_b);
+                    }
                 } else {
                     PP_STAGE_KERNELS_S2_H_G2(ckv, desc_addr, vals_addr, win_addr, es * p.BWb, es * plane, tw, edge,
                                              desc_b, vals_b, valid_b);
@@ -2322,7 +2336,7 @@ std::vector<TileChoice> tile_candidates(int N, int Ho, int Wo, int S, int lanes,
 // fp32 stride-1 stage) in tile t: four phases of 8 lanes, each costing the largest number of its
 // lanes whose loads fall on one bank group (16 bytes = 4 banks; 8 groups).  Lanes take the tile's
 // blocks in raster order, or dealt by bank group as pconv_tm does with lane_sort.
-int window_wavefronts(const Plan& pl, int N, long long t, bool sorted) {
+int window_wavefronts(const Plan& pl, int N, long long t, bool sorted, int S = 1) {
     const TileChoice& tc = pl.tile;
     const int lanes_t = 32 * pl.WS, bpi = tc.BY * tc.BX, plane = tc.IH * tc.BWb;
     int grp[32], key[32], order[32];
@@ -2341,7 +2355,7 @@ int window_wavefronts(const Plan& pl, int N, long long t, bool sorted) {
             active = img < tc.NB;
         }
         const int by = rem / tc.BX, bx = rem - by * tc.BX;
-        const long long off = (long long)img * pl.CK * plane + (long long)by * 4 * tc.BWb + bx * 4;
+        const long long off = (long long)img * pl.CK * plane + (long long)by * 4 * S * tc.BWb + bx * 4 * S;
         grp[l] = active ? (int)((off / 4) & 7) : 8;
     }
     for (int l = 0; l < 32; ++l) {
@@ -2428,7 +2442,7 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
             const long long nt = t.linear ? std::min<long long>(tn, 64) : 1;
             long long w = 0;
             for (long long i = 0; i < nt; ++i)
-                w += std::min(window_wavefronts(q, N, i, false), window_wavefronts(q, N, i, true));
+                w += std::min(window_wavefronts(q, N, i, false, S), window_wavefronts(q, N, i, true, S));
             return w;
         };
         if (S == 1 && t.NB > 1 && ck > 1 && ((size_t)ck * t.IH * t.BWb) % 32 == 0 &&
@@ -2436,6 +2450,27 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
             --ck;
             pl->maxk = maxk_for(ck);
             pl->smem = layout(ck, pl->maxk, &pl->stage_bytes, &pl->kb_bytes);
+        }
+        // stride 2 (fp32, two filter groups per warp): a row's blocks sit 32 bytes apart, on every
+        // other 16-byte bank group, so only blocks of other images can fill a phase's other groups;
+        // an image stride of an odd number of groups lets the blocks dealt by bank group do that.
+        // Up to three channels less per stage where the modelled wavefronts fall
+        if (S == 2 && es == 4 && wg >= 2 && s2_two_groups() && t.NB > 1 && !t.linear) {
+            int best = ck;
+            long long bw = wavefronts_for(ck);
+            for (int c = ck - 1; c >= std::max(1, ck - 3); --c) {
+                if ((C + c - 1) / c > kMaxChunks) break;
+                const long long w = wavefronts_for(c);
+                if (w < bw) {
+                    bw = w;
+                    best = c;
+                }
+            }
+            if (best != ck) {
+                ck = best;
+                pl->maxk = maxk_for(ck);
+                pl->smem = layout(ck, pl->maxk, &pl->stage_bytes, &pl->kb_bytes);
+            }
         }
         pl->CK = ck;
         pl->maxk = std::max(pl->maxk, 1);
@@ -2586,12 +2621,14 @@ int make_plan_uncached(const pp_layer* L, int N, int H, int W, size_t ws_avail, 
     *out = cl < cr ? pli : pr;
     out->shift = shift;
     *cost = std::min(cl, cr);
-    if (S == 1) {   // the bank-group order where it lowers the window loads' wavefronts
+    // the bank-group order where it lowers the window loads' wavefronts (stride 2: fp32 with two
+    // filter groups per warp)
+    if (S == 1 || (es == 4 && out->WG >= 2 && s2_two_groups())) {
         const long long nt = out->tile.linear ? std::min<long long>(out->tiles_n, 64) : 1;
         long long raster = 0, sorted = 0;
         for (long long t = 0; t < nt; ++t) {
-            raster += window_wavefronts(*out, N, t, false);
-            sorted += window_wavefronts(*out, N, t, true);
+            raster += window_wavefronts(*out, N, t, false, S);
+            sorted += window_wavefronts(*out, N, t, true, S);
         }
         out->lane_sort = sorted < raster ? 1 : 0;
     }
@@ -2801,9 +2838,17 @@ TmKernel pick_tm(bool sk, size_t smem, bool* ok, int dg = 1) {
             *ok = allow_max_smem<S, T, SORT, SHIFT, false, 2>(smem);
             return pconv_tm<S, T, SORT, SHIFT, false, 2>;
         }
+        if constexpr (SORT) {   // stride 2 deals blocks by bank group only with two groups per warp
+            *ok = false;
+            return nullptr;
+        }
     }
-    *ok = allow_max_smem<S, T, SORT, SHIFT, false>(smem);
-    return pconv_tm<S, T, SORT, SHIFT, false>;
+    if constexpr (S == 1 || !SORT) {
+        *ok = allow_max_smem<S, T, SORT, SHIFT, false>(smem);
+        return pconv_tm<S, T, SORT, SHIFT, false>;
+    }
+    *ok = false;
+    return nullptr;
 }
 
 template <int S, typename T>
@@ -2910,7 +2955,12 @@ int launch_tm(const pp_layer* L, const void* x, void* y, const float* bias, int 
         if (pl.shift) kern = pick_tm<1, T, false, 1>(sk, smem, &smem_ok);
         else kern = pick_tm<1, T, false, 0>(sk, smem, &smem_ok);
     } else {
-        kern = pick_tm<S, T, false, 0>(sk && pl.dg == 2, smem, &smem_ok, pl.dg);
+        if constexpr (sizeof(T) == 4) {
+            if (pl.lane_sort && pl.dg == 2) kern = pick_tm<S, float, true, 0>(sk, smem, &smem_ok, 2);
+            else kern = pick_tm<S, T, false, 0>(sk && pl.dg == 2, smem, &smem_ok, pl.dg);
+        } else {
+            kern = pick_tm<S, T, false, 0>(sk && pl.dg == 2, smem, &smem_ok, pl.dg);
+        }
     }
     if (!smem_ok) return PP_ERR_CUDA;
     const long long units = pl.ctas * pl.KS;

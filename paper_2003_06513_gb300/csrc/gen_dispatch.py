@@ -59,7 +59,7 @@ def taps(mask):
     return [t for t in range(9) if (mask >> t) & 1]
 
 
-def macro(S, half=False, shift=0, groups=1):
+def macro(S, half=False, shift=0, groups=1, dealt=False):
     RY = RX = 4
     WY, WX = (RY - 1) * S + 3, (RX - 1) * S + 3
     R = RY * RX
@@ -134,7 +134,10 @@ def macro(S, half=False, shift=0, groups=1):
         if S == 2:
             L.append(f"ld.shared.v4.f32 {{x{base + 1}, x{base + 2}, x{base + 3}, x{base + 4}}}, [rb{r}+4];")
             L.append(f"ld.shared.v4.f32 {{x{base + 5}, x{base + 6}, x{base + 7}, x{base + 8}}}, [rb{r}+20];")
-            L.append(f"shfl.sync.up.b32 x{base}, x{base + 8}, 1, 0, -1;")
+            if dealt:   # blocks dealt to lanes by bank group: the left block's lane is %11
+                L.append(f"shfl.sync.idx.b32 x{base}, x{base + 8}, %11, 31, -1;")
+            else:
+                L.append(f"shfl.sync.up.b32 x{base}, x{base + 8}, 1, 0, -1;")
             L.append(f"@EL ld.shared.f32 x{base}, [rb{r}];")
             continue
         if half and aligned:                 # columns 0-1 (4 bytes), columns 2-5 (8 bytes)
@@ -261,14 +264,17 @@ def macro(S, half=False, shift=0, groups=1):
     tag = {0: "", 1: "A", 2: "B"}[shift]
     name = f"PP_STAGE_KERNELS_S{S}" + ("_H" if half else "") + ((tag if half else "_" + tag) if tag else "")
     if groups == 2:
-        name += "_G2"
-        what_g = ", two filter groups per warp"
+        name += "_G2" + ("D" if dealt else "")
+        what_g = ", two filter groups per warp" + (", blocks dealt to lanes by bank group" if dealt else "")
     else:
         what_g = ""
     where = {0: "", 1: ", window column 0 at 2 mod 4", 2: ", window column 0 at 1 mod 4"}[shift]
     what = f"stride {S}{', fp16 stage' if half else ''}{where}{what_g}"
     extra_args = ", desc_b, vals_b, valid_b" if groups == 2 else ""
     extra_ops = ', "r"(desc_b), "r"(vals_b), "r"(valid_b)' if groups == 2 else ""
+    if dealt:
+        extra_args += ", srcl"
+        extra_ops += ', "r"(srcl)'
     return (f"// {what}: 4x4 outputs per lane, {WY}x{WX} input window\n"
             f"#define {name}(nch, desc_addr, vals_addr, win_addr, pitch_b, plane_b, tbase, edge{extra_args}) \\\n"
             f'    asm volatile("{body}" :: "r"(nch), "r"(desc_addr), "r"(vals_addr), "r"(win_addr), '
@@ -283,6 +289,8 @@ def generate() -> str:
             text.append(macro(S, half))
             if S == 2:
                 text.append(macro(S, half, groups=2))
+                if not half:
+                    text.append(macro(S, half, groups=2, dealt=True))
             if S == 1:
                 text.append(macro(S, half, shift=1))
                 if not half:

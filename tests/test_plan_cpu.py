@@ -44,7 +44,8 @@ def _check(layer, shape, ws):
     # units: tiles x filter chunks x splits; persistent CTAs never exceed the units
     assert pl["units"] % pl["splits"] == 0
     assert pl["ctas"] <= pl["units"] or pl["streamk"]
-    assert pl["lane_sort"] in (0, 1) and (layer.stride == 1 or pl["lane_sort"] == 0)
+    # lanes by bank group: stride 1, or stride 2 with two filter groups per warp
+    assert pl["lane_sort"] in (0, 1) and (layer.stride == 1 or pl["lane_sort"] == 0 or pl["groups_per_warp"] == 2)
     assert pl["shift"] in (0, 1, 2) and (layer.stride == 1 or pl["shift"] == 0)
     assert pl["streamk"] in (0, 1)
     # bands (several images, fewer block rows than an image): full-width rows of block rows that
@@ -95,7 +96,8 @@ def _is_linear(pl, shape, stride):
 def _window_wavefronts(pl, shape, stride, t, dealt):
     """Wavefronts of warp 0's 16-byte window loads in tile t: 4 phases of 8 lanes, each costing
     the most lanes on one of the 8 bank groups; lanes in raster order or dealt by
-    (rank within bank group, bank group) with idle lanes last."""
+    (rank within bank group, bank group) with idle lanes last.  A block's window starts 4 * stride
+    elements right of its left neighbour's and 4 * stride rows below the block above."""
     n = shape[0]
     by_t, bx_t, nb = pl["tile_by"], pl["tile_bx"], pl["tile_nb"]
     lanes = 32 * pl["spatial_warps"]
@@ -110,7 +112,7 @@ def _window_wavefronts(pl, shape, stride, t, dealt):
         else:
             img, rem = divmod(lane, by_t * bx_t)
             active = img < nb
-        off = img * pl["channels_per_stage"] * ih * bw + (rem // bx_t) * 4 * bw + (rem % bx_t) * 4
+        off = img * pl["channels_per_stage"] * ih * bw + (rem // bx_t) * 4 * stride * bw + (rem % bx_t) * 4 * stride
         grp.append((off // 4) % 8 if active else None)
     order = list(range(32))
     if dealt:
@@ -132,8 +134,9 @@ def _window_wavefronts(pl, shape, stride, t, dealt):
 @pytest.mark.parametrize("which", ["vgg16", "resnet50"])
 def test_lane_order_by_bank_group(which):
     """The planner deals blocks to lanes by bank group exactly where that lowers the modelled
-    wavefronts of the window loads (stride 1): on VGG-16 the 56x56 and 28x28 layers (rows of 14
-    and 7 blocks), not the 224, 112 or 14 ones."""
+    wavefronts of the window loads (stride 1, and stride 2 with two filter groups per warp): on
+    VGG-16 the 56x56 layers (rows of 14 blocks), not the others; on ResNet-50 the stride-2 heads
+    (a row's blocks 32 bytes apart, on every other bank group; images in between on the others)."""
     layers = WL.vgg16() if which == "vgg16" else WL.resnet50_3x3()
     n = 32 if which == "vgg16" else 64
     got = {}
@@ -142,19 +145,21 @@ def test_lane_order_by_bank_group(which):
         shape = (n, L.cin, L.h, L.w)
         pl = layer.plan(shape, layer.workspace_bytes(shape))
         got[L.name] = pl["lane_sort"]
-        if L.stride != 1:
+        if L.stride != 1 and pl["groups_per_warp"] != 2:
             assert pl["lane_sort"] == 0
             continue
         tiles = 1
         ho, wo = L.ho, L.wo
         nby, nbx = (ho + 3) // 4, _nbx(pl, wo)
-        if pl["tile_by"] == nby and pl["tile_bx"] == nbx and pl["tile_nb"] > 1:
+        if _is_linear(pl, shape, L.stride):
             tiles = min(64, (n * nby * nbx + 31) // 32)
-        raster = sum(_window_wavefronts(pl, shape, 1, t, False) for t in range(tiles))
-        dealt = sum(_window_wavefronts(pl, shape, 1, t, True) for t in range(tiles))
+        raster = sum(_window_wavefronts(pl, shape, L.stride, t, False) for t in range(tiles))
+        dealt = sum(_window_wavefronts(pl, shape, L.stride, t, True) for t in range(tiles))
         assert pl["lane_sort"] == (1 if dealt < raster else 0), (L.name, raster, dealt)
     if which == "vgg16":
         assert [got[f"vgg{i}"] for i in range(1, 14)] == [0, 0, 0, 0, 1, 1, 1, 0, 0, 0, 0, 0, 0]
+    else:   # the stride-2 heads: several images a tile, an odd image stride in bank groups
+        assert [got[L.name] for L in layers if L.stride == 2] == [1, 1, 1]
 
 
 def test_multi_image_stages_are_not_bank_aligned():

@@ -212,8 +212,12 @@ def test_fp16_through_tma(pool):
 
 @pytest.mark.parametrize("io", ["f32", "f16"])
 def test_stride2_heads(io):
+    """Stride 2 with two filter groups per warp over bands of 4 images: fp32 deals each warp's
+    blocks to lanes by shared-memory bank group (window column 0 from the left block's lane by an
+    indexed shuffle); fp16 keeps the raster order."""
     plan, _ = _run(128, 128, 16, 56, 56, 0.4, io, stride=2, seed=8)
-    assert plan["shift"] == 0 and plan["lane_sort"] == 0
+    assert plan["shift"] == 0 and plan["groups_per_warp"] == 2 and plan["tile_nb"] > 1
+    assert plan["lane_sort"] == (1 if io == "f32" else 0)
 
 
 # the single-layer sweep (C = Cin = Cout, H = W, batch, keep, io) at full batch
